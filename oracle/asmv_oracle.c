@@ -1,0 +1,545 @@
+/*
+ * asmv_oracle.c -- the CPU oracle for the differential-oracle hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference legs of bench.py may load this library.  The
+ * product path (the CUDA library) never calls it and shares no code with it:
+ * no header, constant, table or helper is common to the two.
+ *
+ * What it computes, in the paper's terms (AsmEvo, Sec. 3.2 Eq. 1 and
+ * Sec. 3.4 "Tier 1" / "Tier 2"):
+ *   - Tier 1 guarded input synthesis: every allocation is a low guard band,
+ *     a payload and a high guard band; the payload receives deterministic
+ *     seeded values, the guard bands a canary byte, so that an out-of-bounds
+ *     write shows up as a changed guard byte (Sec. 3.4, Tier 1).
+ *   - The equivalence check of Eq. 1 restated per element: floating-point
+ *     outputs pass a tolerance test, integer buffers, opaque state and guard
+ *     bytes must be bit-exact (the iota term of Eq. 1; Sec. 3.4, Tier 2).
+ *     Per region it reports the mismatch count, first mismatching index, the
+ *     exact fp64 maximum absolute and relative error over finite pairs and
+ *     the count of NaN/Inf-position mismatches.
+ *
+ * Everything is a plain scalar loop.  Floating point follows the stated
+ * operation order with -ffp-contract=off; no fast-math.
+ *
+ * Readings where the paper is silent (each one is also listed in the design
+ * notes):
+ *   R1 The random source is Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11,
+ *      "Parallel random numbers: as easy as 1, 2, 3").  key = (seed lo, seed
+ *      hi); counter = (block lo, block hi, region_id, stream tag 0).
+ *   R2 Element generation from Philox words, per distribution (see fill).
+ *   R3 Normal values use Box-Muller in fp32 with in-house ln / sincos(2 pi u)
+ *      routines, so that CPU and GPU produce identical bytes.
+ *   R4 Float predicate: d = |c - r| in fp64 (exact inputs), bound =
+ *      atol + rtol*|r| (multiply, then add), mismatch iff d > bound; both NaN
+ *      match, same-signed Inf match, any other non-finite pair mismatches and
+ *      counts as a NaN/Inf-position mismatch and is excluded from the maxima.
+ *   R5 rel = d / |r|; for r == 0 it is 0 when d == 0, else +Inf.
+ *   R6 Integer and opaque regions: mismatch iff the bits differ; abs error is
+ *      |int(c) - int(r)| and rel error abs/|r| (same r == 0 rule).
+ *   R7 first_mismatch is the lowest element index; first_guard_bad the lowest
+ *      byte offset from the allocation start (low guard before high guard).
+ *
+ * Parity pins live in tests/test_oracle_*.py.  The stats of the large
+ * perturbed workloads (attention outputs, the 4096-region snapshot, the
+ * batched GEMM output) are data-determined: beyond invariants, parity of
+ * those totals is unpinned, and the oracle's value is the reference.
+ */
+#include <stdint.h>
+#include <string.h>
+#include <math.h>
+#include <float.h>
+
+/* ---- dtype and distribution codes (the numbering of the public ABI) ---- */
+enum { OD_F32 = 0, OD_BF16 = 1, OD_F16 = 2, OD_F8E4M3 = 3, OD_I32 = 4,
+       OD_I8 = 5, OD_U8 = 6, OD_NDTYPES = 7 };
+enum { OX_RAW = 0, OX_UNIFORM = 1, OX_NORMAL = 2, OX_INT_RANGE = 3,
+       OX_NONE = 4 };
+
+int oracle_dtype_size(int dt) {
+  switch (dt) {
+    case OD_F32: case OD_I32: return 4;
+    case OD_BF16: case OD_F16: return 2;
+    case OD_F8E4M3: case OD_I8: case OD_U8: return 1;
+    default: return 0;
+  }
+}
+
+static int is_float_dtype(int dt) { return dt <= OD_F8E4M3; }
+
+/* ======================================================================
+ * Philox4x32-10, written from Salmon et al. (SC'11), Sec. 3 / Table 2:
+ * with Ma = 0xD2511F53 and Mb = 0xCD9E8D57, one round maps (x0,x1,x2,x3)
+ * under key (k0,k1) to
+ *   (hi(Mb*x2) ^ x1 ^ k0,  lo(Mb*x2),  hi(Ma*x0) ^ x3 ^ k1,  lo(Ma*x0))
+ * where hi/lo are the halves of the 64-bit product.  Ten rounds; the key
+ * advances by the Weyl constants (golden ratio and sqrt(3)-1 in 0.32 fixed
+ * point) between consecutive rounds.
+ * ====================================================================== */
+#define PHILOX_M_A 0xD2511F53u
+#define PHILOX_M_B 0xCD9E8D57u
+#define PHILOX_W_0 0x9E3779B9u
+#define PHILOX_W_1 0xBB67AE85u
+
+void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2],
+                          uint32_t out[4]) {
+  uint32_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+  uint32_t k0 = key[0], k1 = key[1];
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) { k0 += PHILOX_W_0; k1 += PHILOX_W_1; }
+    uint64_t pa = (uint64_t)PHILOX_M_A * (uint64_t)x0;
+    uint64_t pb = (uint64_t)PHILOX_M_B * (uint64_t)x2;
+    uint32_t pa_hi = (uint32_t)(pa >> 32), pa_lo = (uint32_t)pa;
+    uint32_t pb_hi = (uint32_t)(pb >> 32), pb_lo = (uint32_t)pb;
+    uint32_t y0 = pb_hi ^ x1 ^ k0;
+    uint32_t y1 = pb_lo;
+    uint32_t y2 = pa_hi ^ x3 ^ k1;
+    uint32_t y3 = pa_lo;
+    x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+  }
+  out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/* The block b of region `region_id` under `seed` (stream tag 0 = payload). */
+static void payload_block(uint64_t seed, uint32_t region_id, uint64_t b,
+                          uint32_t w[4]) {
+  uint32_t ctr[4] = {(uint32_t)b, (uint32_t)(b >> 32), region_id, 0u};
+  uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  oracle_philox4x32_10(ctr, key, w);
+}
+
+/* ======================================================================
+ * Exact decoders of the stored formats to fp64 (all are exact in fp64).
+ * ====================================================================== */
+static uint32_t f32_bits(float f) { uint32_t u; memcpy(&u, &f, 4); return u; }
+static float bits_f32(uint32_t u) { float f; memcpy(&f, &u, 4); return f; }
+
+double oracle_decode_bf16(uint16_t h) {
+  return (double)bits_f32((uint32_t)h << 16);
+}
+
+double oracle_decode_f16(uint16_t h) {
+  int sign = (h >> 15) & 1, ex = (h >> 10) & 31, man = h & 1023;
+  double v;
+  if (ex == 31) v = man ? NAN : INFINITY;
+  else if (ex == 0) v = ldexp((double)man, -24);
+  else v = ldexp((double)(1024 + man), ex - 25);
+  return sign ? -v : v;
+}
+
+/* OCP FP8 E4M3 ("fn" variant): bias 7, no infinities, S.1111.111 is NaN. */
+double oracle_decode_f8e4m3(uint8_t b) {
+  int sign = (b >> 7) & 1, ex = (b >> 3) & 15, man = b & 7;
+  double v;
+  if (ex == 15 && man == 7) v = NAN;
+  else if (ex == 0) v = ldexp((double)man, -9);
+  else v = ldexp((double)(8 + man), ex - 10);
+  return sign ? -v : v;
+}
+
+/* Decode element i of a payload of dtype dt to fp64.  Integer types give
+ * their (signed or unsigned) integer value. */
+static double decode_elem(const uint8_t *p, int dt, uint64_t i) {
+  switch (dt) {
+    case OD_F32: { uint32_t u; memcpy(&u, p + 4 * i, 4); return (double)bits_f32(u); }
+    case OD_BF16: { uint16_t h; memcpy(&h, p + 2 * i, 2); return oracle_decode_bf16(h); }
+    case OD_F16: { uint16_t h; memcpy(&h, p + 2 * i, 2); return oracle_decode_f16(h); }
+    case OD_F8E4M3: return oracle_decode_f8e4m3(p[i]);
+    case OD_I32: { int32_t v; memcpy(&v, p + 4 * i, 4); return (double)v; }
+    case OD_I8: return (double)(int8_t)p[i];
+    case OD_U8: return (double)p[i];
+    default: return NAN;
+  }
+}
+
+/* ======================================================================
+ * Round-to-nearest-even encoders from fp32, written on integer bits.
+ * ====================================================================== */
+uint16_t oracle_f32_to_bf16(float f) {
+  uint32_t u = f32_bits(f);
+  if ((u & 0x7FFFFFFFu) > 0x7F800000u) return (uint16_t)((u >> 16) | 0x0040u);
+  uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7FFFu + lsb;                 /* carries into the exponent as needed */
+  return (uint16_t)(u >> 16);
+}
+
+/* Round the positive finite fp32 value with biased exponent field `bexp`
+ * and fraction `frac` to a multiple of 2^qe (RNE); returns the multiplier. */
+static uint32_t rne_to_quantum(uint32_t bexp, uint32_t frac, int qe) {
+  /* value = m24 * 2^(e - 23), e = bexp - 127 (normal) */
+  uint32_t m24;
+  int e;
+  if (bexp == 0) { m24 = frac; e = -126; } else { m24 = frac | 0x800000u; e = (int)bexp - 127; }
+  int shift = qe - (e - 23);          /* bits of m24 below the quantum */
+  if (shift <= 0) return m24 << (-shift);
+  if (shift > 25) return 0;
+  uint32_t q = m24 >> shift;
+  uint32_t rem = m24 & ((1u << shift) - 1u);
+  uint32_t half = 1u << (shift - 1);
+  if (rem > half || (rem == half && (q & 1u))) q += 1;
+  return q;
+}
+
+uint16_t oracle_f32_to_f16(float f) {
+  uint32_t u = f32_bits(f);
+  uint16_t sign = (uint16_t)((u >> 16) & 0x8000u);
+  uint32_t a = u & 0x7FFFFFFFu;
+  if (a > 0x7F800000u) return (uint16_t)(sign | 0x7E00u);
+  if (a == 0x7F800000u) return (uint16_t)(sign | 0x7C00u);
+  uint32_t bexp = a >> 23, frac = a & 0x7FFFFFu;
+  int e = (bexp == 0) ? -126 : (int)bexp - 127;
+  if (e < -25) return sign;                        /* below half the least subnormal */
+  int qe = (e - 10 > -24) ? e - 10 : -24;          /* quantum of binary16 at this magnitude */
+  uint32_t q = rne_to_quantum(bexp, frac, qe);
+  if (qe == -24) return (uint16_t)(sign | q);     /* subnormal, or rounds up to 2^-14 */
+  if (q == 2048) { q = 1024; e += 1; }
+  if (e + 15 >= 31) return (uint16_t)(sign | 0x7C00u);
+  return (uint16_t)(sign | ((uint32_t)(e + 15) << 10) | (q - 1024));
+}
+
+/* fp32 -> OCP E4M3: RNE, finite overflow and infinities saturate to +-448,
+ * NaN maps to S.1111.111. */
+uint8_t oracle_f32_to_f8e4m3(float f) {
+  uint32_t u = f32_bits(f);
+  uint8_t sign = (uint8_t)((u >> 24) & 0x80u);
+  uint32_t a = u & 0x7FFFFFFFu;
+  if (a > 0x7F800000u) return (uint8_t)(sign | 0x7Fu);
+  if (bits_f32(a) >= 448.0f) return (uint8_t)(sign | 0x7Eu);
+  uint32_t bexp = a >> 23, frac = a & 0x7FFFFFu;
+  int e = (bexp == 0) ? -126 : (int)bexp - 127;
+  if (e < -10) return sign;
+  int qe = (e - 3 > -9) ? e - 3 : -9;
+  uint32_t q = rne_to_quantum(bexp, frac, qe);
+  if (qe == -9) return (uint8_t)(sign | q);
+  if (q == 16) { q = 8; e += 1; }
+  return (uint8_t)(sign | ((uint32_t)(e + 7) << 3) | (q - 8));
+}
+
+/* ======================================================================
+ * fp32 Box-Muller pieces.  Coefficients are the Taylor coefficients of the
+ * stated series, computed here in extended precision and rounded once to
+ * fp32; every step below is one IEEE fp32 operation (fmaf where written).
+ * ====================================================================== */
+static float C_LN2_HI, C_LN2_LO, C_AT[5], C_S[5], C_C[6];
+static int consts_ready = 0;
+
+static void init_consts(void) {
+  if (consts_ready) return;
+  long double ln2 = logl(2.0L);
+  /* Cody-Waite split: a short head (9 significant bits) and the rest. */
+  C_LN2_HI = 355.0f / 512.0f;
+  C_LN2_LO = (float)(ln2 - 355.0L / 512.0L);
+  /* atanh series: ln(m) = 2s (1 + s^2/3 + s^4/5 + ...), s = (m-1)/(m+1) */
+  for (int k = 0; k < 5; ++k) C_AT[k] = (float)(1.0L / (long double)(2 * k + 3));
+  /* sin(pi/2 r) and cos(pi/2 r): coefficient of r^j is +-(pi/2)^j / j! */
+  long double h = acosl(-1.0L) / 2.0L, p = 1.0L, fact = 1.0L;
+  long double coef[12];
+  for (int j = 0; j < 12; ++j) {
+    if (j > 0) { p *= h; fact *= (long double)j; }
+    long double c = p / fact;
+    if ((j / 2) % 2 == 1) c = -c;      /* signs: + (j=0,1), - (2,3), + (4,5) ... */
+    coef[j] = c;
+  }
+  for (int k = 0; k < 5; ++k) C_S[k] = (float)coef[2 * k + 1];   /* r^1 .. r^9 */
+  for (int k = 0; k < 6; ++k) C_C[k] = (float)coef[2 * k];       /* r^0 .. r^10 */
+  consts_ready = 1;
+}
+
+void oracle_boxmuller_consts(float out[18]) {
+  init_consts();
+  out[0] = C_LN2_HI; out[1] = C_LN2_LO;
+  for (int k = 0; k < 5; ++k) out[2 + k] = C_AT[k];
+  for (int k = 0; k < 5; ++k) out[7 + k] = C_S[k];
+  for (int k = 0; k < 6; ++k) out[12 + k] = C_C[k];
+}
+
+/* ln(k * 2^-24) for k in [1, 2^24], in fp32. */
+float oracle_ln_u24(uint32_t k) {
+  init_consts();
+  float u = (float)k * 0x1p-24f;                 /* exact */
+  uint32_t b = f32_bits(u);
+  int e = (int)(b >> 23) - 127;
+  float m = bits_f32((b & 0x7FFFFFu) | 0x3F800000u);   /* [1, 2) */
+  if (m > 1.41421356f) { m = m * 0.5f; e += 1; }       /* [sqrt2/2, sqrt2] */
+  float f = m - 1.0f;                              /* exact (Sterbenz) */
+  float s = f / (2.0f + f);
+  float z = s * s;
+  float p = fmaf(z, C_AT[4], C_AT[3]);
+  p = fmaf(z, p, C_AT[2]);
+  p = fmaf(z, p, C_AT[1]);
+  p = fmaf(z, p, C_AT[0]);
+  float s2 = s + s;
+  float lnm = fmaf(s2 * z, p, s2);
+  float ef = (float)e;
+  float r = fmaf(ef, C_LN2_LO, lnm);
+  return fmaf(ef, C_LN2_HI, r);
+}
+
+/* sin and cos of 2*pi*k*2^-24 for k in [0, 2^24), in fp32. */
+void oracle_sincos_2pi_u24(uint32_t k, float *sn_out, float *cs_out) {
+  init_consts();
+  uint32_t q = (k + (1u << 21)) >> 22;             /* nearest quarter turn, 0..4 */
+  int32_t ri = (int32_t)k - (int32_t)(q << 22);    /* [-2^21, 2^21) */
+  float r = (float)ri * 0x1p-22f;                  /* angle = (q + r) * pi/2 */
+  float r2 = r * r;
+  float sp = fmaf(r2, C_S[4], C_S[3]);
+  sp = fmaf(r2, sp, C_S[2]);
+  sp = fmaf(r2, sp, C_S[1]);
+  sp = fmaf(r2, sp, C_S[0]);
+  float sn = r * sp;
+  float cp = fmaf(r2, C_C[5], C_C[4]);
+  cp = fmaf(r2, cp, C_C[3]);
+  cp = fmaf(r2, cp, C_C[2]);
+  cp = fmaf(r2, cp, C_C[1]);
+  float cs = fmaf(r2, cp, C_C[0]);
+  switch (q & 3u) {
+    case 0: *sn_out = sn;  *cs_out = cs;  break;
+    case 1: *sn_out = cs;  *cs_out = -sn; break;
+    case 2: *sn_out = -sn; *cs_out = -cs; break;
+    default: *sn_out = -cs; *cs_out = sn; break;
+  }
+}
+
+/* The two standard normals of Box-Muller from two Philox words. */
+void oracle_boxmuller(uint32_t w0, uint32_t w1, float *z0, float *z1) {
+  float l = oracle_ln_u24((w0 >> 8) + 1u);
+  float rho = sqrtf(-2.0f * l);
+  float sn, cs;
+  oracle_sincos_2pi_u24(w1 >> 8, &sn, &cs);
+  *z0 = rho * cs;
+  *z1 = rho * sn;
+}
+
+/* ======================================================================
+ * Tier 1 fill.
+ * Element i of a payload, per distribution:
+ *   RAW       payload byte j = byte (j mod 16) of block (j div 16); a block
+ *             is its four words in order, each little-endian.
+ *   INT_RANGE word (i mod 4) of block (i div 4): lo + ((w * (hi-lo)) >> 32)
+ *   UNIFORM   word (i mod 4) of block (i div 4): f = (w >> 8) 2^-24,
+ *             v = lo + f*(hi - lo) in fp32, then RNE to the dtype
+ *   NORMAL    block i div 4 gives two pairs (words 0,1 and 2,3); element
+ *             4b+2j+t is z_t of pair j, v = mean + std*z in fp32, then RNE
+ *   NONE      payload untouched
+ * ====================================================================== */
+static void store_float(uint8_t *p, int dt, uint64_t i, float v) {
+  switch (dt) {
+    case OD_F32: { uint32_t u = f32_bits(v); memcpy(p + 4 * i, &u, 4); break; }
+    case OD_BF16: { uint16_t h = oracle_f32_to_bf16(v); memcpy(p + 2 * i, &h, 2); break; }
+    case OD_F16: { uint16_t h = oracle_f32_to_f16(v); memcpy(p + 2 * i, &h, 2); break; }
+    case OD_F8E4M3: p[i] = oracle_f32_to_f8e4m3(v); break;
+  }
+}
+
+static void store_int(uint8_t *p, int dt, uint64_t i, int64_t v) {
+  switch (dt) {
+    case OD_I32: { int32_t x = (int32_t)v; memcpy(p + 4 * i, &x, 4); break; }
+    case OD_I8: case OD_U8: p[i] = (uint8_t)v; break;
+  }
+}
+
+/* Fill elements [i0, i1) of the payload starting at `payload`.  Returns 0,
+ * or -1 for a distribution that does not apply to the dtype. */
+int oracle_fill_payload(uint8_t *payload, int dt, int dist, uint64_t i0,
+                        uint64_t i1, uint32_t region_id, double p0, double p1,
+                        uint64_t seed) {
+  int sz = oracle_dtype_size(dt);
+  if (sz == 0) return -1;
+  if (dist == OX_NONE) return 0;
+  if (dist == OX_RAW) {
+    for (uint64_t j = i0 * (uint64_t)sz; j < i1 * (uint64_t)sz; ++j) {
+      uint32_t w[4];
+      payload_block(seed, region_id, j / 16, w);
+      uint32_t word = w[(j % 16) / 4];
+      payload[j] = (uint8_t)(word >> (8 * (j % 4)));
+    }
+    return 0;
+  }
+  if (dist == OX_INT_RANGE) {
+    if (is_float_dtype(dt)) return -1;
+    int64_t lo = (int64_t)p0, hi = (int64_t)p1;
+    uint64_t span = (uint64_t)(hi - lo);
+    for (uint64_t i = i0; i < i1; ++i) {
+      uint32_t w[4];
+      payload_block(seed, region_id, i / 4, w);
+      uint64_t off = ((uint64_t)w[i % 4] * span) >> 32;
+      store_int(payload, dt, i, lo + (int64_t)off);
+    }
+    return 0;
+  }
+  if (!is_float_dtype(dt)) return -1;
+  if (dist == OX_UNIFORM) {
+    float lo = (float)p0, hi = (float)p1;
+    float width = hi - lo;
+    for (uint64_t i = i0; i < i1; ++i) {
+      uint32_t w[4];
+      payload_block(seed, region_id, i / 4, w);
+      float f = (float)(w[i % 4] >> 8) * 0x1p-24f;
+      float v = lo + f * width;
+      store_float(payload, dt, i, v);
+    }
+    return 0;
+  }
+  if (dist == OX_NORMAL) {
+    float mean = (float)p0, sd = (float)p1;
+    for (uint64_t i = i0; i < i1; ++i) {
+      uint32_t w[4];
+      payload_block(seed, region_id, i / 4, w);
+      unsigned pair = (unsigned)((i % 4) / 2);
+      float z0, z1;
+      oracle_boxmuller(w[2 * pair], w[2 * pair + 1], &z0, &z1);
+      float z = (i % 2 == 0) ? z0 : z1;
+      float v = mean + sd * z;
+      store_float(payload, dt, i, v);
+    }
+    return 0;
+  }
+  return -1;
+}
+
+/* Guard bands: [alloc, alloc+glo) and [alloc+glo+payload_bytes, +ghi). */
+void oracle_fill_guards(uint8_t *alloc, uint64_t payload_bytes, uint32_t glo,
+                        uint32_t ghi, uint8_t canary) {
+  for (uint64_t j = 0; j < glo; ++j) alloc[j] = canary;
+  uint8_t *hi = alloc + glo + payload_bytes;
+  for (uint64_t j = 0; j < ghi; ++j) hi[j] = canary;
+}
+
+/* Count guard bytes differing from the canary; first bad offset from alloc
+ * (UINT64_MAX when none). */
+void oracle_guard_check(const uint8_t *alloc, uint64_t payload_bytes,
+                        uint32_t glo, uint32_t ghi, uint8_t canary,
+                        uint64_t *bad_out, uint64_t *first_out) {
+  uint64_t bad = 0, first = UINT64_MAX;
+  for (uint64_t j = 0; j < glo; ++j)
+    if (alloc[j] != canary) { ++bad; if (first == UINT64_MAX) first = j; }
+  uint64_t base = (uint64_t)glo + payload_bytes;
+  for (uint64_t j = 0; j < ghi; ++j)
+    if (alloc[base + j] != canary) { ++bad; if (first == UINT64_MAX) first = base + j; }
+  *bad_out = bad;
+  *first_out = first;
+}
+
+/* ======================================================================
+ * The per-element equivalence predicate and per-region statistics.
+ * ====================================================================== */
+typedef struct {
+  uint64_t mismatches;
+  uint64_t first_mismatch;
+  double max_abs_err;
+  double max_rel_err;
+  uint64_t nonfinite_mismatches;
+} oracle_stats;
+
+/* Compare elements [i0, i1) of two payloads of dtype dt.  Indices in the
+ * result are absolute element indices. */
+void oracle_compare_range(const uint8_t *ref, const uint8_t *cand, int dt,
+                          uint64_t i0, uint64_t i1, double atol, double rtol,
+                          oracle_stats *out) {
+  oracle_stats st = {0, UINT64_MAX, 0.0, 0.0, 0};
+  int sz = oracle_dtype_size(dt);
+  for (uint64_t i = i0; i < i1; ++i) {
+    int mismatch;
+    double abs_err = 0.0, rel_err = 0.0;
+    int finite_pair = 1;
+    if (!is_float_dtype(dt)) {
+      mismatch = memcmp(ref + (uint64_t)sz * i, cand + (uint64_t)sz * i, (size_t)sz) != 0;
+      double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);
+      abs_err = fabs(c - r);                         /* exact: |c - r| < 2^33 */
+      if (r != 0.0) rel_err = abs_err / fabs(r);
+      else rel_err = (abs_err == 0.0) ? 0.0 : INFINITY;
+    } else {
+      double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);
+      if (isnan(r) || isnan(c) || isinf(r) || isinf(c)) {
+        finite_pair = 0;
+        if (isnan(r) && isnan(c)) mismatch = 0;
+        else if (isinf(r) && isinf(c) && (signbit(r) == signbit(c))) mismatch = 0;
+        else { mismatch = 1; st.nonfinite_mismatches += 1; }
+      } else {
+        double d = fabs(c - r);
+        double bound = atol + rtol * fabs(r);
+        mismatch = d > bound;
+        abs_err = d;
+        if (r != 0.0) rel_err = d / fabs(r);
+        else rel_err = (d == 0.0) ? 0.0 : INFINITY;
+      }
+    }
+    if (mismatch) {
+      st.mismatches += 1;
+      if (st.first_mismatch == UINT64_MAX) st.first_mismatch = i;
+    }
+    if (finite_pair) {
+      if (abs_err > st.max_abs_err) st.max_abs_err = abs_err;
+      if (rel_err > st.max_rel_err) st.max_rel_err = rel_err;
+    }
+  }
+  *out = st;
+}
+
+/* Per-region result in the 8-field layout: mismatches, first_mismatch,
+ * max_abs_err, max_rel_err, nonfinite_mismatches, guard_bad_bytes,
+ * first_guard_bad, ref_guard_bad_bytes. */
+typedef struct {
+  uint64_t mismatches;
+  uint64_t first_mismatch;
+  double max_abs_err;
+  double max_rel_err;
+  uint64_t nonfinite_mismatches;
+  uint64_t guard_bad_bytes;
+  uint64_t first_guard_bad;
+  uint64_t ref_guard_bad_bytes;
+} oracle_region_stats;
+
+void oracle_compare_region(const uint8_t *ref_alloc, uint32_t ref_glo,
+                           uint32_t ref_ghi, uint8_t ref_canary,
+                           const uint8_t *cand_alloc, uint32_t cand_glo,
+                           uint32_t cand_ghi, uint8_t cand_canary,
+                           uint64_t n_elems, int dt, double atol, double rtol,
+                           oracle_region_stats *out) {
+  uint64_t bytes = n_elems * (uint64_t)oracle_dtype_size(dt);
+  oracle_stats st;
+  oracle_compare_range(ref_alloc + ref_glo, cand_alloc + cand_glo, dt, 0,
+                       n_elems, atol, rtol, &st);
+  uint64_t gbad, gfirst, rbad, rfirst;
+  oracle_guard_check(cand_alloc, bytes, cand_glo, cand_ghi, cand_canary, &gbad, &gfirst);
+  oracle_guard_check(ref_alloc, bytes, ref_glo, ref_ghi, ref_canary, &rbad, &rfirst);
+  out->mismatches = st.mismatches;
+  out->first_mismatch = st.first_mismatch;
+  out->max_abs_err = st.max_abs_err;
+  out->max_rel_err = st.max_rel_err;
+  out->nonfinite_mismatches = st.nonfinite_mismatches;
+  out->guard_bad_bytes = gbad;
+  out->first_guard_bad = gfirst;
+  out->ref_guard_bad_bytes = rbad;
+}
+
+/* ======================================================================
+ * Batch entry points for the tests (plain loops over the functions above).
+ * ====================================================================== */
+void oracle_philox_many(const uint32_t *ctr, const uint32_t *key, uint64_t n,
+                        uint32_t *out) {
+  for (uint64_t i = 0; i < n; ++i)
+    oracle_philox4x32_10(ctr + 4 * i, key + 2 * i, out + 4 * i);
+}
+
+void oracle_ln_u24_many(const uint32_t *k, uint64_t n, float *out) {
+  for (uint64_t i = 0; i < n; ++i) out[i] = oracle_ln_u24(k[i]);
+}
+
+void oracle_sincos_2pi_u24_many(const uint32_t *k, uint64_t n, float *sn,
+                                float *cs) {
+  for (uint64_t i = 0; i < n; ++i) oracle_sincos_2pi_u24(k[i], sn + i, cs + i);
+}
+
+void oracle_boxmuller_many(const uint32_t *w0, const uint32_t *w1, uint64_t n,
+                           float *z0, float *z1) {
+  for (uint64_t i = 0; i < n; ++i) oracle_boxmuller(w0[i], w1[i], z0 + i, z1 + i);
+}
+
+void oracle_encode_many(const float *x, uint64_t n, int dt, uint8_t *out) {
+  for (uint64_t i = 0; i < n; ++i) store_float(out, dt, i, x[i]);
+}
+
+void oracle_decode_many(const uint8_t *p, uint64_t n, int dt, double *out) {
+  for (uint64_t i = 0; i < n; ++i) out[i] = decode_elem(p, dt, i);
+}

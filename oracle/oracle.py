@@ -1,0 +1,263 @@
+"""ctypes view of the CPU oracle (test infrastructure only).
+
+Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline and
+reference legs import this module.  It loads oracle/liboracle.so, which
+shares no code with the CUDA library: it is the plain, slow definition of
+the guarded fill and of the per-element equivalence check (AsmEvo, Sec. 3.2
+Eq. 1; Sec. 3.4 Tier 1 and Tier 2), in fp64 where the check is floating
+point.
+
+Arrays are numpy; every call passes raw pointers of C-contiguous arrays.
+"""
+import ctypes
+import os
+import threading
+
+import numpy as np
+
+from . import build as _build
+
+F32, BF16, F16, F8E4M3, I32, I8, U8 = range(7)
+RAW, UNIFORM, NORMAL, INT_RANGE, NONE = range(5)
+DTYPE_SIZE = {F32: 4, BF16: 2, F16: 2, F8E4M3: 1, I32: 4, I8: 1, U8: 1}
+FLOAT_DTYPES = (F32, BF16, F16, F8E4M3)
+U64_NONE = (1 << 64) - 1
+
+_u8p = ctypes.POINTER(ctypes.c_uint8)
+_u32p = ctypes.POINTER(ctypes.c_uint32)
+_f32p = ctypes.POINTER(ctypes.c_float)
+_f64p = ctypes.POINTER(ctypes.c_double)
+_u64p = ctypes.POINTER(ctypes.c_uint64)
+
+
+class _Stats(ctypes.Structure):
+    _fields_ = [("mismatches", ctypes.c_uint64),
+                ("first_mismatch", ctypes.c_uint64),
+                ("max_abs_err", ctypes.c_double),
+                ("max_rel_err", ctypes.c_double),
+                ("nonfinite_mismatches", ctypes.c_uint64)]
+
+
+class _RegionStats(ctypes.Structure):
+    _fields_ = _Stats._fields_ + [("guard_bad_bytes", ctypes.c_uint64),
+                                  ("first_guard_bad", ctypes.c_uint64),
+                                  ("ref_guard_bad_bytes", ctypes.c_uint64)]
+
+
+STATS_FIELDS = [f for f, _ in _RegionStats._fields_]
+
+_lib = None
+_lock = threading.Lock()
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build()
+            L = ctypes.CDLL(path)
+            c = ctypes
+            L.oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
+            L.oracle_philox_many.argtypes = [_u32p, _u32p, c.c_uint64, _u32p]
+            L.oracle_ln_u24_many.argtypes = [_u32p, c.c_uint64, _f32p]
+            L.oracle_sincos_2pi_u24_many.argtypes = [_u32p, c.c_uint64, _f32p, _f32p]
+            L.oracle_boxmuller_many.argtypes = [_u32p, _u32p, c.c_uint64, _f32p, _f32p]
+            L.oracle_boxmuller_consts.argtypes = [_f32p]
+            L.oracle_encode_many.argtypes = [_f32p, c.c_uint64, c.c_int, _u8p]
+            L.oracle_decode_many.argtypes = [_u8p, c.c_uint64, c.c_int, _f64p]
+            L.oracle_fill_payload.argtypes = [_u8p, c.c_int, c.c_int, c.c_uint64,
+                                              c.c_uint64, c.c_uint32, c.c_double,
+                                              c.c_double, c.c_uint64]
+            L.oracle_fill_payload.restype = c.c_int
+            L.oracle_fill_guards.argtypes = [_u8p, c.c_uint64, c.c_uint32,
+                                             c.c_uint32, c.c_uint8]
+            L.oracle_guard_check.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
+                                             c.c_uint8, _u64p, _u64p]
+            L.oracle_compare_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
+                                               c.c_uint64, c.c_double, c.c_double,
+                                               c.POINTER(_Stats)]
+            L.oracle_compare_region.argtypes = [
+                _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
+                _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
+                c.c_uint64, c.c_int, c.c_double, c.c_double,
+                c.POINTER(_RegionStats)]
+            _lib = L
+    return _lib
+
+
+def _ptr(a, t):
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data_as(t)
+
+
+def _bytes_view(a):
+    a = np.ascontiguousarray(a)
+    return a.view(np.uint8).reshape(-1)
+
+
+# ---------------------------------------------------------------- primitives
+def philox(ctr, key):
+    """Philox4x32-10 blocks: ctr (n,4) uint32, key (n,2) uint32 -> (n,4)."""
+    ctr = np.ascontiguousarray(ctr, dtype=np.uint32).reshape(-1, 4)
+    key = np.ascontiguousarray(key, dtype=np.uint32).reshape(-1, 2)
+    assert ctr.shape[0] == key.shape[0]
+    out = np.empty_like(ctr)
+    lib().oracle_philox_many(_ptr(ctr, _u32p), _ptr(key, _u32p), ctr.shape[0],
+                             _ptr(out, _u32p))
+    return out
+
+
+def ln_u24(k):
+    k = np.ascontiguousarray(k, dtype=np.uint32)
+    out = np.empty(k.shape, np.float32)
+    lib().oracle_ln_u24_many(_ptr(k, _u32p), k.size, _ptr(out, _f32p))
+    return out
+
+
+def sincos_2pi_u24(k):
+    k = np.ascontiguousarray(k, dtype=np.uint32)
+    sn = np.empty(k.shape, np.float32)
+    cs = np.empty(k.shape, np.float32)
+    lib().oracle_sincos_2pi_u24_many(_ptr(k, _u32p), k.size, _ptr(sn, _f32p),
+                                     _ptr(cs, _f32p))
+    return sn, cs
+
+
+def boxmuller(w0, w1):
+    w0 = np.ascontiguousarray(w0, dtype=np.uint32)
+    w1 = np.ascontiguousarray(w1, dtype=np.uint32)
+    z0 = np.empty(w0.shape, np.float32)
+    z1 = np.empty(w0.shape, np.float32)
+    lib().oracle_boxmuller_many(_ptr(w0, _u32p), _ptr(w1, _u32p), w0.size,
+                                _ptr(z0, _f32p), _ptr(z1, _f32p))
+    return z0, z1
+
+
+def boxmuller_consts():
+    out = np.empty(18, np.float32)
+    lib().oracle_boxmuller_consts(_ptr(out, _f32p))
+    return out
+
+
+def encode(x, dtype):
+    """fp32 array -> raw bytes of the float dtype (RNE)."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(x.size * DTYPE_SIZE[dtype], np.uint8)
+    lib().oracle_encode_many(_ptr(x, _f32p), x.size, dtype, _ptr(out, _u8p))
+    return out
+
+
+def decode(raw, dtype):
+    """raw bytes -> float64 values of the dtype (exact)."""
+    raw = _bytes_view(raw)
+    n = raw.size // DTYPE_SIZE[dtype]
+    out = np.empty(n, np.float64)
+    lib().oracle_decode_many(_ptr(raw, _u8p), n, dtype, _ptr(out, _f64p))
+    return out
+
+
+# ---------------------------------------------------------------- fill
+def fill_payload(payload, dtype, dist, i0, i1, region_id, p0, p1, seed):
+    """Write elements [i0, i1) of `payload` (uint8 view of element 0 on)."""
+    assert payload.dtype == np.uint8 and payload.flags["C_CONTIGUOUS"]
+    assert i1 * DTYPE_SIZE[dtype] <= payload.size
+    rc = lib().oracle_fill_payload(_ptr(payload, _u8p), dtype, dist, i0, i1,
+                                   region_id, float(p0), float(p1), seed)
+    if rc != 0:
+        raise ValueError("distribution %d does not apply to dtype %d" % (dist, dtype))
+
+
+def _split(n, parts):
+    parts = max(1, min(parts, n)) if n else 1
+    edges = [n * k // parts for k in range(parts + 1)]
+    return list(zip(edges[:-1], edges[1:]))
+
+
+def _run_threads(fns):
+    if len(fns) == 1:
+        fns[0]()
+        return
+    ts = [threading.Thread(target=f) for f in fns]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+
+
+def fill_region(alloc, n_elems, dtype, dist, guard_lo, guard_hi, region_id,
+                canary, p0, p1, seed, threads=1):
+    """Guarded fill of one allocation (uint8 array covering the whole
+    allocation: low guard, payload, high guard)."""
+    nbytes = n_elems * DTYPE_SIZE[dtype]
+    assert alloc.size >= guard_lo + nbytes + guard_hi
+    payload = alloc[guard_lo:guard_lo + nbytes]
+    lib().oracle_fill_guards(_ptr(alloc, _u8p), nbytes, guard_lo, guard_hi, canary)
+    fns = [lambda a=a, b=b: fill_payload(payload, dtype, dist, a, b, region_id, p0, p1, seed)
+           for a, b in _split(n_elems, threads)]
+    _run_threads(fns)
+
+
+def guard_check(alloc, payload_bytes, guard_lo, guard_hi, canary):
+    bad = ctypes.c_uint64()
+    first = ctypes.c_uint64()
+    lib().oracle_guard_check(_ptr(alloc, _u8p), payload_bytes, guard_lo, guard_hi,
+                             canary, ctypes.byref(bad), ctypes.byref(first))
+    return int(bad.value), int(first.value)
+
+
+# ---------------------------------------------------------------- compare
+def compare_range(ref_payload, cand_payload, dtype, i0, i1, atol, rtol):
+    st = _Stats()
+    lib().oracle_compare_range(_ptr(ref_payload, _u8p), _ptr(cand_payload, _u8p),
+                               dtype, i0, i1, float(atol), float(rtol), ctypes.byref(st))
+    return {f: getattr(st, f) for f, _ in _Stats._fields_}
+
+
+def merge_partials(parts):
+    """Combine range results: sums, min of first index, max of the maxima."""
+    out = {"mismatches": 0, "first_mismatch": U64_NONE, "max_abs_err": 0.0,
+           "max_rel_err": 0.0, "nonfinite_mismatches": 0}
+    for p in parts:
+        out["mismatches"] += p["mismatches"]
+        out["first_mismatch"] = min(out["first_mismatch"], p["first_mismatch"])
+        out["max_abs_err"] = max(out["max_abs_err"], p["max_abs_err"])
+        out["max_rel_err"] = max(out["max_rel_err"], p["max_rel_err"])
+        out["nonfinite_mismatches"] += p["nonfinite_mismatches"]
+    return out
+
+
+def compare_payload(ref_payload, cand_payload, dtype, n_elems, atol, rtol, threads=1):
+    parts = [None] * len(_split(n_elems, threads))
+
+    def job(k, a, b):
+        parts[k] = compare_range(ref_payload, cand_payload, dtype, a, b, atol, rtol)
+    _run_threads([lambda k=k, a=a, b=b: job(k, a, b)
+                  for k, (a, b) in enumerate(_split(n_elems, threads))])
+    return merge_partials(parts)
+
+
+def compare_region(ref_alloc, ref_glo, ref_ghi, ref_canary, cand_alloc, cand_glo,
+                   cand_ghi, cand_canary, n_elems, dtype, atol, rtol, threads=1):
+    """Full per-region statistics (8 fields), guards included."""
+    if threads <= 1:
+        st = _RegionStats()
+        lib().oracle_compare_region(_ptr(ref_alloc, _u8p), ref_glo, ref_ghi, ref_canary,
+                                    _ptr(cand_alloc, _u8p), cand_glo, cand_ghi, cand_canary,
+                                    n_elems, dtype, float(atol), float(rtol), ctypes.byref(st))
+        return {f: getattr(st, f) for f in STATS_FIELDS}
+    nbytes = n_elems * DTYPE_SIZE[dtype]
+    out = compare_payload(ref_alloc[ref_glo:ref_glo + nbytes],
+                          cand_alloc[cand_glo:cand_glo + nbytes], dtype, n_elems,
+                          atol, rtol, threads)
+    out["guard_bad_bytes"], out["first_guard_bad"] = guard_check(
+        cand_alloc, nbytes, cand_glo, cand_ghi, cand_canary)
+    out["ref_guard_bad_bytes"] = guard_check(ref_alloc, nbytes, ref_glo, ref_ghi,
+                                             ref_canary)[0]
+    return out
+
+
+def host_threads():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
