@@ -1,0 +1,453 @@
+"""Throughput of the differential-oracle hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic
+input: the Tier 1 guarded fill of the workload's input regions followed by
+the equivalence check of the reference output against every candidate
+(AsmEvo Sec. 3.4 and Eq. 1).  Default workload: a 16 GiB guarded fill of
+GEMM input buffers, then one fp16 [32768, 32768] reference checked against
+8 candidates carrying 0..8 ULP of noise.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
+                       [--workload NAME] [--no-e2e] [--no-cpu]
+For N > 1 launch under torchrun; every rank runs its own replica (weak
+scaling, no data-path collective) and rank 0 prints one JSON line.
+"""
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verify GB/s (ref+cand bytes compared per s) and fill GB/s, % of GB300 HBM peak"
+UNIT = "GB/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ------------------------------------------------------------------ helpers
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.out = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        if not self.out:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        # median over samples taken under load (the busiest half)
+        loaded = sorted(sm)[len(sm) // 2:] if len(sm) > 3 else sm
+        return {"sm_mhz": float(np.median(loaded)), "sm_max_mhz": float(max(smax)),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def kernel_traffic(kernel, workload):
+    """dram read+write bytes per launch from a committed ncu summary, if it
+    was taken on the kernel source as it is now."""
+    path = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
+    if not os.path.exists(path):
+        return None, None
+    txt = open(path).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    h = re.search(r"source_sha256:\s*([0-9a-f]+)", txt)
+    if not m or not h or h.group(1) != source_hash():
+        return None, path
+    return float(m.group(1)), path
+
+
+def source_hash():
+    d = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_20711_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            d.update(f.encode() + fh.read())
+    return d.hexdigest()[:16]
+
+
+# ------------------------------------------------------------------ workload
+class Setup:
+    """Device buffers and region tables of one workload replica."""
+
+    def __init__(self, name, device):
+        import torch
+        from paper_2608_20711_gb300 import asmv
+        from paper_2608_20711_gb300 import workloads as W
+        self.torch, self.asmv, self.W = torch, asmv, W
+        self.name = name
+        self.device = device
+        wl = W.WORKLOADS[name]()
+        self.wl = wl
+        self.ctx = asmv.Context(device.index or 0)
+        dev = device
+        self.ref = torch.empty(wl.arena_bytes, dtype=torch.uint8, device=dev)
+        self.ref_regs = asmv.regions_in_arena(wl.regions, self.ref.data_ptr())
+        self.ctx.fill(self.ref_regs, seed=wl.seed)
+        if wl.input_regions:
+            self.inp = torch.empty(wl.input_arena_bytes, dtype=torch.uint8, device=dev)
+            self.fill_regs = asmv.regions_in_arena(wl.input_regions, self.inp.data_ptr())
+            self.fill_specs = wl.input_regions
+        else:
+            self.inp = None
+            self.fill_regs = self.ref_regs
+            self.fill_specs = wl.regions
+        # candidates (input construction, outside the timed region)
+        rng = np.random.default_rng(wl.seed + 77)
+        self.cands = []
+        ncand = wl.n_cands
+        for j in range(ncand):
+            c = self.ref.clone()
+            if name == "batched_gemm_fp16":
+                W.perturb_uniform_ulps(c, wl.regions[0], seed=wl.seed * 100 + j,
+                                       magnitude=wl.ulp_magnitudes[j])
+            elif name == "fp32_1m":
+                W.perturb_fp32_single(c, wl)
+            elif name == "attention_bf16":
+                for r in wl.regions:
+                    W.perturb_ulp_noise(c, r, seed=wl.seed * 10 + r.region_id)
+            elif name == "int_exact":
+                for r in wl.regions:
+                    W.flip_bit(c, r, rng)
+            elif name == "snapshot_4096":
+                for r in wl.regions:
+                    W.perturb_sparse(c, r, rng, rate=1e-6)
+                for k in rng.choice(len(wl.regions), 3, replace=False):
+                    W.corrupt_guard(c, wl.regions[int(k)], rng, "hi")
+            self.cands.append(c)
+        self.cand_regs = [asmv.regions_in_arena(wl.regions, c.data_ptr()) for c in self.cands]
+        torch.cuda.synchronize(dev)
+        self.fill_bytes = sum(r.alloc_bytes if r.dist != "none" else r.guard_lo + r.guard_hi
+                              for r in self.fill_specs)
+        ref_payload = sum(r.payload_bytes for r in wl.regions)
+        guards = sum(r.guard_lo + r.guard_hi for r in wl.regions)
+        self.verify_physical = ref_payload * (1 + ncand) + guards * (1 + ncand)
+        self.verify_logical = 2 * ref_payload * ncand
+        self.tol = wl.tol
+
+    def step(self):
+        """Fill, then check every candidate (K <= 8 share one reference read)."""
+        self.ctx.fill(self.fill_regs, seed=self.wl.seed)
+        if len(self.cands) == 1:
+            return [self.ctx.compare(self.ref_regs, self.cand_regs[0], self.tol)]
+        return self.ctx.compare_batched(self.ref_regs, self.cand_regs, self.tol)
+
+
+# ------------------------------------------------------------------ CPU oracle
+def _timed_until(budget_s, fn, n0, nmax):
+    """Run fn(n) with n doubling until one run takes >= budget_s (or n hits
+    nmax); return (n, seconds, result) of the last run."""
+    n = n0
+    while True:
+        t0 = time.perf_counter()
+        res = fn(n)
+        dt = time.perf_counter() - t0
+        if dt >= budget_s or n >= nmax:
+            return n, dt, res
+        n = min(nmax, n * max(2, int(budget_s / max(dt, 1e-3) * 0.7)))
+
+
+def cpu_oracle_sample(setup, budget_s=12.0):
+    """The oracle as it stands, on the host cores, over a bounded sample of
+    the same workload: element prefixes of the fill regions (one of each
+    dtype/distribution kind) and of the reference/candidate payloads.  The
+    two measured rates are combined over the step's byte mix."""
+    from oracle import oracle as O
+    ORACLE_DTYPE, ORACLE_DIST = O.CODE_OF_DTYPE, O.CODE_OF_DIST
+    W = setup.W
+    threads = O.host_threads()
+    kinds = {}
+    for r in setup.fill_specs:
+        kinds.setdefault((r.dtype, r.dist), r)
+    cap_bytes = 256 << 20
+    bufs = {k: np.zeros(min(r.payload_bytes, cap_bytes), np.uint8) for k, r in kinds.items()}
+
+    def fill(n_bytes):
+        done = 0
+        for (dt, dist), r in kinds.items():
+            sz = W.DTYPE_SIZE[dt]
+            n = min(n_bytes // sz, bufs[(dt, dist)].size // sz)
+            O.fill_region(bufs[(dt, dist)], n, ORACLE_DTYPE[dt], ORACLE_DIST[dist], 0, 0,
+                          r.region_id, r.canary, r.p0, r.p1, setup.wl.seed, threads=threads)
+            done += n * sz
+        return done
+
+    _, t_fill, fill_done = _timed_until(budget_s / 2, fill, 1 << 16, cap_bytes)
+    # reference/candidate payload prefixes of the first region
+    r = setup.wl.regions[0]
+    nb = min(r.payload_bytes, cap_bytes // max(1, len(setup.cands)))
+    a = setup.ref[r.payload_offset:r.payload_offset + nb].cpu().numpy()
+    cs = [c[r.payload_offset:r.payload_offset + nb].cpu().numpy() for c in setup.cands]
+    t = setup.tol.get(r.dtype, W.Tolerance(0.0, 0.0))
+    sz = W.DTYPE_SIZE[r.dtype]
+
+    def compare(n_bytes):
+        n = min(n_bytes, nb) // sz
+        for c in cs:
+            O.compare_payload(a, c, ORACLE_DTYPE[r.dtype], n, t.atol, t.rtol, threads=threads)
+        return n * sz * (1 + len(cs))
+
+    _, t_cmp, cmp_done = _timed_until(budget_s / 2, compare, 1 << 16, nb)
+    fill_rate = fill_done / t_fill
+    cmp_rate = cmp_done / t_cmp
+    step_s = setup.fill_bytes / fill_rate + setup.verify_physical / cmp_rate
+    value = (setup.fill_bytes + setup.verify_physical) / step_s / 1e9
+    sample = ("oracle fill of %.1f MB over %d region kinds and compare of %.1f MB of "
+              "reference + %d candidate payload prefixes, %d threads; rates combined over the "
+              "step's fill/verify byte mix" % (fill_done / 1e6, len(kinds), cmp_done / 1e6,
+                                               len(cs), threads))
+    return {"value": round(value, 4), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": sample, "fill_gbs": round(fill_rate / 1e9, 4),
+            "verify_gbs": round(cmp_rate / 1e9, 4), "seconds": round(t_fill + t_cmp, 2)}
+
+
+# ------------------------------------------------------------------ runs
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_mine(args):
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    setup = Setup(args.workload, device)
+    ctx = setup.ctx
+    stream = torch.cuda.current_stream(device)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(device)
+
+    for _ in range(args.warmup):
+        stats = setup.step()
+    barrier()
+    # kernel durations: CUDA events around each launch (one step at a time)
+    ctx.set_timing(True)
+    fill_ms, cmp_ms = [], []
+    for _ in range(max(3, args.steps)):
+        ctx.fill(setup.fill_regs, seed=setup.wl.seed)
+        fill_ms.append(ctx.kernel_ms())
+        if len(setup.cands) == 1:
+            ctx.compare(setup.ref_regs, setup.cand_regs[0], setup.tol)
+        else:
+            ctx.compare_batched(setup.ref_regs, setup.cand_regs, setup.tol)
+        cmp_ms.append(ctx.kernel_ms())
+    ctx.set_timing(False)
+    barrier()
+    # the timed region: K whole steps
+    launches0 = ctx.launches
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            stats = setup.step()
+        ev1.record(stream)
+        barrier()
+    elapsed = ev0.elapsed_time(ev1) / 1e3
+    launches = ctx.launches - launches0
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([elapsed], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    step_bytes = setup.fill_bytes + setup.verify_physical
+    value = world * step_bytes * args.steps / elapsed / 1e9
+    # e2e: the public API with host buffers (pinned), copies inside the timed region
+    e2e = None
+    if args.e2e:
+        e2e = run_e2e(setup, args, device, world, barrier)
+    peak, peak_kind = measured_peaks()
+    f_ms, c_ms = float(np.mean(fill_ms)), float(np.mean(cmp_ms))
+    fill_gbs = setup.fill_bytes / (f_ms / 1e3) / 1e9
+    verify_gbs = setup.verify_physical / (c_ms / 1e3) / 1e9
+    if c_ms >= f_ms:
+        dom, dom_bytes, dom_ms = "compare", setup.verify_physical, c_ms
+    else:
+        dom, dom_bytes, dom_ms = "fill", setup.fill_bytes, f_ms
+    achieved = dom_bytes / (dom_ms / 1e3) / 1e9
+    traffic, _ = kernel_traffic(dom, args.workload)
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": traffic,
+                "kernel": dom, "peak_kind": peak_kind + " (copy bandwidth, burst)",
+                "algorithmic_bytes_per_launch": dom_bytes, "avg_launch_ms": round(dom_ms, 4)}
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(elapsed / args.steps * 1e3, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded Philox fill; seeded candidate perturbations)",
+        "config": {"workload": args.workload, "description": setup.wl.description,
+                   "fill_bytes": setup.fill_bytes, "verify_bytes_physical": setup.verify_physical,
+                   "verify_bytes_logical": setup.verify_logical, "candidates": len(setup.cands),
+                   "l2": "inputs larger than L2 (129 MB); no flush",
+                   "parallelism": "replica per GPU" if world > 1 else "1 GPU"},
+        "fill_gbs": round(fill_gbs, 1), "verify_gbs": round(verify_gbs, 1),
+        "fill_frac": round(fill_gbs / peak, 4), "verify_frac": round(verify_gbs / peak, 4),
+        "clocks": clk.summary(), "gpu_launches": launches, "roofline": roofline,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and args.cpu:
+        line["cpu_baseline"] = cpu_oracle_sample(setup)
+    if rank == 0:
+        mism = sum(int(s["mismatches"]) for cs in stats for s in cs)
+        line["check"] = {"total_mismatches": mism}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_e2e(setup, args, device, world, barrier):
+    """Host buffers through the public API: every step copies the reference
+    and candidate outputs from pinned host memory, fills, checks, and reads
+    the statistics back."""
+    import torch
+    ctx = setup.ctx
+    host_ref = setup.ref.cpu().pin_memory()
+    host_cands = [c.cpu().pin_memory() for c in setup.cands]
+    stream = torch.cuda.current_stream(device)
+    h2d = host_ref.numel() + sum(h.numel() for h in host_cands)
+    nstat = len(setup.wl.regions) * len(setup.cands)
+    d2h = 64 * nstat
+
+    def e2e_step():
+        setup.ref.copy_(host_ref, non_blocking=True)
+        for c, h in zip(setup.cands, host_cands):
+            c.copy_(h, non_blocking=True)
+        return setup.step()                        # stats come back to the host inside
+
+    for _ in range(2):
+        e2e_step()
+    barrier()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    ev1.record(stream)
+    barrier()
+    el = ev0.elapsed_time(ev1) / 1e3
+    step_bytes = setup.fill_bytes + setup.verify_physical
+    return {"value": round(world * step_bytes * args.steps / el / 1e9, 1), "unit": UNIT,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "ms_per_step": round(el / args.steps * 1e3, 3)}
+
+
+def run_reference(args):
+    """The oracle (plain CPU program) on the same workload: each step is a
+    bounded sample, extrapolated to the step's byte mix."""
+    world, rank, local = dist_env()
+    if rank != 0:
+        return
+    import torch
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    setup = Setup(args.workload, device)
+    for _ in range(args.warmup):
+        pass
+    vals, secs = [], []
+    for _ in range(args.steps):
+        r = cpu_oracle_sample(setup, budget_s=max(2.0, 60.0 / max(1, args.steps)))
+        vals.append(r["value"])
+        secs.append(r["seconds"])
+    step_bytes = setup.fill_bytes + setup.verify_physical
+    value = float(np.median(vals))
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(step_bytes / (value * 1e9) * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": args.workload},
+            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": r["cores"],
+                             "kind": "oracle", "sample": r["sample"]},
+            "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="mine", choices=["mine", "reference"])
+    ap.add_argument("--workload", default="batched_gemm_fp16")
+    ap.add_argument("--no-e2e", dest="e2e", action="store_false")
+    ap.add_argument("--no-cpu", dest="cpu", action="store_false")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    import __graft_entry__
+    __graft_entry__.build()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_mine(args)
+
+
+if __name__ == "__main__":
+    main()

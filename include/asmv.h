@@ -1,0 +1,220 @@
+/*
+ * asmv.h -- C ABI of the GB300 differential-oracle hot path.
+ *
+ * The library implements the data-parallel core of the differential oracle
+ * that gates every candidate kernel in AsmEvo (arXiv 2608.20711):
+ *
+ *   - Tier 1 guarded input synthesis (Sec. 3.4, "Tier 1: synthetic
+ *     inference"): every allocation a kernel references is filled with
+ *     deterministic seeded values, and guard bands on both sides of the
+ *     payload are set to a canary byte so that out-of-bounds writes become
+ *     visible.
+ *   - The equivalence check eq(K', x) of Eq. 1 (Sec. 3.2, R2) applied to the
+ *     captured output regions (Sec. 3.4, "Tier 2: real-dispatch capture"):
+ *     floating-point outputs are checked against a tolerance, integer
+ *     buffers, opaque state and guard bytes must match byte-exactly (the
+ *     iota term of Eq. 1).  The tolerance is applied per element with a
+ *     per-dtype (atol, rtol): element r (reference) and c (candidate) match
+ *     iff |c - r| <= atol + rtol*|r|, evaluated in fp64 on the exactly
+ *     decoded values.  Per region the library reports the mismatch count,
+ *     the first mismatching element, the exact fp64 maximum absolute and
+ *     relative error over finite pairs (the ||Delta||_inf of Eq. 1 is
+ *     max_abs_err when nonfinite_mismatches == 0), NaN/Inf-position
+ *     mismatches and guard-band damage.
+ *
+ * All device work runs in CUDA kernels on the caller's stream.  There is no
+ * CPU fallback: a call whose tables point at host memory fails with
+ * ASMV_EINVAL.
+ *
+ * Threading: a context is not thread-safe.  Use one context per host
+ * thread; calls on one context are ordered on the device even when they
+ * name different streams (each call waits for the previous call's use of
+ * the context's workspace).
+ */
+#ifndef ASMV_H_
+#define ASMV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ASMV_ABI_VERSION 1
+
+/* A CUDA stream (the same type as cudaStream_t); NULL is the legacy
+ * default stream. */
+typedef struct CUstream_st *asmv_stream_t;
+
+/* Element types of a region.  Float types are compared with the tolerance
+ * test; integer and opaque types bit-exactly (Sec. 3.4, Tier 2). */
+typedef enum {
+  ASMV_F32 = 0,        /* IEEE binary32 */
+  ASMV_BF16 = 1,       /* bfloat16 */
+  ASMV_F16 = 2,        /* IEEE binary16 */
+  ASMV_F8E4M3 = 3,     /* OCP FP8 E4M3 (no Inf; S.1111.111 is NaN; max 448) */
+  ASMV_I32 = 4,        /* two's complement int32 */
+  ASMV_I8 = 5,         /* two's complement int8 */
+  ASMV_U8_OPAQUE = 6,  /* opaque bytes (compared as unsigned 8-bit values) */
+  ASMV_NDTYPES = 7
+} asmv_dtype;
+
+/* Payload distributions of asmv_fill (Sec. 3.4, Tier 1: deterministic
+ * inputs from random seeds).  Element i draws from Philox4x32-10 with
+ * key = (seed lo, seed hi) and counter = (block lo, block hi, region_id, 0):
+ *   RAW       payload byte j is byte (j mod 16) of block (j div 16); the
+ *             block's four 32-bit words in order, each little-endian.
+ *             Any dtype.
+ *   UNIFORM   float dtypes: word w = word (i mod 4) of block (i div 4),
+ *             f = (w >> 8) * 2^-24, v = p0 + f*(p1 - p0) in fp32 (p0, p1 and
+ *             p1 - p0 rounded to fp32 first; multiply then add), then
+ *             round-to-nearest-even to the dtype (fp8 saturates to +-448).
+ *   NORMAL    float dtypes: Box-Muller on words (0,1) and (2,3) of block
+ *             (i div 4): u1 = ((w0 >> 8) + 1) 2^-24, u2 = (w1 >> 8) 2^-24,
+ *             z0 = sqrt(-2 ln u1) cos(2 pi u2), z1 = ... sin(2 pi u2);
+ *             element 4b+2p+t is z_t of pair p; v = p0 + p1*z in fp32, then
+ *             RNE to the dtype.  ln and sincos are fixed fp32 series
+ *             evaluations, so results are bit-reproducible.
+ *   INT_RANGE integer dtypes: w as for UNIFORM, v = lo + ((w*(hi-lo)) >> 32)
+ *             with lo = p0, hi = p1 (integers; 1 <= hi - lo <= 2^32 and
+ *             [lo, hi) inside the dtype's range).
+ *   NONE      the payload is left untouched; only guard bands are written. */
+typedef enum {
+  ASMV_DIST_RAW = 0,
+  ASMV_DIST_UNIFORM = 1,
+  ASMV_DIST_NORMAL = 2,
+  ASMV_DIST_INT_RANGE = 3,
+  ASMV_DIST_NONE = 4
+} asmv_dist;
+
+/* One guarded allocation (Sec. 3.4: a referenced device-memory region with
+ * guard regions initialised with canaries).  Layout in device memory:
+ *   [alloc, alloc+guard_lo)                   low guard band
+ *   [alloc+guard_lo, +n_elems*size(dtype))    payload
+ *   [payload end, +guard_hi)                  high guard band
+ * All three lie in one device allocation owned by the caller.  56 bytes. */
+typedef struct {
+  uint64_t alloc;      /* device address of the allocation start */
+  uint64_t n_elems;    /* payload elements (may be 0) */
+  uint32_t dtype;      /* asmv_dtype */
+  uint32_t dist;       /* asmv_dist; read by asmv_fill only */
+  uint32_t guard_lo;   /* guard bytes below the payload (may be 0) */
+  uint32_t guard_hi;   /* guard bytes above the payload (may be 0) */
+  uint32_t region_id;  /* Philox counter word 2 for this region's payload */
+  uint8_t canary;      /* guard byte value */
+  uint8_t pad_[3];
+  double p0, p1;       /* distribution parameters (see asmv_dist) */
+} asmv_region;
+
+/* Per-dtype tolerance, indexed by asmv_dtype; entries of integer and opaque
+ * dtypes are ignored.  Both must be >= 0 and not NaN for float dtypes. */
+typedef struct {
+  double atol;
+  double rtol;
+} asmv_tol;
+
+/* Per-region result (64 bytes). */
+typedef struct {
+  uint64_t mismatches;           /* elements failing the check (incl. non-finite) */
+  uint64_t first_mismatch;       /* lowest failing element index; UINT64_MAX if none */
+  double max_abs_err;            /* max over finite pairs of |c - r| (exact fp64); 0 if none */
+  double max_rel_err;            /* max over finite pairs of |c - r| / |r|; r == 0 gives
+                                    0 when c == r, else +Inf */
+  uint64_t nonfinite_mismatches; /* failing pairs with a NaN or Inf on either side */
+  uint64_t guard_bad_bytes;      /* guard bytes != canary (candidate side, or the region
+                                    itself for asmv_guard_check) */
+  uint64_t first_guard_bad;      /* lowest such byte offset from alloc; UINT64_MAX if none */
+  uint64_t ref_guard_bad_bytes;  /* asmv_compare*: damaged reference guard bytes */
+} asmv_stats;
+
+/* Status codes.  A failed call leaves out_host untouched. */
+#define ASMV_OK 0
+#define ASMV_EINVAL (-1)    /* bad argument or table (see each call) */
+#define ASMV_ECUDA (-2)     /* a CUDA runtime call failed; see asmv_ctx_cuda_error */
+#define ASMV_ETIMEOUT (-3)  /* a bounded device wait expired */
+#define ASMV_ENOMEM (-4)    /* workspace or staging allocation failed */
+
+typedef struct asmv_ctx asmv_ctx;
+
+/* Create a context on CUDA device `device`.  The context owns a device
+ * workspace (region tables, statistics) and pinned host staging, both grown
+ * on demand.  Returns ASMV_OK and *out, or EINVAL (null out, bad device),
+ * ECUDA, ENOMEM. */
+int asmv_ctx_create(asmv_ctx **out, int device);
+
+/* Release the context (synchronises its outstanding work).  NULL is a no-op. */
+void asmv_ctx_destroy(asmv_ctx *ctx);
+
+/* Tier 1 guarded fill (Sec. 3.4, Tier 1).  Writes every region's payload
+ * from its distribution and both guard bands with its canary.  The table is
+ * copied before return; the fill itself is asynchronous on `stream`.
+ * EINVAL: null ctx/table with n > 0, unknown dtype or dist, a distribution
+ * that does not apply to the dtype or parameters out of range, size
+ * overflow, a zero alloc address with a non-empty allocation, overlapping
+ * allocations, or memory that is not device memory of ctx's device (or
+ * that ends past its allocation). */
+int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed,
+              asmv_stream_t stream);
+
+/* Guard-band integrity (the "intact out-of-bounds guards" of the iota term
+ * of Eq. 1, Sec. 3.2).  For each region, counts guard bytes that differ
+ * from its canary and the first such offset from alloc (low band first).
+ * out_host[i] receives guard_bad_bytes and first_guard_bad; the other
+ * fields are their empty values (0, UINT64_MAX).  Synchronous: returns
+ * after the results are in out_host.  Errors as asmv_fill (overlap is
+ * allowed), plus EINVAL for null out_host. */
+int asmv_guard_check(asmv_ctx *ctx, const asmv_region *regions, size_t n,
+                     asmv_stats *out_host, asmv_stream_t stream);
+
+/* The equivalence check (Eq. 1 per element, Sec. 3.2; Tier 2 rule, Sec.
+ * 3.4) of n (reference, candidate) region pairs: ref[i] against cand[i].
+ * Pairs must agree in dtype and n_elems.  Candidate guards feed
+ * guard_bad_bytes / first_guard_bad, reference guards ref_guard_bad_bytes.
+ * tol has ASMV_NDTYPES entries.  Synchronous.  EINVAL as asmv_guard_check,
+ * plus dtype/count disagreement and invalid tolerances. */
+int asmv_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cand,
+                 size_t n, const asmv_tol *tol, asmv_stats *out_host,
+                 asmv_stream_t stream);
+
+/* The check over many candidates at once (the eq loop of Algorithm 1 run
+ * for k candidates against one oracle output): cands[j] is an array of n
+ * regions matching ref; out_host has k*n entries, out_host[j*n + i] being
+ * compare(ref[i], cands[j][i]).  Each reference tile is read from device
+ * memory once per group of up to 8 candidates.  Synchronous.  Errors as
+ * asmv_compare, plus EINVAL for k == 0 or a null cands entry. */
+int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref,
+                         const asmv_region *const *cands, size_t k, size_t n,
+                         const asmv_tol *tol, asmv_stats *out_host,
+                         asmv_stream_t stream);
+
+/* Host-only validation of a region table, the checks every call above
+ * makes before touching the device, except the device-memory checks.
+ * for_fill != 0 adds the distribution and overlap rules of asmv_fill.
+ * Makes no CUDA call.  Returns ASMV_OK or ASMV_EINVAL. */
+int asmv_check_regions(const asmv_region *regions, size_t n, int for_fill);
+
+/* Kernel timing: when enabled, each call records CUDA events around its
+ * kernel launch on the call's stream; asmv_ctx_kernel_ms then returns the
+ * device time of the last call's kernel (waiting for it to finish).
+ * EINVAL for a null ctx or ms, or when timing is off / nothing ran. */
+int asmv_ctx_set_timing(asmv_ctx *ctx, int enable);
+int asmv_ctx_kernel_ms(asmv_ctx *ctx, float *ms);
+
+/* The CUDA error code behind the last ASMV_ECUDA on this context (0 if none). */
+int asmv_ctx_cuda_error(const asmv_ctx *ctx);
+
+/* Number of kernels this context has launched since creation. */
+uint64_t asmv_ctx_launches(const asmv_ctx *ctx);
+
+/* Static description of a status code. */
+const char *asmv_strerror(int status);
+
+/* ASMV_ABI_VERSION of the loaded library. */
+int asmv_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASMV_H_ */

@@ -22,6 +22,11 @@ RAW, UNIFORM, NORMAL, INT_RANGE, NONE = range(5)
 DTYPE_SIZE = {F32: 4, BF16: 2, F16: 2, F8E4M3: 1, I32: 4, I8: 1, U8: 1}
 FLOAT_DTYPES = (F32, BF16, F16, F8E4M3)
 U64_NONE = (1 << 64) - 1
+# codes by the names the workload descriptions use
+CODE_OF_DTYPE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32,
+                 "i8": I8, "u8": U8}
+CODE_OF_DIST = {"raw": RAW, "uniform": UNIFORM, "normal": NORMAL, "int_range": INT_RANGE,
+                "none": NONE}
 
 _u8p = ctypes.POINTER(ctypes.c_uint8)
 _u32p = ctypes.POINTER(ctypes.c_uint32)

@@ -1,0 +1,253 @@
+"""ctypes binding of the C ABI in include/asmv.h (argument marshalling only).
+
+Every step of the fill, guard check and comparison runs in the CUDA
+kernels of libasmv.so; this module converts Python region descriptions to
+the C structs, passes raw device addresses and a CUDA stream handle, and
+turns status codes into exceptions.  There is no fallback: if the library
+is missing or the GPU is absent, calls fail loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Iterable, List, Optional, Sequence
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libasmv.so")
+
+# asmv_dtype / asmv_dist codes
+F32, BF16, F16, F8E4M3, I32, I8, U8_OPAQUE = range(7)
+NDTYPES = 7
+DIST_RAW, DIST_UNIFORM, DIST_NORMAL, DIST_INT_RANGE, DIST_NONE = range(5)
+DTYPE_CODE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32,
+              "i8": I8, "u8": U8_OPAQUE}
+DIST_CODE = {"raw": DIST_RAW, "uniform": DIST_UNIFORM, "normal": DIST_NORMAL,
+             "int_range": DIST_INT_RANGE, "none": DIST_NONE}
+OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM = 0, -1, -2, -3, -4
+U64_NONE = (1 << 64) - 1
+
+
+class Region(ctypes.Structure):
+    """asmv_region (56 bytes)."""
+    _fields_ = [("alloc", ctypes.c_uint64), ("n_elems", ctypes.c_uint64),
+                ("dtype", ctypes.c_uint32), ("dist", ctypes.c_uint32),
+                ("guard_lo", ctypes.c_uint32), ("guard_hi", ctypes.c_uint32),
+                ("region_id", ctypes.c_uint32), ("canary", ctypes.c_uint8),
+                ("pad_", ctypes.c_uint8 * 3), ("p0", ctypes.c_double), ("p1", ctypes.c_double)]
+
+
+class Tol(ctypes.Structure):
+    _fields_ = [("atol", ctypes.c_double), ("rtol", ctypes.c_double)]
+
+
+class Stats(ctypes.Structure):
+    """asmv_stats (64 bytes)."""
+    _fields_ = [("mismatches", ctypes.c_uint64), ("first_mismatch", ctypes.c_uint64),
+                ("max_abs_err", ctypes.c_double), ("max_rel_err", ctypes.c_double),
+                ("nonfinite_mismatches", ctypes.c_uint64), ("guard_bad_bytes", ctypes.c_uint64),
+                ("first_guard_bad", ctypes.c_uint64), ("ref_guard_bad_bytes", ctypes.c_uint64)]
+
+
+STATS_FIELDS = [f for f, _ in Stats._fields_]
+assert ctypes.sizeof(Region) == 56 and ctypes.sizeof(Stats) == 64
+
+ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard_check",
+                 "asmv_compare", "asmv_compare_batched", "asmv_check_regions",
+                 "asmv_ctx_set_timing", "asmv_ctx_kernel_ms", "asmv_ctx_cuda_error",
+                 "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version")
+
+
+class AsmvError(RuntimeError):
+    def __init__(self, status: int, message: str, cuda_error: int = 0):
+        super().__init__("asmv status %d (%s)%s" % (
+            status, message, ", cudaError %d" % cuda_error if cuda_error else ""))
+        self.status = status
+        self.cuda_error = cuda_error
+
+
+_lib = None
+
+
+def lib():
+    """Load libasmv.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libasmv.so is not built: run paper_2608_20711_gb300.build.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, sz = ctypes.c_void_p, ctypes.c_size_t
+        RP, SP, TP = ctypes.POINTER(Region), ctypes.POINTER(Stats), ctypes.POINTER(Tol)
+        L.asmv_ctx_create.argtypes = [ctypes.POINTER(vp), ctypes.c_int]
+        L.asmv_ctx_destroy.argtypes = [vp]
+        L.asmv_ctx_destroy.restype = None
+        L.asmv_fill.argtypes = [vp, RP, sz, ctypes.c_uint64, vp]
+        L.asmv_guard_check.argtypes = [vp, RP, sz, SP, vp]
+        L.asmv_compare.argtypes = [vp, RP, RP, sz, TP, SP, vp]
+        L.asmv_compare_batched.argtypes = [vp, RP, ctypes.POINTER(RP), sz, sz, TP, SP, vp]
+        L.asmv_check_regions.argtypes = [RP, sz, ctypes.c_int]
+        L.asmv_ctx_set_timing.argtypes = [vp, ctypes.c_int]
+        L.asmv_ctx_kernel_ms.argtypes = [vp, ctypes.POINTER(ctypes.c_float)]
+        L.asmv_ctx_cuda_error.argtypes = [vp]
+        L.asmv_ctx_launches.argtypes = [vp]
+        L.asmv_ctx_launches.restype = ctypes.c_uint64
+        L.asmv_strerror.argtypes = [ctypes.c_int]
+        L.asmv_strerror.restype = ctypes.c_char_p
+        L.asmv_abi_version.argtypes = []
+        _lib = L
+    return _lib
+
+
+def strerror(status: int) -> str:
+    return lib().asmv_strerror(status).decode()
+
+
+def region_array(regions: Sequence) -> ctypes.Array:
+    """ctypes array of Region from Region instances or dicts."""
+    arr = (Region * max(1, len(regions)))()
+    for i, r in enumerate(regions):
+        if isinstance(r, Region):
+            arr[i] = r
+        else:
+            arr[i] = make_region(**r)
+    return arr
+
+
+def make_region(alloc: int, n_elems: int, dtype, dist="raw", guard_lo=0, guard_hi=0,
+                region_id=0, canary=0xA5, p0=0.0, p1=0.0) -> Region:
+    r = Region()
+    r.alloc = int(alloc)
+    r.n_elems = int(n_elems)
+    r.dtype = DTYPE_CODE[dtype] if isinstance(dtype, str) else int(dtype)
+    r.dist = DIST_CODE[dist] if isinstance(dist, str) else int(dist)
+    r.guard_lo = int(guard_lo)
+    r.guard_hi = int(guard_hi)
+    r.region_id = int(region_id)
+    r.canary = int(canary)
+    r.p0 = float(p0)
+    r.p1 = float(p1)
+    return r
+
+
+def regions_in_arena(specs: Iterable, base: int) -> List[Region]:
+    """Regions of workload specs (objects with dtype, n_elems, dist, p0, p1,
+    guard_lo, guard_hi, canary, region_id, offset) placed at `base`."""
+    return [make_region(base + s.offset, s.n_elems, s.dtype, s.dist, s.guard_lo, s.guard_hi,
+                        s.region_id, s.canary, s.p0, s.p1) for s in specs]
+
+
+def tol_array(tol: Optional[Dict] = None) -> ctypes.Array:
+    """Per-dtype tolerances: dict of dtype name/code -> (atol, rtol) or an
+    object with .atol/.rtol; unspecified float dtypes get (0, 0)."""
+    arr = (Tol * NDTYPES)()
+    for k, v in (tol or {}).items():
+        code = DTYPE_CODE[k] if isinstance(k, str) else int(k)
+        if hasattr(v, "atol"):
+            arr[code] = Tol(float(v.atol), float(v.rtol))
+        else:
+            arr[code] = Tol(float(v[0]), float(v[1]))
+    return arr
+
+
+def stats_dicts(arr, count: int) -> List[dict]:
+    return [{f: getattr(arr[i], f) for f in STATS_FIELDS} for i in range(count)]
+
+
+def check_regions(regions: Sequence, for_fill: bool = False) -> int:
+    """Host-only table validation (no GPU needed); returns the status."""
+    arr = region_array(regions)
+    return lib().asmv_check_regions(arr, len(regions), 1 if for_fill else 0)
+
+
+def _stream_handle(stream) -> Optional[int]:
+    if stream is None:
+        try:
+            import torch
+            return torch.cuda.current_stream().cuda_stream
+        except Exception:
+            return None
+    if hasattr(stream, "cuda_stream"):
+        return stream.cuda_stream
+    return int(stream)
+
+
+class Context:
+    """One asmv context on one CUDA device (not thread-safe)."""
+
+    def __init__(self, device: int = 0):
+        self._lib = lib()
+        h = ctypes.c_void_p()
+        rc = self._lib.asmv_ctx_create(ctypes.byref(h), int(device))
+        if rc != OK:
+            raise AsmvError(rc, strerror(rc))
+        self._h = h
+        self.device = device
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            self._lib.asmv_ctx_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def _check(self, rc):
+        if rc != OK:
+            raise AsmvError(rc, strerror(rc), self._lib.asmv_ctx_cuda_error(self._h))
+
+    @property
+    def launches(self) -> int:
+        return int(self._lib.asmv_ctx_launches(self._h))
+
+    def set_timing(self, enable: bool = True):
+        self._check(self._lib.asmv_ctx_set_timing(self._h, 1 if enable else 0))
+
+    def kernel_ms(self) -> float:
+        ms = ctypes.c_float()
+        self._check(self._lib.asmv_ctx_kernel_ms(self._h, ctypes.byref(ms)))
+        return float(ms.value)
+
+    def fill(self, regions: Sequence, seed: int, stream=None):
+        arr = region_array(regions)
+        self._check(self._lib.asmv_fill(self._h, arr, len(regions), int(seed),
+                                        _stream_handle(stream)))
+
+    def guard_check(self, regions: Sequence, stream=None) -> List[dict]:
+        arr = region_array(regions)
+        out = (Stats * max(1, len(regions)))()
+        self._check(self._lib.asmv_guard_check(self._h, arr, len(regions), out,
+                                               _stream_handle(stream)))
+        return stats_dicts(out, len(regions))
+
+    def compare(self, ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:
+        ra, ca = region_array(ref), region_array(cand)
+        out = (Stats * max(1, len(ref)))()
+        self._check(self._lib.asmv_compare(self._h, ra, ca, len(ref), tol_array(tol)
+                                           if not isinstance(tol, ctypes.Array) else tol,
+                                           out, _stream_handle(stream)))
+        return stats_dicts(out, len(ref))
+
+    def compare_batched(self, ref: Sequence, cands: Sequence[Sequence], tol,
+                        stream=None) -> List[List[dict]]:
+        n, k = len(ref), len(cands)
+        ra = region_array(ref)
+        cas = [region_array(c) for c in cands]
+        ptrs = (ctypes.POINTER(Region) * max(1, k))(*[ctypes.cast(c, ctypes.POINTER(Region))
+                                                      for c in cas])
+        out = (Stats * max(1, k * n))()
+        self._check(self._lib.asmv_compare_batched(
+            self._h, ra, ptrs, k, n,
+            tol_array(tol) if not isinstance(tol, ctypes.Array) else tol, out,
+            _stream_handle(stream)))
+        flat = stats_dicts(out, k * n)
+        return [flat[j * n:(j + 1) * n] for j in range(k)]

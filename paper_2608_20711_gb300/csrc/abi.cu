@@ -1,0 +1,636 @@
+// abi.cu -- the C ABI of include/asmv.h: argument validation, device-memory
+// checks, launch-plan packing, workspace management and result readback.
+//
+// Each call packs its plan (region descriptors with tile prefixes, candidate
+// addresses, guard segments, initial statistics) into pinned staging,
+// copies it to the context's device workspace with one asynchronous copy,
+// launches the kernel(s) on the caller's stream and, for the checking
+// calls, copies the statistics back and synchronises the stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <utility>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "asmv.h"
+#include "plan.h"
+
+using namespace asmv;
+
+static_assert(sizeof(asmv_region) == 56, "asmv_region layout");
+static_assert(sizeof(asmv_stats) == 64, "asmv_stats layout");
+static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
+static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
+              "plan layouts");
+
+namespace {
+
+typedef int (*AddrRangeFn)(unsigned long long *base, size_t *size, unsigned long long ptr);
+
+const int kDtypeSize[ASMV_NDTYPES] = {4, 2, 2, 1, 4, 1, 1};
+
+bool is_float(uint32_t dt) { return dt <= ASMV_F8E4M3; }
+
+// ------------------------------------------------------------ validation
+bool region_extent(const asmv_region &r, uint64_t *payload_bytes, uint64_t *total) {
+  if (r.dtype >= ASMV_NDTYPES) return false;
+  const uint64_t sz = (uint64_t)kDtypeSize[r.dtype];
+  if (r.n_elems > UINT64_MAX / sz) return false;
+  const uint64_t pb = r.n_elems * sz;
+  const uint64_t t = pb + (uint64_t)r.guard_lo;
+  if (t < pb || t + (uint64_t)r.guard_hi < t) return false;
+  const uint64_t tot = t + (uint64_t)r.guard_hi;
+  if (tot > 0 && r.alloc == 0) return false;
+  if (r.alloc + tot < r.alloc) return false;
+  *payload_bytes = pb;
+  *total = tot;
+  return true;
+}
+
+bool fits_f32(double x) { return std::isfinite(x) && std::fabs(x) <= (double)3.4028234663852886e38; }
+
+bool dist_ok(const asmv_region &r) {
+  switch (r.dist) {
+    case ASMV_DIST_RAW:
+    case ASMV_DIST_NONE:
+      return true;
+    case ASMV_DIST_UNIFORM: {
+      if (!is_float(r.dtype) || !fits_f32(r.p0) || !fits_f32(r.p1) || !(r.p0 <= r.p1)) return false;
+      const float w = (float)r.p1 - (float)r.p0;
+      return std::isfinite(w);
+    }
+    case ASMV_DIST_NORMAL: {
+      if (!is_float(r.dtype) || !fits_f32(r.p0) || !fits_f32(r.p1) || !(r.p1 >= 0.0)) return false;
+      // |mean| + 6 std bounds mean + std*z (|z| <= 5.8) away from fp32 overflow
+      return std::fabs((double)(float)r.p0) + 6.0 * (double)(float)r.p1 <= 3.4e38;
+    }
+    case ASMV_DIST_INT_RANGE: {
+      if (is_float(r.dtype)) return false;
+      if (!std::isfinite(r.p0) || !std::isfinite(r.p1)) return false;
+      if (r.p0 != std::floor(r.p0) || r.p1 != std::floor(r.p1) || !(r.p0 < r.p1)) return false;
+      double lo_lim, hi_lim;
+      if (r.dtype == ASMV_I32) { lo_lim = -2147483648.0; hi_lim = 2147483648.0; }
+      else if (r.dtype == ASMV_I8) { lo_lim = -128.0; hi_lim = 128.0; }
+      else { lo_lim = 0.0; hi_lim = 256.0; }
+      return r.p0 >= lo_lim && r.p1 <= hi_lim && (r.p1 - r.p0) <= 4294967296.0;
+    }
+    default:
+      return false;
+  }
+}
+
+int check_table(const asmv_region *regs, size_t n, bool for_fill) {
+  if (n > 0 && regs == nullptr) return ASMV_EINVAL;
+  if (n > (size_t)0x7FFFFFFF) return ASMV_EINVAL;
+  std::vector<std::pair<uint64_t, uint64_t>> spans;
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    if (!region_extent(regs[i], &pb, &tot)) return ASMV_EINVAL;
+    if (for_fill) {
+      if (!dist_ok(regs[i])) return ASMV_EINVAL;
+      if (tot > 0) spans.emplace_back(regs[i].alloc, regs[i].alloc + tot);
+    }
+  }
+  if (for_fill && spans.size() > 1) {
+    std::sort(spans.begin(), spans.end());
+    for (size_t i = 1; i < spans.size(); ++i)
+      if (spans[i].first < spans[i - 1].second) return ASMV_EINVAL;
+  }
+  return ASMV_OK;
+}
+
+bool tol_ok(const asmv_tol *tol) {
+  if (tol == nullptr) return false;
+  for (int d = 0; d <= ASMV_F8E4M3; ++d) {
+    if (std::isnan(tol[d].atol) || std::isnan(tol[d].rtol)) return false;
+    if (tol[d].atol < 0.0 || tol[d].rtol < 0.0) return false;
+  }
+  return true;
+}
+
+float round_down_f32(double x) {
+  float f = (float)x;
+  if ((double)f > x) f = std::nextafter(f, -INFINITY);
+  return f;
+}
+float round_up_f32(double x) {
+  float f = (float)x;
+  if ((double)f < x) f = std::nextafter(f, INFINITY);
+  return f;
+}
+
+// fp32 screen thresholds bracketing atol + rtol*|r| (see compare.cu).
+TolF make_tolf(const asmv_tol &t) {
+  TolF f;
+  const double lo_scale = 1.0 - 0x1p-21, hi_scale = 1.0 + 0x1p-21;
+  f.alo = (t.atol >= 0x1p-100) ? round_down_f32(t.atol * lo_scale) : -0x1p-100f;
+  f.rlo = round_down_f32(t.rtol * lo_scale);
+  f.ahi = round_up_f32(t.atol * hi_scale + 0x1p-100);
+  f.rhi = round_up_f32(t.rtol * hi_scale);
+  f.atol = t.atol;
+  f.rtol = t.rtol;
+  return f;
+}
+
+uint64_t tiles_of(uint64_t payload_bytes) { return (payload_bytes + kTileBytes - 1) / kTileBytes; }
+
+void add_guard_segments(std::vector<GuardSeg> &segs, uint64_t ptr, uint64_t offset, uint64_t len,
+                        uint8_t canary, uint8_t kind, uint32_t stats) {
+  for (uint64_t o = 0; o < len; o += kGuardSegBytes) {
+    GuardSeg g;
+    std::memset(&g, 0, sizeof g);
+    g.ptr = ptr + o;
+    g.offset = offset + o;
+    g.len = (uint32_t)std::min<uint64_t>(kGuardSegBytes, len - o);
+    g.stats = stats;
+    g.canary = canary;
+    g.kind = kind;
+    segs.push_back(g);
+  }
+}
+
+void add_region_guards(std::vector<GuardSeg> &segs, const asmv_region &r, uint8_t kind, uint32_t stats) {
+  uint64_t pb, tot;
+  region_extent(r, &pb, &tot);
+  if (r.guard_lo) add_guard_segments(segs, r.alloc, 0, r.guard_lo, r.canary, kind, stats);
+  if (r.guard_hi)
+    add_guard_segments(segs, r.alloc + r.guard_lo + pb, (uint64_t)r.guard_lo + pb, r.guard_hi,
+                       r.canary, kind, stats);
+}
+
+StatsDev empty_stats() {
+  StatsDev s;
+  s.mismatches = 0; s.first = ~0ull; s.abs_bits = 0; s.rel_bits = 0; s.nonfinite = 0;
+  s.guard_bad = 0; s.guard_first = ~0ull; s.ref_guard_bad = 0;
+  return s;
+}
+
+// Packs sections into one byte image with 256-byte aligned offsets.
+struct Image {
+  std::vector<unsigned char> bytes;
+  size_t add(const void *p, size_t n) {
+    const size_t off = (bytes.size() + 255) & ~(size_t)255;
+    bytes.resize(off + n);
+    if (n) std::memcpy(bytes.data() + off, p, n);
+    return off;
+  }
+};
+
+struct DeviceScope {
+  int prev = -1;
+  bool ok = false;
+  explicit DeviceScope(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceScope() { if (prev >= 0) cudaSetDevice(prev); }
+};
+
+}  // namespace
+
+struct asmv_ctx {
+  int device = 0;
+  int sms = 0;
+  int fill_ctas = 1, cmp1_ctas = 1, cmpk_ctas = 1;
+  void *dws = nullptr;
+  size_t dws_cap = 0;
+  unsigned char *hst = nullptr;
+  size_t hst_cap = 0;
+  cudaEvent_t staged = nullptr;   // previous upload of the staging buffer finished
+  cudaEvent_t ws_done = nullptr;  // previous kernel using the workspace finished
+  bool staged_pending = false, ws_pending = false;
+  int timing = 0;
+  bool timed = false;
+  cudaEvent_t t0 = nullptr, t1 = nullptr;
+  int cuda_err = 0;
+  uint64_t launches = 0;
+  AddrRangeFn addr_range = nullptr;
+};
+
+namespace {
+
+int fail_cuda(asmv_ctx *ctx, cudaError_t e) {
+  ctx->cuda_err = (int)e;
+  return (e == cudaErrorMemoryAllocation) ? ASMV_ENOMEM : ASMV_ECUDA;
+}
+
+// Every byte [alloc, alloc+total) must be device memory of ctx's device
+// inside one allocation.  `last` caches the most recent allocation range.
+int check_device_span(asmv_ctx *ctx, uint64_t alloc, uint64_t total,
+                      std::pair<uint64_t, uint64_t> &last) {
+  if (total == 0) return ASMV_OK;
+  if (alloc >= last.first && alloc + total <= last.second) return ASMV_OK;
+  cudaPointerAttributes a;
+  cudaError_t e = cudaPointerGetAttributes(&a, (const void *)alloc);
+  if (e != cudaSuccess) { cudaGetLastError(); return ASMV_EINVAL; }
+  if (a.type == cudaMemoryTypeDevice) {
+    if (a.device != ctx->device) return ASMV_EINVAL;
+  } else if (a.type != cudaMemoryTypeManaged) {
+    return ASMV_EINVAL;                              // host or unregistered memory
+  }
+  if (ctx->addr_range) {
+    unsigned long long base = 0;
+    size_t size = 0;
+    if (ctx->addr_range(&base, &size, alloc) != 0) return ASMV_EINVAL;
+    if (alloc + total > base + size) return ASMV_EINVAL;
+    last = std::make_pair((uint64_t)base, (uint64_t)(base + size));
+  }
+  return ASMV_OK;
+}
+
+int check_device_table(asmv_ctx *ctx, const asmv_region *regs, size_t n,
+                       std::pair<uint64_t, uint64_t> &last) {
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    region_extent(regs[i], &pb, &tot);
+    const int rc = check_device_span(ctx, regs[i].alloc, tot, last);
+    if (rc != ASMV_OK) return rc;
+  }
+  return ASMV_OK;
+}
+
+// Upload `img` (and reserve `readback` bytes of staging after it) to the
+// workspace on `s`; returns the device base in *dev.
+int stage(asmv_ctx *ctx, const Image &img, size_t readback, cudaStream_t s, unsigned char **dev) {
+  const size_t need_dev = std::max<size_t>(img.bytes.size(), 256);
+  const size_t need_host = ((img.bytes.size() + 255) & ~(size_t)255) + readback;
+  cudaError_t e;
+  if (ctx->staged_pending) {
+    if ((e = cudaEventSynchronize(ctx->staged)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->staged_pending = false;
+  }
+  if (need_host > ctx->hst_cap) {
+    const size_t cap = std::max(need_host, std::max((size_t)1 << 20, ctx->hst_cap * 2));
+    if (ctx->hst) cudaFreeHost(ctx->hst);
+    ctx->hst = nullptr;
+    ctx->hst_cap = 0;
+    if ((e = cudaHostAlloc((void **)&ctx->hst, cap, cudaHostAllocDefault)) != cudaSuccess) {
+      ctx->hst = nullptr;
+      fail_cuda(ctx, e);
+      return ASMV_ENOMEM;
+    }
+    ctx->hst_cap = cap;
+  }
+  if (need_dev > ctx->dws_cap) {
+    if (ctx->ws_pending) {
+      if ((e = cudaEventSynchronize(ctx->ws_done)) != cudaSuccess) return fail_cuda(ctx, e);
+      ctx->ws_pending = false;
+    }
+    const size_t cap = std::max(need_dev, std::max((size_t)1 << 20, ctx->dws_cap * 2));
+    if (ctx->dws) cudaFree(ctx->dws);
+    ctx->dws = nullptr;
+    ctx->dws_cap = 0;
+    if ((e = cudaMalloc(&ctx->dws, cap)) != cudaSuccess) {
+      ctx->dws = nullptr;
+      fail_cuda(ctx, e);
+      return ASMV_ENOMEM;
+    }
+    ctx->dws_cap = cap;
+  }
+  if (ctx->ws_pending && (e = cudaStreamWaitEvent(s, ctx->ws_done, 0)) != cudaSuccess)
+    return fail_cuda(ctx, e);
+  std::memcpy(ctx->hst, img.bytes.data(), img.bytes.size());
+  if ((e = cudaMemcpyAsync(ctx->dws, ctx->hst, img.bytes.size(), cudaMemcpyHostToDevice, s)) !=
+      cudaSuccess)
+    return fail_cuda(ctx, e);
+  if ((e = cudaEventRecord(ctx->staged, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  ctx->staged_pending = true;
+  *dev = (unsigned char *)ctx->dws;
+  return ASMV_OK;
+}
+
+int after_launch(asmv_ctx *ctx, cudaStream_t s) {
+  cudaError_t e;
+  if ((e = cudaEventRecord(ctx->ws_done, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  ctx->ws_pending = true;
+  return ASMV_OK;
+}
+
+int grid_for(asmv_ctx *ctx, uint64_t ntiles, size_t nsegs, int ctas_per_sm) {
+  const uint64_t cap = (uint64_t)ctx->sms * (uint64_t)ctas_per_sm;
+  uint64_t g = std::max<uint64_t>(ntiles, (nsegs + kWarps - 1) / kWarps);
+  g = std::min<uint64_t>(g, cap);
+  return (int)std::max<uint64_t>(g, 1);
+}
+
+// Read back k*n statistics from the workspace and finish the call.
+int readback(asmv_ctx *ctx, size_t stats_off, size_t img_bytes, size_t count, cudaStream_t s,
+             asmv_stats *out, size_t ref_n) {
+  cudaError_t e;
+  unsigned char *host = ctx->hst + ((img_bytes + 255) & ~(size_t)255);
+  if ((e = cudaMemcpyAsync(host, (unsigned char *)ctx->dws + stats_off, count * sizeof(StatsDev),
+                           cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+    return fail_cuda(ctx, e);
+  if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return fail_cuda(ctx, e);
+  ctx->staged_pending = false;
+  ctx->ws_pending = false;
+  std::memcpy(out, host, count * sizeof(asmv_stats));
+  if (ref_n) {
+    // reference-guard damage was accumulated in the first candidate's entries
+    for (size_t j = 1; j < count / ref_n; ++j)
+      for (size_t i = 0; i < ref_n; ++i) out[j * ref_n + i].ref_guard_bad_bytes = out[i].ref_guard_bad_bytes;
+  }
+  return ASMV_OK;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+int asmv_abi_version(void) { return ASMV_ABI_VERSION; }
+
+const char *asmv_strerror(int status) {
+  switch (status) {
+    case ASMV_OK: return "ok";
+    case ASMV_EINVAL: return "invalid argument or region table";
+    case ASMV_ECUDA: return "CUDA runtime error";
+    case ASMV_ETIMEOUT: return "bounded device wait expired";
+    case ASMV_ENOMEM: return "out of memory (workspace or staging)";
+    default: return "unknown status";
+  }
+}
+
+int asmv_check_regions(const asmv_region *regions, size_t n, int for_fill) {
+  return check_table(regions, n, for_fill != 0);
+}
+
+int asmv_ctx_create(asmv_ctx **out, int device) {
+  if (out == nullptr) return ASMV_EINVAL;
+  *out = nullptr;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess) { cudaGetLastError(); return ASMV_ECUDA; }
+  if (device < 0 || device >= ndev) return ASMV_EINVAL;
+  asmv_ctx *ctx = new (std::nothrow) asmv_ctx();
+  if (!ctx) return ASMV_ENOMEM;
+  ctx->device = device;
+  DeviceScope ds(device);
+  cudaError_t e = cudaSuccess;
+  if (!ds.ok) e = cudaErrorInvalidDevice;
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, device);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->staged, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->ws_done, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreate(&ctx->t0);
+  if (e == cudaSuccess) e = cudaEventCreate(&ctx->t1);
+  if (e != cudaSuccess) {
+    asmv_ctx_destroy(ctx);
+    return ASMV_ECUDA;
+  }
+  ctx->fill_ctas = fill_max_ctas_per_sm();
+  ctx->cmp1_ctas = compare_max_ctas_per_sm(1);
+  ctx->cmpk_ctas = compare_max_ctas_per_sm(kMaxCands);
+  void *fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &fn, 12000, cudaEnableDefault, &q) ==
+          cudaSuccess && q == cudaDriverEntryPointSuccess)
+    ctx->addr_range = (AddrRangeFn)fn;
+  else
+    cudaGetLastError();
+  *out = ctx;
+  return ASMV_OK;
+}
+
+void asmv_ctx_destroy(asmv_ctx *ctx) {
+  if (ctx == nullptr) return;
+  DeviceScope ds(ctx->device);
+  if (ctx->ws_pending) cudaEventSynchronize(ctx->ws_done);
+  if (ctx->staged_pending) cudaEventSynchronize(ctx->staged);
+  if (ctx->dws) cudaFree(ctx->dws);
+  if (ctx->hst) cudaFreeHost(ctx->hst);
+  if (ctx->staged) cudaEventDestroy(ctx->staged);
+  if (ctx->ws_done) cudaEventDestroy(ctx->ws_done);
+  if (ctx->t0) cudaEventDestroy(ctx->t0);
+  if (ctx->t1) cudaEventDestroy(ctx->t1);
+  delete ctx;
+}
+
+int asmv_ctx_set_timing(asmv_ctx *ctx, int enable) {
+  if (ctx == nullptr) return ASMV_EINVAL;
+  ctx->timing = enable != 0;
+  ctx->timed = false;
+  return ASMV_OK;
+}
+
+int asmv_ctx_kernel_ms(asmv_ctx *ctx, float *ms) {
+  if (ctx == nullptr || ms == nullptr || !ctx->timing || !ctx->timed) return ASMV_EINVAL;
+  DeviceScope ds(ctx->device);
+  cudaError_t e = cudaEventSynchronize(ctx->t1);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(ms, ctx->t0, ctx->t1);
+  return e == cudaSuccess ? ASMV_OK : fail_cuda(ctx, e);
+}
+
+int asmv_ctx_cuda_error(const asmv_ctx *ctx) { return ctx ? ctx->cuda_err : 0; }
+
+uint64_t asmv_ctx_launches(const asmv_ctx *ctx) { return ctx ? ctx->launches : 0; }
+
+int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed,
+              asmv_stream_t stream) {
+  if (ctx == nullptr) return ASMV_EINVAL;
+  int rc = check_table(regions, n, true);
+  if (rc != ASMV_OK) return rc;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  std::pair<uint64_t, uint64_t> last(0, 0);
+  if ((rc = check_device_table(ctx, regions, n, last)) != ASMV_OK) return rc;
+
+  std::vector<FillRegion> fr(n + 1);
+  std::vector<GuardSeg> segs;
+  uint64_t tile = 0;
+  for (size_t i = 0; i < n; ++i) {
+    const asmv_region &r = regions[i];
+    uint64_t pb, tot;
+    region_extent(r, &pb, &tot);
+    FillRegion &f = fr[i];
+    std::memset(&f, 0, sizeof f);
+    f.payload = r.alloc + r.guard_lo;
+    f.bytes = (r.dist == ASMV_DIST_NONE) ? 0 : pb;
+    f.tile0 = tile;
+    f.dtype = r.dtype;
+    f.dist = r.dist;
+    f.region_id = r.region_id;
+    f.vec = (f.payload % 16) == 0;
+    if (r.dist == ASMV_DIST_UNIFORM) {
+      f.f0 = (float)r.p0;
+      f.f1 = (float)r.p1 - f.f0;
+    } else if (r.dist == ASMV_DIST_NORMAL) {
+      f.f0 = (float)r.p0;
+      f.f1 = (float)r.p1;
+    } else if (r.dist == ASMV_DIST_INT_RANGE) {
+      f.ilo = (int64_t)r.p0;
+      f.ispan = (uint64_t)((int64_t)r.p1 - (int64_t)r.p0);
+    }
+    tile += tiles_of(f.bytes);
+    add_region_guards(segs, r, kSegFill, (uint32_t)i);
+  }
+  std::memset(&fr[n], 0, sizeof(FillRegion));
+  fr[n].tile0 = tile;
+  if (tile == 0 && segs.empty()) return ASMV_OK;
+
+  Image img;
+  const size_t o_regs = img.add(fr.data(), fr.size() * sizeof(FillRegion));
+  const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
+  unsigned char *dev = nullptr;
+  cudaStream_t s = (cudaStream_t)stream;
+  if ((rc = stage(ctx, img, 0, s, &dev)) != ASMV_OK) return rc;
+  FillParams p;
+  p.regions = (const FillRegion *)(dev + o_regs);
+  p.segs = (const GuardSeg *)(dev + o_segs);
+  p.ntiles = tile;
+  p.seed = seed;
+  p.nregions = (uint32_t)n;
+  p.nsegs = (uint32_t)segs.size();
+  cudaError_t e;
+  if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  if ((e = (cudaError_t)launch_fill(p, grid_for(ctx, tile, segs.size(), ctx->fill_ctas), s)) !=
+      cudaSuccess)
+    return fail_cuda(ctx, e);
+  ctx->launches += 1;
+  if (ctx->timing) {
+    if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->timed = true;
+  }
+  return after_launch(ctx, s);
+}
+
+// Shared body of guard_check / compare / compare_batched.
+static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                       size_t k, size_t n, const asmv_tol *tol, asmv_stats *out, cudaStream_t s,
+                       bool guard_only) {
+  std::pair<uint64_t, uint64_t> last(0, 0);
+  int rc;
+  if ((rc = check_device_table(ctx, ref, n, last)) != ASMV_OK) return rc;
+  for (size_t j = 0; j < k && !guard_only; ++j)
+    if ((rc = check_device_table(ctx, cands[j], n, last)) != ASMV_OK) return rc;
+
+  std::vector<CmpRegion> cr(n + 1);
+  std::vector<uint64_t> caddr(guard_only ? 0 : k * n);
+  std::vector<GuardSeg> segs;
+  uint64_t tile = 0;
+  for (size_t i = 0; i < n; ++i) {
+    const asmv_region &r = ref[i];
+    uint64_t pb, tot;
+    region_extent(r, &pb, &tot);
+    CmpRegion &c = cr[i];
+    std::memset(&c, 0, sizeof c);
+    c.ref = r.alloc + r.guard_lo;
+    c.bytes = guard_only ? 0 : pb;
+    c.tile0 = tile;
+    c.dtype = r.dtype;
+    bool vec = (c.ref % 16) == 0;
+    for (size_t j = 0; j < caddr.size() / (n ? n : 1); ++j) {
+      const uint64_t a = cands[j][i].alloc + cands[j][i].guard_lo;
+      caddr[j * n + i] = a;
+      vec = vec && (a % 16) == 0;
+    }
+    c.vec = vec;
+    tile += tiles_of(c.bytes);
+    if (guard_only) {
+      add_region_guards(segs, r, kSegSelf, (uint32_t)i);
+    } else {
+      add_region_guards(segs, r, kSegRef, (uint32_t)i);
+      for (size_t j = 0; j < k; ++j) add_region_guards(segs, cands[j][i], kSegCand, (uint32_t)(j * n + i));
+    }
+  }
+  std::memset(&cr[n], 0, sizeof(CmpRegion));
+  cr[n].tile0 = tile;
+  const size_t nstats = guard_only ? n : k * n;
+  if (nstats == 0) return ASMV_OK;
+  std::vector<StatsDev> st(nstats, empty_stats());
+
+  Image img;
+  const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CmpRegion));
+  const size_t o_cand = img.add(caddr.data(), caddr.size() * sizeof(uint64_t));
+  const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
+  const size_t o_stats = img.add(st.data(), st.size() * sizeof(StatsDev));
+  unsigned char *dev = nullptr;
+  if ((rc = stage(ctx, img, nstats * sizeof(StatsDev), s, &dev)) != ASMV_OK) return rc;
+
+  CmpParams p;
+  std::memset(&p, 0, sizeof p);
+  p.regions = (const CmpRegion *)(dev + o_regs);
+  p.segs = (const GuardSeg *)(dev + o_segs);
+  p.seg_stats = (StatsDev *)(dev + o_stats);
+  p.ntiles = tile;
+  p.nregions = (uint32_t)n;
+  for (int d = 0; d < 7; ++d) {
+    if (is_float((uint32_t)d) && tol) p.tol[d] = make_tolf(tol[d]);
+  }
+  cudaError_t e;
+  if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  const size_t groups = guard_only ? 1 : (k + kMaxCands - 1) / kMaxCands;
+  for (size_t g = 0; g < groups; ++g) {
+    const size_t kg = guard_only ? 1 : std::min<size_t>(kMaxCands, k - g * kMaxCands);
+    p.K = (uint32_t)kg;
+    p.cands = (const uint64_t *)(dev + o_cand) + g * kMaxCands * n;
+    p.stats = (StatsDev *)(dev + o_stats) + g * kMaxCands * n;
+    p.nsegs = (g == 0) ? (uint32_t)segs.size() : 0u;
+    if (guard_only) p.ntiles = 0;
+    const int ctas = (kg > 1) ? ctx->cmpk_ctas : ctx->cmp1_ctas;
+    if ((e = (cudaError_t)launch_compare(p, grid_for(ctx, p.ntiles, p.nsegs, ctas), s)) != cudaSuccess)
+      return fail_cuda(ctx, e);
+    ctx->launches += 1;
+  }
+  if (ctx->timing) {
+    if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->timed = true;
+  }
+  if ((rc = after_launch(ctx, s)) != ASMV_OK) return rc;
+  return readback(ctx, o_stats, img.bytes.size(), nstats, s, out, guard_only ? 0 : n);
+}
+
+int asmv_guard_check(asmv_ctx *ctx, const asmv_region *regions, size_t n, asmv_stats *out_host,
+                     asmv_stream_t stream) {
+  if (ctx == nullptr || (n > 0 && out_host == nullptr)) return ASMV_EINVAL;
+  int rc = check_table(regions, n, false);
+  if (rc != ASMV_OK) return rc;
+  if (n == 0) return ASMV_OK;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  return run_compare(ctx, regions, nullptr, 0, n, nullptr, out_host, (cudaStream_t)stream, true);
+}
+
+static int check_pairs(const asmv_region *ref, const asmv_region *const *cands, size_t k, size_t n) {
+  int rc = check_table(ref, n, false);
+  if (rc != ASMV_OK) return rc;
+  for (size_t j = 0; j < k; ++j) {
+    if (n > 0 && cands[j] == nullptr) return ASMV_EINVAL;
+    if ((rc = check_table(cands[j], n, false)) != ASMV_OK) return rc;
+    for (size_t i = 0; i < n; ++i)
+      if (cands[j][i].dtype != ref[i].dtype || cands[j][i].n_elems != ref[i].n_elems)
+        return ASMV_EINVAL;
+  }
+  return ASMV_OK;
+}
+
+int asmv_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cand, size_t n,
+                 const asmv_tol *tol, asmv_stats *out_host, asmv_stream_t stream) {
+  if (ctx == nullptr || (n > 0 && (out_host == nullptr || cand == nullptr)) || !tol_ok(tol))
+    return ASMV_EINVAL;
+  const asmv_region *cands[1] = {cand};
+  int rc = check_pairs(ref, cands, 1, n);
+  if (rc != ASMV_OK) return rc;
+  if (n == 0) return ASMV_OK;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  return run_compare(ctx, ref, cands, 1, n, tol, out_host, (cudaStream_t)stream, false);
+}
+
+int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                         size_t k, size_t n, const asmv_tol *tol, asmv_stats *out_host,
+                         asmv_stream_t stream) {
+  if (ctx == nullptr || k == 0 || cands == nullptr || (n > 0 && out_host == nullptr) || !tol_ok(tol))
+    return ASMV_EINVAL;
+  if (k > (size_t)0x7FFFFFFF / (n ? n : 1)) return ASMV_EINVAL;
+  int rc = check_pairs(ref, cands, k, n);
+  if (rc != ASMV_OK) return rc;
+  if (n == 0) return ASMV_OK;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  return run_compare(ctx, ref, cands, k, n, tol, out_host, (cudaStream_t)stream, false);
+}
+
+}  // extern "C"

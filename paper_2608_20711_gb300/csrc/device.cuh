@@ -1,0 +1,197 @@
+// device.cuh -- device building blocks of the fill and compare kernels.
+//
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) and the fp32 Box-Muller
+// transform used for the NORMAL distribution of the Tier 1 fill (AsmEvo
+// Sec. 3.4).  Every floating-point step uses an explicit _rn intrinsic so
+// that nvcc cannot contract or reorder it; the sequence of IEEE operations
+// is the one the library's specification states, which makes the filled
+// bytes reproducible on any IEEE machine.
+#pragma once
+#include <stdint.h>
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+#include <cuda_fp8.h>
+#include "plan.h"
+
+namespace asmv {
+
+// ---------------------------------------------------------------- Philox
+// Round: (x0,x1,x2,x3) -> (hi(B*x2)^x1^k0, B*x2, hi(A*x0)^x3^k1, A*x0) with
+// A = 0xD2511F53, B = 0xCD9E8D57; key bumped by the Weyl increments
+// 0x9E3779B9 / 0xBB67AE85 between rounds (SC'11, Sec. 3).
+__device__ __forceinline__ uint4 philox10(uint4 x, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) { k0 += 0x9E3779B9u; k1 += 0xBB67AE85u; }
+    const uint32_t a_hi = __umulhi(0xD2511F53u, x.x), a_lo = 0xD2511F53u * x.x;
+    const uint32_t b_hi = __umulhi(0xCD9E8D57u, x.z), b_lo = 0xCD9E8D57u * x.z;
+    x = make_uint4(b_hi ^ x.y ^ k0, b_lo, a_hi ^ x.w ^ k1, a_lo);
+  }
+  return x;
+}
+
+// Block `b` of a region's payload stream.
+__device__ __forceinline__ uint4 payload_block(uint64_t seed, uint32_t region_id, uint64_t b) {
+  return philox10(make_uint4((uint32_t)b, (uint32_t)(b >> 32), region_id, 0u),
+                  (uint32_t)seed, (uint32_t)(seed >> 32));
+}
+
+// ---------------------------------------------------------------- Box-Muller
+// Series coefficients, each the fp32 rounding of the exact value:
+//   ln(m) = 2s (1 + s^2/3 + s^4/5 + ... + s^10/11),  s = (m-1)/(m+1)
+//   sin(pi/2 r) = sum_k (-1)^k (pi/2)^(2k+1) r^(2k+1) / (2k+1)!,  k = 0..4
+//   cos(pi/2 r) = sum_k (-1)^k (pi/2)^(2k) r^(2k) / (2k)!,        k = 0..5
+// ln 2 is split Cody-Waite style into 355/512 and the fp32 rounding of the
+// remainder.
+#define ASMV_LN2_HI 0x1.63p-1f
+#define ASMV_LN2_LO (-0x1.bd0106p-13f)
+#define ASMV_AT3 0x1.555556p-2f
+#define ASMV_AT5 0x1.99999ap-3f
+#define ASMV_AT7 0x1.24924ap-3f
+#define ASMV_AT9 0x1.c71c72p-4f
+#define ASMV_AT11 0x1.745d18p-4f
+#define ASMV_S1 0x1.921fb6p+0f
+#define ASMV_S3 (-0x1.4abbcep-1f)
+#define ASMV_S5 0x1.466bc6p-4f
+#define ASMV_S7 (-0x1.32d2ccp-8f)
+#define ASMV_S9 0x1.507834p-13f
+#define ASMV_C2 (-0x1.3bd3ccp+0f)
+#define ASMV_C4 0x1.03c1f0p-2f
+#define ASMV_C6 (-0x1.55d3c8p-6f)
+#define ASMV_C8 0x1.e1f506p-11f
+#define ASMV_C10 (-0x1.a6d1f2p-16f)
+// fp32 nearest to sqrt(2): reduction threshold for the mantissa
+#define ASMV_SQRT2 0x1.6a09e6p+0f
+
+// ln(k 2^-24) for k in [1, 2^24]: exponent/mantissa split, mantissa folded
+// into [sqrt2/2, sqrt2], atanh series, e*ln2 added back in two parts.
+__device__ __forceinline__ float ln_u24(uint32_t k) {
+  const float u = __fmul_rn(__uint2float_rn(k), 0x1p-24f);   // exact
+  const uint32_t bits = __float_as_uint(u);
+  int e = (int)(bits >> 23) - 127;
+  float m = __uint_as_float((bits & 0x7FFFFFu) | 0x3F800000u);
+  if (m > ASMV_SQRT2) { m = __fmul_rn(m, 0.5f); e += 1; }
+  const float f = __fsub_rn(m, 1.0f);
+  const float s = __fdiv_rn(f, __fadd_rn(2.0f, f));
+  const float z = __fmul_rn(s, s);
+  float p = __fmaf_rn(z, ASMV_AT11, ASMV_AT9);
+  p = __fmaf_rn(z, p, ASMV_AT7);
+  p = __fmaf_rn(z, p, ASMV_AT5);
+  p = __fmaf_rn(z, p, ASMV_AT3);
+  const float s2 = __fadd_rn(s, s);
+  const float lnm = __fmaf_rn(__fmul_rn(s2, z), p, s2);
+  const float ef = (float)e;
+  return __fmaf_rn(ef, ASMV_LN2_HI, __fmaf_rn(ef, ASMV_LN2_LO, lnm));
+}
+
+// sin and cos of 2 pi k 2^-24, k in [0, 2^24): nearest quarter turn q
+// removed exactly in integers, the remainder r in [-1/2, 1/2) quarter turns.
+__device__ __forceinline__ void sincos_u24(uint32_t k, float &sn, float &cs) {
+  const uint32_t q = (k + (1u << 21)) >> 22;
+  const int32_t ri = (int32_t)k - (int32_t)(q << 22);
+  const float r = __fmul_rn((float)ri, 0x1p-22f);
+  const float r2 = __fmul_rn(r, r);
+  float sp = __fmaf_rn(r2, ASMV_S9, ASMV_S7);
+  sp = __fmaf_rn(r2, sp, ASMV_S5);
+  sp = __fmaf_rn(r2, sp, ASMV_S3);
+  sp = __fmaf_rn(r2, sp, ASMV_S1);
+  const float s = __fmul_rn(r, sp);
+  float cp = __fmaf_rn(r2, ASMV_C10, ASMV_C8);
+  cp = __fmaf_rn(r2, cp, ASMV_C6);
+  cp = __fmaf_rn(r2, cp, ASMV_C4);
+  cp = __fmaf_rn(r2, cp, ASMV_C2);
+  const float c = __fmaf_rn(r2, cp, 1.0f);
+  switch (q & 3u) {
+    case 0: sn = s; cs = c; break;
+    case 1: sn = c; cs = -s; break;
+    case 2: sn = -s; cs = -c; break;
+    default: sn = -c; cs = s; break;
+  }
+}
+
+__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, float &z0, float &z1) {
+  const float l = ln_u24((w0 >> 8) + 1u);
+  const float rho = __fsqrt_rn(__fmul_rn(-2.0f, l));
+  float sn, cs;
+  sincos_u24(w1 >> 8, sn, cs);
+  z0 = __fmul_rn(rho, cs);
+  z1 = __fmul_rn(rho, sn);
+}
+
+// ---------------------------------------------------------------- encoders
+// Hardware round-to-nearest-even conversions (fp8: saturating to +-448).
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  const __nv_bfloat16 x = __float2bfloat16_rn(a), y = __float2bfloat16_rn(b);
+  return (uint32_t)__bfloat16_as_ushort(x) | ((uint32_t)__bfloat16_as_ushort(y) << 16);
+}
+__device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
+  const __half x = __float2half_rn(a), y = __float2half_rn(b);
+  return (uint32_t)__half_as_ushort(x) | ((uint32_t)__half_as_ushort(y) << 16);
+}
+__device__ __forceinline__ uint32_t pack_f8x4(float a, float b, float c, float d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c, d), __NV_SATFINITE, __NV_E4M3);
+  return (lo & 0xFFFFu) | (hi << 16);
+}
+
+// ---------------------------------------------------------------- decoders
+__device__ __forceinline__ float2 f16x2_to_f32(uint32_t w) {
+  return __half22float2(*reinterpret_cast<const __half2 *>(&w));
+}
+__device__ __forceinline__ float2 f8x2_to_f32(uint32_t w16) {
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(w16 & 0xFFFFu), __NV_E4M3);
+  uint32_t u = (uint32_t)h.x | ((uint32_t)h.y << 16);
+  return f16x2_to_f32(u);
+}
+
+// ---------------------------------------------------------------- integers
+__device__ __forceinline__ unsigned long long umin64(unsigned long long a, unsigned long long b) {
+  return a < b ? a : b;
+}
+__device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
+  return a > b ? a : b;
+}
+
+// ---------------------------------------------------------------- memory
+__device__ __forceinline__ uint4 ldg16(uint64_t addr) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(addr));
+  return v;
+}
+__device__ __forceinline__ void stg16(uint64_t addr, uint4 v) {
+  asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};"
+               :: "l"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+}
+
+// Up to 16 bytes at any alignment; bytes past `n` read as zero.
+__device__ __forceinline__ uint4 load_bytes(uint64_t addr, uint32_t n) {
+  uint32_t w[4] = {0u, 0u, 0u, 0u};
+  const uint8_t *p = reinterpret_cast<const uint8_t *>(addr);
+#pragma unroll
+  for (uint32_t j = 0; j < 16; ++j)
+    if (j < n) w[j >> 2] |= (uint32_t)__ldg(p + j) << (8 * (j & 3));
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+__device__ __forceinline__ void store_bytes(uint64_t addr, uint4 v, uint32_t n) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint8_t *p = reinterpret_cast<uint8_t *>(addr);
+#pragma unroll
+  for (uint32_t j = 0; j < 16; ++j)
+    if (j < n) p[j] = (uint8_t)(w[j >> 2] >> (8 * (j & 3)));
+}
+
+// Region owning tile t: the last i with tile0[i] <= t (regions with no
+// tiles share their successor's tile0 and are skipped).
+template <class R>
+__device__ __forceinline__ uint32_t find_region(const R *regs, uint32_t n, uint64_t t) {
+  uint32_t lo = 0, hi = n;          // invariant: regs[lo].tile0 <= t < regs[hi].tile0
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (regs[mid].tile0 <= t) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+}  // namespace asmv

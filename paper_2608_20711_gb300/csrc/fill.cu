@@ -1,0 +1,175 @@
+// fill.cu -- Tier 1 guarded input synthesis (AsmEvo Sec. 3.4, Tier 1):
+// every region's payload receives its seeded Philox4x32-10 stream shaped to
+// its distribution, and both guard bands receive the region's canary byte.
+//
+// One 16-byte chunk c of a payload always holds the same bytes, whatever
+// the payload's address: RAW chunk c is Philox block c; other distributions
+// map element i to word (i mod 4) of block (i div 4) (NORMAL: Box-Muller on
+// word pairs (0,1) and (2,3)).  Aligned payloads are written with 128-bit
+// stores; unaligned payloads and the short last chunk with byte stores.
+//
+// Roofline: HBM writes of payload + guard bytes; Philox (about 80 integer
+// operations per 16-byte block) and Box-Muller for NORMAL also load the
+// ALUs, so 16-bit and 8-bit NORMAL fills are arithmetic-bound.
+#include "device.cuh"
+
+namespace asmv {
+namespace {
+
+__device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
+  const float f = __fmul_rn(__uint2float_rn(w >> 8), 0x1p-24f);
+  return __fadd_rn(lo, __fmul_rn(f, width));
+}
+
+__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, float v[4]) {
+  float z[4];
+  box_muller(w.x, w.y, z[0], z[1]);
+  box_muller(w.z, w.w, z[2], z[3]);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) v[j] = __fadd_rn(mean, __fmul_rn(sd, z[j]));
+}
+
+__device__ __forceinline__ void uniform4(uint4 w, float lo, float width, float v[4]) {
+  v[0] = uniform_of(w.x, lo, width);
+  v[1] = uniform_of(w.y, lo, width);
+  v[2] = uniform_of(w.z, lo, width);
+  v[3] = uniform_of(w.w, lo, width);
+}
+
+__device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span) {
+  return (uint32_t)(lo + (int64_t)(((uint64_t)w * span) >> 32));
+}
+
+// Four fp32 values of one block, per float distribution.
+template <uint32_t DIST>
+__device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, float v[4]) {
+  if (DIST == kNormal) normal4(w, r.f0, r.f1, v);
+  else uniform4(w, r.f0, r.f1, v);
+}
+
+// The 16 bytes of chunk c.
+template <uint32_t DIST, uint32_t DT>
+__device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, uint64_t c) {
+  if (DIST == kRaw) return payload_block(seed, r.region_id, c);
+  if (DIST == kIntRange) {
+    if (DT == kI32) {
+      const uint4 w = payload_block(seed, r.region_id, c);
+      return make_uint4(int_of(w.x, r.ilo, r.ispan), int_of(w.y, r.ilo, r.ispan),
+                        int_of(w.z, r.ilo, r.ispan), int_of(w.w, r.ilo, r.ispan));
+    } else {                                    // 8-bit: 16 elements, blocks 4c..4c+3
+      uint32_t out[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 w = payload_block(seed, r.region_id, 4 * c + q);
+        out[q] = (int_of(w.x, r.ilo, r.ispan) & 0xFFu) | ((int_of(w.y, r.ilo, r.ispan) & 0xFFu) << 8) |
+                 ((int_of(w.z, r.ilo, r.ispan) & 0xFFu) << 16) | (int_of(w.w, r.ilo, r.ispan) << 24);
+      }
+      return make_uint4(out[0], out[1], out[2], out[3]);
+    }
+  }
+  // UNIFORM / NORMAL on float dtypes
+  if (DT == kF32) {
+    float v[4];
+    float4_of<DIST>(payload_block(seed, r.region_id, c), r, v);
+    return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                      __float_as_uint(v[3]));
+  } else if (DT == kBF16 || DT == kF16) {       // 8 elements: blocks 2c, 2c+1
+    uint32_t out[4];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      float v[4];
+      float4_of<DIST>(payload_block(seed, r.region_id, 2 * c + q), r, v);
+      if (DT == kBF16) { out[2 * q] = pack_bf16x2(v[0], v[1]); out[2 * q + 1] = pack_bf16x2(v[2], v[3]); }
+      else { out[2 * q] = pack_f16x2(v[0], v[1]); out[2 * q + 1] = pack_f16x2(v[2], v[3]); }
+    }
+    return make_uint4(out[0], out[1], out[2], out[3]);
+  } else {                                      // fp8: 16 elements, blocks 4c..4c+3
+    uint32_t out[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float v[4];
+      float4_of<DIST>(payload_block(seed, r.region_id, 4 * c + q), r, v);
+      out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
+    }
+    return make_uint4(out[0], out[1], out[2], out[3]);
+  }
+}
+
+template <uint32_t DIST, uint32_t DT>
+__device__ void fill_tile(const FillRegion &r, uint64_t seed, uint64_t tile_in_region) {
+  const uint64_t c0 = tile_in_region * kTileChunks;
+  const uint64_t nchunks = (r.bytes + 15) >> 4;
+  const uint64_t full = r.bytes >> 4;
+  const uint32_t nloc = (uint32_t)umin64(kTileChunks, nchunks - c0);
+  for (uint32_t i = threadIdx.x; i < nloc; i += kThreads) {
+    const uint64_t c = c0 + i;
+    const uint4 v = make_chunk<DIST, DT>(r, seed, c);
+    const uint64_t addr = r.payload + 16 * c;
+    if (r.vec && c < full) stg16(addr, v);
+    else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * c));
+  }
+}
+
+__device__ void fill_tile_dispatch(const FillRegion &r, uint64_t seed, uint64_t t) {
+  switch (r.dist) {
+    case kRaw: fill_tile<kRaw, kU8>(r, seed, t); break;
+    case kIntRange:
+      if (r.dtype == kI32) fill_tile<kIntRange, kI32>(r, seed, t);
+      else fill_tile<kIntRange, kI8>(r, seed, t);
+      break;
+    case kUniform:
+      switch (r.dtype) {
+        case kF32: fill_tile<kUniform, kF32>(r, seed, t); break;
+        case kBF16: fill_tile<kUniform, kBF16>(r, seed, t); break;
+        case kF16: fill_tile<kUniform, kF16>(r, seed, t); break;
+        default: fill_tile<kUniform, kF8>(r, seed, t); break;
+      }
+      break;
+    case kNormal:
+      switch (r.dtype) {
+        case kF32: fill_tile<kNormal, kF32>(r, seed, t); break;
+        case kBF16: fill_tile<kNormal, kBF16>(r, seed, t); break;
+        case kF16: fill_tile<kNormal, kF16>(r, seed, t); break;
+        default: fill_tile<kNormal, kF8>(r, seed, t); break;
+      }
+      break;
+    default: break;                              // NONE: payload untouched
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) fill_kernel(const FillParams p) {
+  const uint64_t G = gridDim.x, b = blockIdx.x;
+  const uint64_t t0 = p.ntiles * b / G, t1 = p.ntiles * (b + 1) / G;
+  if (t0 < t1) {
+    uint32_t ri = find_region(p.regions, p.nregions, t0);
+    for (uint64_t t = t0; t < t1; ++t) {
+      while (p.regions[ri + 1].tile0 <= t) ++ri;
+      const FillRegion r = p.regions[ri];
+      fill_tile_dispatch(r, p.seed, t - r.tile0);
+    }
+  }
+  // guard bands: one warp per segment
+  const uint32_t lane = threadIdx.x & 31;
+  const uint64_t warp = b * kWarps + (threadIdx.x >> 5), nw = G * kWarps;
+  for (uint64_t s = warp; s < p.nsegs; s += nw) {
+    const GuardSeg g = p.segs[s];
+    uint8_t *dst = reinterpret_cast<uint8_t *>(g.ptr);
+    for (uint32_t j = lane; j < g.len; j += 32) dst[j] = g.canary;
+  }
+}
+
+}  // namespace
+
+int fill_max_ctas_per_sm() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fill_kernel, kThreads, 0) != cudaSuccess)
+    return 1;
+  return n > 0 ? n : 1;
+}
+
+int launch_fill(const FillParams &p, int grid, void *stream) {
+  fill_kernel<<<grid, kThreads, 0, (cudaStream_t)stream>>>(p);
+  return (int)cudaGetLastError();
+}
+
+}  // namespace asmv

@@ -1,0 +1,111 @@
+// plan.h -- launch descriptors shared by the host ABI layer (abi.cu) and
+// the kernels (fill.cu, compare.cu).  Internal to the library.
+//
+// Work decomposition.  Every region's payload is cut into tiles of
+// kTileBytes (the last tile of a region may be short).  Tiles of all
+// regions form one index space; region i owns tiles [tile0[i], tile0[i+1]).
+// A launch runs a persistent grid; CTA b takes the contiguous tile range
+// [T*b/G, T*(b+1)/G), so a CTA crosses few region boundaries and flushes its
+// per-region partial statistics once per boundary.  Inside a tile, thread t
+// handles 16-byte chunks t, t+256, ... (coalesced 128-bit accesses).
+//
+// Guard bands are cut into segments of at most kGuardSegBytes and handled
+// one warp per segment after the payload tiles.
+#pragma once
+#include <stdint.h>
+
+namespace asmv {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kChunkBytes = 16;
+constexpr int kTileChunks = 1024;
+constexpr uint64_t kTileBytes = (uint64_t)kChunkBytes * kTileChunks;  // 16 KiB
+constexpr uint32_t kGuardSegBytes = 4096;
+constexpr int kMaxCands = 8;            // candidates per batched launch
+
+enum : uint32_t { kF32 = 0, kBF16 = 1, kF16 = 2, kF8 = 3, kI32 = 4, kI8 = 5, kU8 = 6 };
+enum : uint32_t { kRaw = 0, kUniform = 1, kNormal = 2, kIntRange = 3, kNone = 4 };
+enum : uint32_t { kSegFill = 0, kSegSelf = 1, kSegCand = 2, kSegRef = 3 };
+
+// One region of a fill launch (64 B).
+struct FillRegion {
+  uint64_t payload;     // device address of element 0
+  uint64_t bytes;       // payload bytes
+  uint64_t tile0;       // first tile; the table has a sentinel entry after the last region
+  uint32_t dtype, dist;
+  uint32_t region_id;
+  uint32_t vec;         // payload is 16-byte aligned
+  float f0, f1;         // UNIFORM: lo, width; NORMAL: mean, std (fp32)
+  int64_t ilo;          // INT_RANGE: lo
+  uint64_t ispan;       // INT_RANGE: hi - lo
+};
+
+// One region of a compare launch (32 B).  Candidate payload addresses live
+// in a separate [K][nregions] array.
+struct CmpRegion {
+  uint64_t ref;         // reference payload address
+  uint64_t bytes;       // payload bytes
+  uint64_t tile0;
+  uint32_t dtype;
+  uint32_t vec;         // reference and every candidate payload 16-byte aligned
+};
+
+// A guard band segment (32 B).
+struct GuardSeg {
+  uint64_t ptr;         // first byte of the segment
+  uint64_t offset;      // its offset from the allocation start
+  uint32_t len;         // bytes (<= kGuardSegBytes)
+  uint32_t stats;       // index into the statistics array
+  uint8_t canary;
+  uint8_t kind;         // kSeg*
+  uint8_t pad_[6];
+};
+
+// fp32 screening thresholds and exact fp64 tolerances of one float dtype.
+// alo/rlo bound atol + rtol*|r| from below, ahi/rhi from above, with a
+// relative margin of 2^-21 and an absolute slack of 2^-100 (the proof of the
+// screen is in compare.cu).
+struct TolF {
+  float alo, rlo, ahi, rhi;
+  double atol, rtol;
+};
+
+// Device statistics entry; bit-compatible with asmv_stats (the two maxima
+// are non-negative doubles kept as their bit patterns, so that integer
+// atomicMax orders them).
+struct StatsDev {
+  unsigned long long mismatches, first, abs_bits, rel_bits, nonfinite;
+  unsigned long long guard_bad, guard_first, ref_guard_bad;
+};
+
+struct FillParams {
+  const FillRegion *regions;   // nregions + 1 entries (sentinel)
+  const GuardSeg *segs;
+  uint64_t ntiles;
+  uint64_t seed;
+  uint32_t nregions;
+  uint32_t nsegs;
+};
+
+struct CmpParams {
+  const CmpRegion *regions;    // nregions + 1 entries (sentinel)
+  const uint64_t *cands;       // [K][nregions] candidate payload addresses
+  const GuardSeg *segs;
+  StatsDev *stats;             // [K][nregions] (this launch's candidates)
+  StatsDev *seg_stats;         // guard segments index from here
+  uint64_t ntiles;
+  uint32_t nregions;
+  uint32_t nsegs;
+  uint32_t K;
+  uint32_t pad_;
+  TolF tol[7];
+};
+
+// Launchers (defined in fill.cu / compare.cu).  Return a cudaError_t.
+int launch_fill(const FillParams &p, int grid, void *stream);
+int launch_compare(const CmpParams &p, int grid, void *stream);
+int fill_max_ctas_per_sm();
+int compare_max_ctas_per_sm(int K);
+
+}  // namespace asmv
