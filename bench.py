@@ -152,20 +152,21 @@ class Setup:
         rng = np.random.default_rng(wl.seed + 77)
         self.cands = []
         ncand = wl.n_cands
+        recipe = wl.name               # the recipe, shared by the size variants
         for j in range(ncand):
             c = self.ref.clone()
-            if name == "batched_gemm_fp16":
+            if recipe == "batched_gemm_fp16":
                 W.perturb_uniform_ulps(c, wl.regions[0], seed=wl.seed * 100 + j,
                                        magnitude=wl.ulp_magnitudes[j])
-            elif name == "fp32_1m":
+            elif recipe == "fp32_1m":
                 W.perturb_fp32_single(c, wl)
-            elif name == "attention_bf16":
+            elif recipe == "attention_bf16":
                 for r in wl.regions:
                     W.perturb_ulp_noise(c, r, seed=wl.seed * 10 + r.region_id)
-            elif name == "int_exact":
+            elif recipe == "int_exact":
                 for r in wl.regions:
                     W.flip_bit(c, r, rng)
-            elif name == "snapshot_4096":
+            elif recipe == "snapshot_4096":
                 for r in wl.regions:
                     W.perturb_sparse(c, r, rng, rate=1e-6)
                 for k in rng.choice(len(wl.regions), 3, replace=False):

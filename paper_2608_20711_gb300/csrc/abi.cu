@@ -195,7 +195,7 @@ struct DeviceScope {
 struct asmv_ctx {
   int device = 0;
   int sms = 0;
-  int fill_ctas = 1, cmp1_ctas = 1, cmpk_ctas = 1;
+  int fill_ctas = 1;
   void *dws = nullptr;
   size_t dws_cap = 0;
   unsigned char *hst = nullptr;
@@ -322,12 +322,15 @@ int readback(asmv_ctx *ctx, size_t stats_off, size_t img_bytes, size_t count, cu
              asmv_stats *out, size_t ref_n) {
   cudaError_t e;
   unsigned char *host = ctx->hst + ((img_bytes + 255) & ~(size_t)255);
-  if ((e = cudaMemcpyAsync(host, (unsigned char *)ctx->dws + stats_off, count * sizeof(StatsDev),
-                           cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+  if ((e = cudaMemcpyAsync(host, (unsigned char *)ctx->dws + stats_off,
+                           (count + 1) * sizeof(StatsDev), cudaMemcpyDeviceToHost, s)) != cudaSuccess)
     return fail_cuda(ctx, e);
   if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return fail_cuda(ctx, e);
   ctx->staged_pending = false;
   ctx->ws_pending = false;
+  uint32_t err;
+  std::memcpy(&err, host + count * sizeof(StatsDev), sizeof err);
+  if (err) return ASMV_ETIMEOUT;                     // a bounded device wait expired
   std::memcpy(out, host, count * sizeof(asmv_stats));
   if (ref_n) {
     // reference-guard damage was accumulated in the first candidate's entries
@@ -381,8 +384,6 @@ int asmv_ctx_create(asmv_ctx **out, int device) {
     return ASMV_ECUDA;
   }
   ctx->fill_ctas = fill_max_ctas_per_sm();
-  ctx->cmp1_ctas = compare_max_ctas_per_sm(1);
-  ctx->cmpk_ctas = compare_max_ctas_per_sm(kMaxCands);
   void *fn = nullptr;
   cudaDriverEntryPointQueryResult q;
   if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &fn, 12000, cudaEnableDefault, &q) ==
@@ -510,6 +511,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   std::vector<uint64_t> caddr(guard_only ? 0 : k * n);
   std::vector<GuardSeg> segs;
   uint64_t tile = 0;
+  const uint32_t tile_bytes = compare_tile_bytes((uint32_t)std::min<size_t>(std::max<size_t>(k, 1), kMaxCands));
   for (size_t i = 0; i < n; ++i) {
     const asmv_region &r = ref[i];
     uint64_t pb, tot;
@@ -527,7 +529,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
       vec = vec && (a % 16) == 0;
     }
     c.vec = vec;
-    tile += tiles_of(c.bytes);
+    tile += (c.bytes + tile_bytes - 1) / tile_bytes;
     if (guard_only) {
       add_region_guards(segs, r, kSegSelf, (uint32_t)i);
     } else {
@@ -539,7 +541,9 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   cr[n].tile0 = tile;
   const size_t nstats = guard_only ? n : k * n;
   if (nstats == 0) return ASMV_OK;
-  std::vector<StatsDev> st(nstats, empty_stats());
+  // statistics, then one error word, read back together
+  std::vector<StatsDev> st(nstats + 1, empty_stats());
+  std::memset(&st[nstats], 0, sizeof(StatsDev));
 
   Image img;
   const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CmpRegion));
@@ -547,15 +551,17 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
   const size_t o_stats = img.add(st.data(), st.size() * sizeof(StatsDev));
   unsigned char *dev = nullptr;
-  if ((rc = stage(ctx, img, nstats * sizeof(StatsDev), s, &dev)) != ASMV_OK) return rc;
+  if ((rc = stage(ctx, img, st.size() * sizeof(StatsDev), s, &dev)) != ASMV_OK) return rc;
 
   CmpParams p;
   std::memset(&p, 0, sizeof p);
   p.regions = (const CmpRegion *)(dev + o_regs);
   p.segs = (const GuardSeg *)(dev + o_segs);
   p.seg_stats = (StatsDev *)(dev + o_stats);
+  p.err = (uint32_t *)((StatsDev *)(dev + o_stats) + nstats);
   p.ntiles = tile;
   p.nregions = (uint32_t)n;
+  p.tile_bytes = tile_bytes;
   for (int d = 0; d < 7; ++d) {
     if (is_float((uint32_t)d) && tol) p.tol[d] = make_tolf(tol[d]);
   }
@@ -569,9 +575,11 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
     p.stats = (StatsDev *)(dev + o_stats) + g * kMaxCands * n;
     p.nsegs = (g == 0) ? (uint32_t)segs.size() : 0u;
     if (guard_only) p.ntiles = 0;
-    const int ctas = (kg > 1) ? ctx->cmpk_ctas : ctx->cmp1_ctas;
-    if ((e = (cudaError_t)launch_compare(p, grid_for(ctx, p.ntiles, p.nsegs, ctas), s)) != cudaSuccess)
-      return fail_cuda(ctx, e);
+    // one CTA per SM: the shared-memory pipeline sizes itself to the SM
+    const uint64_t segs_per_cta = kConsumerWarps + 1;
+    const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(
+        std::max<uint64_t>(p.ntiles, (p.nsegs + segs_per_cta - 1) / segs_per_cta), (uint64_t)ctx->sms));
+    if ((e = (cudaError_t)launch_compare(p, grid, s)) != cudaSuccess) return fail_cuda(ctx, e);
     ctx->launches += 1;
   }
   if (ctx->timing) {

@@ -23,12 +23,13 @@
 //      D >= as(1-2^-24) > b(1+2^-22) + 2^-101 > B, so d > B.
 //  Anything else (ambiguous band, NaN/Inf on either side, fp32 overflow of
 //  c - r) is evaluated exactly in fp64.
-//  (3) max_abs: RN is monotone, so for as_j < as_k the exact D_j < D_k.
-//      Per thread we keep m32 = max as and, over the elements tied at m32,
-//      the largest TwoSum residual me (D = m32 + me exactly); the exact
-//      maximum is RN64(m32 + me).  Only elements with as >= m32 are touched.
+//  (3) max_abs: when as < |r|/2 the pair is within a factor of two, so
+//      c - r is exact in fp32 (Sterbenz) and as equals D; such "plain"
+//      elements update an fp32 running maximum m32 with fmaxf, exactly.
+//      Every other element goes to the exact path, which keeps the fp64
+//      maximum of RN64(D).  max_abs = max(m32, that maximum).
 //  (4) max_rel: a thread keeps its exact maximum Rmax and T <= Rmax(1-2^-19)
-//      in fp32.  An element can exceed Rmax only if as >= T*|r| (the
+//      in fp32.  An element can exceed Rmax only if as > T*|r| (the
 //      relative error of as/|r| against d/|r| is below 2^-23), which
 //      one fma decides exactly in sign; those elements get the exact
 //      RN64(d/|r|).
@@ -56,10 +57,10 @@ namespace {
 struct Hot {
   uint32_t cnt;          // mismatches in the current region (per thread; < 2^32 for any HBM size)
   uint32_t nonfin;       // NaN/Inf-position mismatches
-  uint32_t found;        // first mismatch recorded
-  unsigned long long first;
-  float m32, me, T;
-  double dabs;           // exact max |c - r| over fp64-path elements
+  unsigned long long first;   // lowest mismatching element index seen (~0 if none)
+  float m32;             // exact max |c - r| over plain elements (see (3))
+  float T;               // relative-error screen threshold
+  double dabs;           // exact max |c - r| over exact-path elements
   double drel;           // exact max relative error
 };
 
@@ -97,23 +98,13 @@ __device__ __forceinline__ void exact_int(int64_t r, int64_t c, Hot &h) {
   rel_update(h, d, (double)r);
 }
 
-// A rare element that the screen decided (definite match or mismatch) but
-// that may raise max_abs or max_rel.
+// A rare element that the screen decided (definite match or mismatch):
+// exact maximum updates.
 __device__ __forceinline__ void decided_update(float r, float c, Hot &h) {
-  const float s = __fsub_rn(c, r);
-  const float as = fabsf(s), ar = fabsf(r);
-  if (as >= h.m32) {
-    // TwoSum of c and -r: s + e == c - r exactly
-    const float bb = __fsub_rn(s, c);
-    const float e = __fadd_rn(__fsub_rn(c, __fsub_rn(s, bb)), __fsub_rn(-r, bb));
-    const float ep = (s >= 0.0f) ? e : -e;                // |c - r| == as + ep
-    if (as > h.m32) { h.m32 = as; h.me = ep; }
-    else h.me = fmaxf(h.me, ep);
-  }
-  if (__fmaf_rn(-h.T, ar, as) >= 0.0f) {
-    const double d = fabs(__dsub_rn((double)c, (double)r));
-    rel_update(h, d, (double)r);
-  }
+  const double r64 = (double)r;
+  const double d = fabs(__dsub_rn((double)c, r64));
+  h.dabs = fmax(h.dabs, d);
+  rel_update(h, d, r64);
 }
 
 // Masks of one chunk: bit j for element j.
@@ -122,15 +113,16 @@ struct Masks {
   uint32_t rare;   // elements needing the exact path or a maxima update
 };
 
-__device__ __forceinline__ void screen(float r, float c, int j, const Hot &h, const TolF &t,
-                                       Masks &m) {
+__device__ __forceinline__ void screen(float r, float c, int j, Hot &h, const TolF &t, Masks &m) {
   const float s = __fsub_rn(c, r);
   const float as = fabsf(s), ar = fabsf(r);
   const float lo = __fmaf_rn(t.rlo, ar, t.alo);
   const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
   const bool ok = as < lo;
-  const bool bad = (as > hi) & (as <= FLT_MAX);
-  const bool rare = !(ok | bad) | (as >= h.m32) | (__fmaf_rn(-h.T, ar, as) >= 0.0f);
+  const bool bad = as > hi;                       // Inf/NaN cases are rare below
+  const bool plain = __fadd_rn(as, as) < ar;      // c - r exact (Sterbenz)
+  const bool rare = !(ok | bad) | !plain | (__fmaf_rn(-h.T, ar, as) > 0.0f);
+  if (plain) h.m32 = fmaxf(h.m32, as);
   m.bad |= (uint32_t)bad << j;
   m.rare |= (uint32_t)rare << j;
 }
@@ -168,7 +160,7 @@ __device__ __forceinline__ int64_t elem_int(const uint4 &v, int j) {
 
 // Screen one differing 32-bit word of a float chunk.
 template <uint32_t DT>
-__device__ __forceinline__ void screen_word(uint32_t rw, uint32_t cw, int w, const Hot &h,
+__device__ __forceinline__ void screen_word(uint32_t rw, uint32_t cw, int w, Hot &h,
                                             const TolF &t, Masks &m) {
   if (DT == kF32) {
     screen(__uint_as_float(rw), __uint_as_float(cw), w, h, t, m);
@@ -192,54 +184,107 @@ __device__ __forceinline__ void screen_word(uint32_t rw, uint32_t cw, int w, con
   }
 }
 
-struct RareOut {
-  Hot h;
-  uint32_t bad;    // mismatches found on the exact path
+// Rare elements are queued per warp in shared memory and evaluated exactly
+// once per tile, lane-parallel, instead of diverging inside the screen.
+constexpr uint32_t kQueue = 256;          // entries per warp
+
+struct QEntry {
+  uint32_t r, c;                          // fp32 bits (floats) or int32 values
+  unsigned long long idx;                 // element index in the region
 };
 
-// Every element of one chunk flagged by the screen (or, for integers,
-// every differing element).  Out of line: it is rare, and the fp64
-// arithmetic would otherwise inflate the hot loop's register budget.
+struct Queue {
+  QEntry e[kQueue];
+  uint32_t count;
+};
+
+// Exact evaluation of one queued element; returns the mismatch bit.
 template <uint32_t DT>
-__device__ __noinline__ RareOut rare_chunk(const uint4 R, const uint4 C, uint32_t rare, Hot h,
-                                           const TolF t) {
-  uint32_t bad = 0;
+__device__ __forceinline__ uint32_t exact_elem(uint32_t rb, uint32_t cb, Hot &h, const TolF &t) {
+  if (DT == kI32 || DT == kI8 || DT == kU8) {
+    exact_int((int64_t)(int32_t)rb, (int64_t)(int32_t)cb, h);
+    return 1u;
+  }
+  const float r = __uint_as_float(rb), c = __uint_as_float(cb);
+  const float as = fabsf(__fsub_rn(c, r)), ar = fabsf(r);
+  const bool ok = as < __fmaf_rn(t.rlo, ar, t.alo);
+  const bool definite_bad = (as > __fmaf_rn(t.rhi, ar, t.ahi)) & (as <= FLT_MAX);
+  if (ok | definite_bad) {
+    decided_update(r, c, h);
+    return definite_bad ? 1u : 0u;
+  }
+  return exact_float(r, c, h, t);
+}
+
+template <uint32_t DT>
+__device__ __forceinline__ void record(uint32_t bad, unsigned long long idx, Hot &h) {
+  if (bad) { h.cnt += 1; h.first = umin64(h.first, idx); }
+}
+
+// Drain the warp's queue: lanes take entries in turn; then every lane
+// adopts the warp's largest exact relative error (only the overall maximum
+// matters, so a shared threshold is as valid as a per-lane one).
+template <uint32_t DT>
+__device__ __noinline__ Hot drain(Queue *q, Hot h, const TolF t) {
+  __syncwarp();
+  const uint32_t n = min(q->count, kQueue);
+  for (uint32_t j = threadIdx.x & 31; j < n; j += 32) {
+    const QEntry e = q->e[j];
+    record<DT>(exact_elem<DT>(e.r, e.c, h, t), e.idx, h);
+  }
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) q->count = 0;
+  unsigned long long rb = (unsigned long long)__double_as_longlong(h.drel);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) rb = umax64(rb, __shfl_xor_sync(0xFFFFFFFFu, rb, o));
+  const double d = __longlong_as_double((long long)rb);
+  if (d > h.drel) { h.drel = d; h.T = tfloor(d); }
+  __syncwarp();
+  return h;
+}
+
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t elem_bits(const uint4 &v, int j) {
+  if (DT == kI32 || DT == kI8 || DT == kU8) return (uint32_t)(int32_t)elem_int<DT>(v, j);
+  return __float_as_uint(elem_f32<DT>(v, j));
+}
+
+// Queue the flagged elements of one chunk; a full queue falls back to
+// evaluating in this lane.
+template <uint32_t DT>
+__device__ __noinline__ Hot push_rare(const uint4 R, const uint4 C, uint32_t rare,
+                                      unsigned long long e0, Queue *q, Hot h, const TolF t) {
   while (rare) {
     const int j = __ffs(rare) - 1;
     rare &= rare - 1;
-    if (DT == kI32 || DT == kI8 || DT == kU8) {
-      exact_int(elem_int<DT>(R, j), elem_int<DT>(C, j), h);
-      bad |= 1u << j;
+    const uint32_t rb = elem_bits<DT>(R, j), cb = elem_bits<DT>(C, j);
+    const uint32_t slot = atomicAdd(&q->count, 1u);
+    if (slot < kQueue) {
+      QEntry e;
+      e.r = rb; e.c = cb; e.idx = e0 + (unsigned long long)j;
+      q->e[slot] = e;
     } else {
-      const float r = elem_f32<DT>(R, j), c = elem_f32<DT>(C, j);
-      const float as = fabsf(__fsub_rn(c, r)), ar = fabsf(r);
-      const bool ok = as < __fmaf_rn(t.rlo, ar, t.alo);
-      const bool definite_bad = (as > __fmaf_rn(t.rhi, ar, t.ahi)) & (as <= FLT_MAX);
-      if (ok | definite_bad) decided_update(r, c, h);
-      else bad |= exact_float(r, c, h, t) << j;
+      record<DT>(exact_elem<DT>(rb, cb, h, t), e0 + (unsigned long long)j, h);
     }
   }
-  RareOut o;
-  o.h = h;
-  o.bad = bad;
-  return o;
+  return h;
 }
 
 // One 16-byte chunk whose first element has index e0.
 template <uint32_t DT>
 __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e0, Hot &h,
-                                      const TolF &t) {
+                                      const TolF &t, Queue *q) {
   if (R.x == C.x && R.y == C.y && R.z == C.z && R.w == C.w) return;
-  uint32_t allbad = 0, rare = 0;
+  uint32_t rare = 0;
   if (DT == kI32 || DT == kI8 || DT == kU8) {
-    // integers: every differing element is a mismatch, handled exactly
+    // integers: every differing element is a mismatch, evaluated exactly
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const uint32_t d = word_of(R, w) ^ word_of(C, w);
       if (DT == kI32) rare |= (uint32_t)(d != 0) << w;
       else
 #pragma unroll
-        for (int q = 0; q < 4; ++q) rare |= (uint32_t)(((d >> (8 * q)) & 0xFFu) != 0) << (4 * w + q);
+        for (int qq = 0; qq < 4; ++qq) rare |= (uint32_t)(((d >> (8 * qq)) & 0xFFu) != 0) << (4 * w + qq);
     }
   } else {
     Masks m = {0u, 0u};
@@ -248,31 +293,27 @@ __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e
       const uint32_t rw = word_of(R, w), cw = word_of(C, w);
       if (rw != cw) screen_word<DT>(rw, cw, w, h, t, m);
     }
-    allbad = m.bad;
+    const uint32_t bad = m.bad & ~m.rare;     // decided here; rare ones are decided exactly
+    if (bad) {
+      h.cnt += __popc(bad);
+      h.first = umin64(h.first, e0 + (uint64_t)(__ffs(bad) - 1));
+    }
     rare = m.rare;
   }
-  if (rare) {
-    const RareOut o = rare_chunk<DT>(R, C, rare, h, t);
-    h = o.h;
-    allbad |= o.bad;
-  }
-  if (allbad) {
-    h.cnt += __popc(allbad);
-    if (!h.found) { h.found = 1; h.first = e0 + (uint64_t)(__ffs(allbad) - 1); }
-  }
+  if (rare) h = push_rare<DT>(R, C, rare, e0, q, h, t);
 }
 
 __device__ __forceinline__ void reset_hot(Hot &h) {
-  h.cnt = 0; h.nonfin = 0; h.found = 0; h.first = ~0ull;
-  h.m32 = 0.0f; h.me = 0.0f; h.T = 0.0f; h.dabs = 0.0; h.drel = 0.0;
+  h.cnt = 0; h.nonfin = 0; h.first = ~0ull;
+  h.m32 = 0.0f; h.T = 0.0f; h.dabs = 0.0; h.drel = 0.0;
 }
 
 // Merge a warp's statistics for region `ri`, candidate k into the global
 // entry with order-independent atomics; then reset.
 __device__ __forceinline__ void flush(Hot &h, const CmpParams &p, uint32_t k, uint32_t ri) {
   unsigned long long cnt = h.cnt, nonfin = h.nonfin;
-  unsigned long long first = h.found ? h.first : ~0ull;
-  const double a = fmax(h.dabs, __dadd_rn((double)h.m32, (double)h.me));
+  unsigned long long first = h.first;
+  const double a = fmax(h.dabs, (double)h.m32);
   unsigned long long ab = (unsigned long long)__double_as_longlong(a);
   unsigned long long rb = (unsigned long long)__double_as_longlong(h.drel);
 #pragma unroll
@@ -300,59 +341,111 @@ __device__ __forceinline__ uint4 load_chunk(uint64_t base, uint64_t c, uint64_t 
   return load_bytes(base + 16 * c, (uint32_t)umin64(16, bytes - 16 * c));
 }
 
+// ---------------------------------------------------------------- pipeline
+// mbarrier helpers (shared::cta addresses).  Waits are bounded: after
+// kWaitRounds tries of up to kWaitHintNs each, the wait reports failure.
+constexpr uint32_t kWaitRounds = 20000;
+constexpr uint32_t kWaitHintNs = 100000;
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("{ .reg .b64 st; mbarrier.arrive.shared::cta.b64 st, [%0]; }" :: "r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t tx) {
+  asm volatile("{ .reg .b64 st; mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1; }"
+               :: "r"(bar), "r"(tx) : "memory");
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kWaitRounds; ++i) {
+    uint32_t done;
+    asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;"
+                 " selp.u32 %0, 1, 0, p; }"
+                 : "=r"(done) : "r"(bar), "r"(parity), "r"(kWaitHintNs) : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+// 1-D bulk copy global -> shared, completing `bytes` on the mbarrier.
+__device__ __forceinline__ void bulk_load(uint32_t dst, uint64_t src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+// Tile geometry of tile t of region r (tile_bytes per tile).
+struct TileInfo {
+  uint64_t off;        // byte offset of the tile in the payload
+  uint32_t nloc;       // 16-byte chunks in the tile (last may be short)
+  uint32_t nsm;        // chunks staged in shared memory (whole 16-byte chunks of vec regions)
+};
+__device__ __forceinline__ TileInfo tile_info(const CmpRegion &r, uint64_t t, uint32_t tile_bytes) {
+  TileInfo ti;
+  ti.off = (t - r.tile0) * (uint64_t)tile_bytes;
+  const uint64_t nb = umin64(tile_bytes, r.bytes - ti.off);
+  ti.nloc = (uint32_t)((nb + 15) >> 4);
+  ti.nsm = r.vec ? (uint32_t)(nb >> 4) : 0u;
+  return ti;
+}
+
 // A warp's share of one tile for its candidate: chunks part*32 + lane +
-// j*32*G of the tile, U at a time.
-template <uint32_t DT, bool STAGE>
-__device__ __noinline__ Hot tile(const CmpRegion r, uint64_t cbase, uint64_t tile_in_region,
-                                 uint32_t part, uint32_t G, Hot h, const TolF t,
-                                 const uint4 *ref_tile) {
+// j*32*W; staged chunks come from shared memory, the rest from global.
+template <uint32_t DT>
+__device__ __noinline__ Hot tile(const CmpRegion r, uint64_t cbase, TileInfo ti, const uint4 *sref,
+                                 const uint4 *scand, uint32_t part, uint32_t W, Hot h, const TolF t,
+                                 Queue *q) {
   constexpr int E = Fmt<DT>::E;
-  constexpr int U = 4;
-  const uint64_t c0 = tile_in_region * kTileChunks;
-  const uint64_t nchunks = (r.bytes + 15) >> 4, full = r.bytes >> 4;
-  const uint32_t nloc = (uint32_t)umin64(kTileChunks, nchunks - c0);
-  const bool vec = r.vec != 0;
-  const uint32_t stride = 32 * G;
-  for (uint32_t i0 = part * 32 + (threadIdx.x & 31); i0 < nloc; i0 += U * stride) {
+  constexpr int U = 2;
+  const uint64_t c0 = ti.off >> 4;
+  const uint64_t full = r.bytes >> 4;
+  const uint32_t stride = 32 * W;
+  uint32_t i0 = part * 32 + (threadIdx.x & 31);
+  for (; i0 + (U - 1) * stride < ti.nsm; i0 += U * stride) {
     uint4 R[U], C[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const uint32_t i = i0 + u * stride;
-      if (i < nloc) {
-        C[u] = load_chunk(cbase, c0 + i, full, r.bytes, vec);
-        R[u] = STAGE ? ref_tile[i] : load_chunk(r.ref, c0 + i, full, r.bytes, vec);
-      }
-    }
+    for (int u = 0; u < U; ++u) { R[u] = sref[i0 + u * stride]; C[u] = scand[i0 + u * stride]; }
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const uint32_t i = i0 + u * stride;
-      if (i < nloc) chunk<DT>(R[u], C[u], (c0 + i) * E, h, t);
-    }
+    for (int u = 0; u < U; ++u) chunk<DT>(R[u], C[u], (c0 + i0 + u * stride) * E, h, t, q);
+    __syncwarp();
+    if (q->count >= kQueue / 2) h = drain<DT>(q, h, t);
   }
+  for (uint32_t i = i0; i < ti.nloc; i += stride) {
+    uint4 R, C;
+    if (i < ti.nsm) { R = sref[i]; C = scand[i]; }
+    else {
+      R = load_chunk(r.ref, c0 + i, full, r.bytes, false);
+      C = load_chunk(cbase, c0 + i, full, r.bytes, false);
+    }
+    chunk<DT>(R, C, (c0 + i) * E, h, t, q);
+  }
+  __syncwarp();
+  if (q->count) h = drain<DT>(q, h, t);
   return h;
 }
 
-template <bool STAGE>
-__device__ __forceinline__ void tile_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
-                                              uint64_t tr, uint32_t part, uint32_t G, Hot &h,
-                                              const uint4 *ref_tile) {
+__device__ __forceinline__ Hot tile_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
+                                             TileInfo ti, const uint4 *sref, const uint4 *scand,
+                                             uint32_t part, uint32_t W, Hot h, Queue *q) {
   switch (r.dtype) {
-    case kF32: h = tile<kF32, STAGE>(r, cbase, tr, part, G, h, p.tol[kF32], ref_tile); break;
-    case kBF16: h = tile<kBF16, STAGE>(r, cbase, tr, part, G, h, p.tol[kBF16], ref_tile); break;
-    case kF16: h = tile<kF16, STAGE>(r, cbase, tr, part, G, h, p.tol[kF16], ref_tile); break;
-    case kF8: h = tile<kF8, STAGE>(r, cbase, tr, part, G, h, p.tol[kF8], ref_tile); break;
-    case kI32: h = tile<kI32, STAGE>(r, cbase, tr, part, G, h, p.tol[0], ref_tile); break;
-    case kI8: h = tile<kI8, STAGE>(r, cbase, tr, part, G, h, p.tol[0], ref_tile); break;
-    default: h = tile<kU8, STAGE>(r, cbase, tr, part, G, h, p.tol[0], ref_tile); break;
+    case kF32: return tile<kF32>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF32], q);
+    case kBF16: return tile<kBF16>(r, cbase, ti, sref, scand, part, W, h, p.tol[kBF16], q);
+    case kF16: return tile<kF16>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF16], q);
+    case kF8: return tile<kF8>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF8], q);
+    case kI32: return tile<kI32>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
+    case kI8: return tile<kI8>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
+    default: return tile<kU8>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
   }
 }
 
 // Guard segments: one warp per segment; bad bytes and the first bad offset.
-__device__ void guard_phase(const CmpParams &p) {
+__device__ void guard_phase(const CmpParams &p, uint32_t warp, uint32_t nwarps) {
   const uint32_t lane = threadIdx.x & 31;
-  const uint64_t warp = (uint64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
-  const uint64_t nw = (uint64_t)gridDim.x * kWarps;
-  for (uint64_t s = warp; s < p.nsegs; s += nw) {
+  const uint64_t gw = (uint64_t)blockIdx.x * nwarps + warp;
+  const uint64_t nw = (uint64_t)gridDim.x * nwarps;
+  for (uint64_t s = gw; s < p.nsegs; s += nw) {
     const GuardSeg g = p.segs[s];
     const uint8_t *src = reinterpret_cast<const uint8_t *>(g.ptr);
     unsigned long long bad = 0, first = ~0ull;
@@ -376,58 +469,122 @@ __device__ void guard_phase(const CmpParams &p) {
   }
 }
 
-// STAGE (K > 1): the reference tile goes through shared memory once.
-template <bool STAGE>
-__global__ void __launch_bounds__(kThreads, 2) compare_kernel(const CmpParams p) {
-  __shared__ __align__(16) uint4 ref_tile[STAGE ? kTileChunks : 1];
+// Warps 0..kConsumerWarps-1 check; the last warp feeds the stages.  Stage s
+// holds the reference tile and the K candidate tiles (tile_bytes each);
+// full[s] completes when its bulk copies land, empty[s] when every
+// consumer warp has finished with it.
+__global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams p) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem);
+  uint64_t *empty = full + kStages;
+  Queue *queues = reinterpret_cast<Queue *>(smem + 128);
+  unsigned char *bufs = smem + 128 + kConsumerWarps * sizeof(Queue);
+  const uint32_t K = p.K, TB = p.tile_bytes;
+  const uint32_t stage_bytes = (1 + K) * TB;
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x < kConsumerWarps) queues[threadIdx.x].count = 0;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_addr(&full[s]), 1);
+      mbar_init(smem_addr(&empty[s]), kConsumerWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
   const uint64_t G = gridDim.x, b = blockIdx.x;
   const uint64_t t0 = p.ntiles * b / G, t1 = p.ntiles * (b + 1) / G;
-  const uint32_t warp = threadIdx.x >> 5;
-  const uint32_t K = p.K, W = kWarps / K;              // warps per candidate
-  const bool active = warp < W * K;
-  const uint32_t k = warp % K, part = warp / K;
-  if (t0 < t1) {
+  bool ok = true;
+  if (warp == kConsumerWarps) {
+    // producer
+    if (lane == 0 && t0 < t1) {
+      uint32_t ri = find_region(p.regions, p.nregions, t0);
+      uint32_t u = 0;
+      for (uint64_t t = t0; t < t1 && ok; ++t, ++u) {
+        while (p.regions[ri + 1].tile0 <= t) ++ri;
+        const uint32_t s = u % kStages;
+        if (u >= (uint32_t)kStages && !mbar_wait(smem_addr(&empty[s]), ((u / kStages) & 1u) ^ 1u)) {
+          ok = false;
+          break;
+        }
+        const CmpRegion r = p.regions[ri];
+        const TileInfo ti = tile_info(r, t, TB);
+        const uint32_t nb = ti.nsm * 16u;
+        const uint32_t fb = smem_addr(&full[s]);
+        mbar_arrive_tx(fb, nb * (1 + K));
+        if (nb) {
+          const uint32_t dst = smem_addr(bufs + (size_t)s * stage_bytes);
+          bulk_load(dst, r.ref + ti.off, nb, fb);
+          for (uint32_t k = 0; k < K; ++k)
+            bulk_load(dst + (1 + k) * TB, p.cands[(size_t)k * p.nregions + ri] + ti.off, nb, fb);
+        }
+      }
+      if (!ok) {
+        atomicOr(p.err, 1u);
+        // let copies already issued land before the CTA exits
+        for (uint32_t v = (u >= (uint32_t)kStages ? u - kStages : 0); v < u; ++v)
+          mbar_wait(smem_addr(&full[v % kStages]), (v / kStages) & 1u);
+      }
+    }
+  } else if (t0 < t1) {
+    // consumers
+    const uint32_t W = kConsumerWarps / K;                  // warps per candidate
+    const bool active = warp < W * K;
+    const uint32_t k = warp % K, part = warp / K;
     Hot h;
     reset_hot(h);
     uint32_t ri = find_region(p.regions, p.nregions, t0);
-    for (uint64_t t = t0; t < t1; ++t) {
+    uint32_t u = 0;
+    for (uint64_t t = t0; t < t1; ++t, ++u) {
       if (p.regions[ri + 1].tile0 <= t) {
         if (active) flush(h, p, k, ri);
         while (p.regions[ri + 1].tile0 <= t) ++ri;
       }
-      const CmpRegion r = p.regions[ri];
-      if (STAGE) {
-        const uint64_t c0 = (t - r.tile0) * kTileChunks;
-        const uint64_t nchunks = (r.bytes + 15) >> 4, full = r.bytes >> 4;
-        const uint32_t nloc = (uint32_t)umin64(kTileChunks, nchunks - c0);
-        for (uint32_t i = threadIdx.x; i < nloc; i += kThreads)
-          ref_tile[i] = load_chunk(r.ref, c0 + i, full, r.bytes, r.vec != 0);
-        __syncthreads();
+      const uint32_t s = u % kStages;
+      if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u)) {
+        ok = false;
+        break;
       }
-      if (active)
-        tile_dispatch<STAGE>(p, r, p.cands[(size_t)k * p.nregions + ri], t - r.tile0, part, W, h,
-                             ref_tile);
-      if (STAGE) __syncthreads();
+      if (active) {
+        const CmpRegion r = p.regions[ri];
+        const TileInfo ti = tile_info(r, t, TB);
+        const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
+        const uint4 *scand = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes +
+                                                              (size_t)(1 + k) * TB);
+        h = tile_dispatch(p, r, p.cands[(size_t)k * p.nregions + ri], ti, sref, scand, part, W, h,
+                          &queues[warp]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
     }
-    if (active) flush(h, p, k, ri);
+    if (!ok) {
+      if (lane == 0) atomicOr(p.err, 1u);
+    } else if (active) {
+      flush(h, p, k, ri);
+    }
   }
-  guard_phase(p);
+  guard_phase(p, warp, kConsumerWarps + 1);
 }
 
 }  // namespace
 
-int compare_max_ctas_per_sm(int K) {
-  int n = 0;
-  const cudaError_t e = (K > 1)
-      ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compare_kernel<true>, kThreads, 0)
-      : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compare_kernel<false>, kThreads, 0);
-  if (e != cudaSuccess || n < 1) return 1;
-  return n;
+size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes) {
+  return 128 + kConsumerWarps * sizeof(Queue) + (size_t)kStages * (1 + K) * tile_bytes;
+}
+
+uint32_t compare_tile_bytes(uint32_t K) {
+  // stage = (1 + K) tiles; keep a stage near 32-36 KiB
+  if (K <= 1) return 16384;
+  if (K == 2) return 12288;
+  if (K == 3) return 8192;
+  return 4096;
 }
 
 int launch_compare(const CmpParams &p, int grid, void *stream) {
-  if (p.K > 1) compare_kernel<true><<<grid, kThreads, 0, (cudaStream_t)stream>>>(p);
-  else compare_kernel<false><<<grid, kThreads, 0, (cudaStream_t)stream>>>(p);
+  const size_t smem = compare_smem_bytes(p.K, p.tile_bytes);
+  cudaError_t e = cudaFuncSetAttribute(compare_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return (int)e;
+  compare_kernel<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }
 

@@ -2,7 +2,8 @@
 // the kernels (fill.cu, compare.cu).  Internal to the library.
 //
 // Work decomposition.  Every region's payload is cut into tiles of
-// kTileBytes (the last tile of a region may be short).  Tiles of all
+// kTileBytes for the fill, and of a per-launch tile size for the compare
+// (the last tile of a region may be short).  Tiles of all
 // regions form one index space; region i owns tiles [tile0[i], tile0[i+1]).
 // A launch runs a persistent grid; CTA b takes the contiguous tile range
 // [T*b/G, T*(b+1)/G), so a CTA crosses few region boundaries and flushes its
@@ -23,6 +24,9 @@ constexpr int kTileChunks = 1024;
 constexpr uint64_t kTileBytes = (uint64_t)kChunkBytes * kTileChunks;  // 16 KiB
 constexpr uint32_t kGuardSegBytes = 4096;
 constexpr int kMaxCands = 8;            // candidates per batched launch
+constexpr int kConsumerWarps = 16;      // compare: checking warps per CTA
+constexpr int kStages = 4;              // compare: shared-memory pipeline depth
+constexpr int kCmpThreads = (kConsumerWarps + 1) * 32;   // + one producer warp
 
 enum : uint32_t { kF32 = 0, kBF16 = 1, kF16 = 2, kF8 = 3, kI32 = 4, kI8 = 5, kU8 = 6 };
 enum : uint32_t { kRaw = 0, kUniform = 1, kNormal = 2, kIntRange = 3, kNone = 4 };
@@ -94,11 +98,12 @@ struct CmpParams {
   const GuardSeg *segs;
   StatsDev *stats;             // [K][nregions] (this launch's candidates)
   StatsDev *seg_stats;         // guard segments index from here
+  uint32_t *err;               // set non-zero when a bounded wait expires
   uint64_t ntiles;
   uint32_t nregions;
   uint32_t nsegs;
   uint32_t K;
-  uint32_t pad_;
+  uint32_t tile_bytes;         // payload bytes per tile (multiple of 16)
   TolF tol[7];
 };
 
@@ -106,6 +111,7 @@ struct CmpParams {
 int launch_fill(const FillParams &p, int grid, void *stream);
 int launch_compare(const CmpParams &p, int grid, void *stream);
 int fill_max_ctas_per_sm();
-int compare_max_ctas_per_sm(int K);
+uint32_t compare_tile_bytes(uint32_t K);
+size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes);
 
 }  // namespace asmv

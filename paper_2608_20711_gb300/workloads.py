@@ -213,9 +213,11 @@ WORKLOADS = {
     "int_exact": int_exact,
     "snapshot_4096": snapshot,
     "batched_gemm_fp16": batched_gemm,
-    # a smaller case of the same kernels (above L2, a few GB on the device)
+    # smaller cases of the same kernels (above L2, a few GB on the device)
     "batched_gemm_fp16_8kx16k": lambda: batched_gemm(rows=8192, cols=16384,
                                                      input_bytes=1 << 30, input_regions=8),
+    "batched_gemm_fp16_4kx16k": lambda: batched_gemm(rows=4096, cols=16384,
+                                                     input_bytes=512 << 20, input_regions=4),
 }
 
 
