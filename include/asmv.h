@@ -213,6 +213,37 @@ const char *asmv_strerror(int status);
 /* ASMV_ABI_VERSION of the loaded library. */
 int asmv_abi_version(void);
 
+/* Size of the fixed device scratch behind asmv_compare_noalloc. */
+#define ASMV_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/* asmv_compare for callers that must not allocate memory (the paper has no
+ * counterpart; this is a convenience of this library).  A harness that
+ * replays captured dispatches at their original virtual addresses needs
+ * its reserved address space left untouched, and one that times candidate
+ * kernels cannot take the device-wide synchronisation an allocation may
+ * bring; neither can create a context, whose workspace and staging are
+ * allocated.  This call needs no context and allocates nothing: the launch
+ * plan and the statistics live in a file-scope device array of
+ * ASMV_NOALLOC_SCRATCH_BYTES that every GPU loading this library holds
+ * until the process exits, staged through a static host buffer.
+ *   - Runs on the calling thread's current CUDA device.  The first call on
+ *     a device looks up that device's address of the array (and the SM
+ *     count); make that first call before any stream capture.
+ *   - ref/cand/n/tol/out_host/stream as asmv_compare (one candidate).
+ *   - The plan must fit the scratch: regions (32 B each, plus one), one
+ *     candidate address (8 B) and one statistics entry (64 B) per region,
+ *     32 B per 4 KiB of guard band on either side, each part rounded to
+ *     256 B, plus one 64-byte error entry.  Larger tables, and every table
+ *     asmv_compare would reject, return ASMV_EINVAL.
+ *   - Every call reuses the same scratch and overwrites the previous
+ *     call's contents (the statistics are reset by each call).  Calls that
+ *     overlap on the GPU, on any streams or host threads, race; host
+ *     threads are serialised by a lock, but the caller must order the GPU
+ *     work of successive calls (the call synchronises its own stream).
+ * Returns ASMV_OK, ASMV_EINVAL, ASMV_ECUDA or ASMV_ETIMEOUT. */
+int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *cand, size_t n,
+                         const asmv_tol *tol, asmv_stats *out_host, asmv_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

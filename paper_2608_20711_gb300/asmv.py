@@ -56,7 +56,9 @@ assert ctypes.sizeof(Region) == 56 and ctypes.sizeof(Stats) == 64
 ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard_check",
                  "asmv_compare", "asmv_compare_batched", "asmv_check_regions",
                  "asmv_ctx_set_timing", "asmv_ctx_kernel_ms", "asmv_ctx_cuda_error",
-                 "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version")
+                 "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version",
+                 "asmv_compare_noalloc")
+NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
 class AsmvError(RuntimeError):
@@ -95,6 +97,7 @@ def lib():
         L.asmv_strerror.argtypes = [ctypes.c_int]
         L.asmv_strerror.restype = ctypes.c_char_p
         L.asmv_abi_version.argtypes = []
+        L.asmv_compare_noalloc.argtypes = [RP, RP, sz, TP, SP, vp]
         _lib = L
     return _lib
 
@@ -251,3 +254,19 @@ class Context:
             _stream_handle(stream)))
         flat = stats_dicts(out, k * n)
         return [flat[j * n:(j + 1) * n] for j in range(k)]
+
+
+def compare_noalloc(ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:
+    """asmv_compare_noalloc: the check of one candidate on the current CUDA
+    device, for callers that must not allocate device memory (no context;
+    the plan and statistics live in the library's fixed device scratch).
+    Raises AsmvError on a non-OK status."""
+    L = lib()
+    ra, ca = region_array(ref), region_array(cand)
+    out = (Stats * max(1, len(ref)))()
+    rc = L.asmv_compare_noalloc(ra, ca, len(ref),
+                                tol_array(tol) if not isinstance(tol, ctypes.Array) else tol,
+                                out, _stream_handle(stream))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return stats_dicts(out, len(ref))

@@ -10,6 +10,7 @@
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <utility>
 #include <vector>
@@ -642,3 +643,208 @@ int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref, const asmv_regio
 }
 
 }  // extern "C"
+
+// ==================================================== compare without allocation
+// Some callers must not allocate device memory while they check a
+// candidate: a differential-testing harness that replays captured
+// dispatches restores regions at their original virtual addresses and
+// needs the address space it reserved to stay exactly as it was, and a
+// harness that times candidate kernels cannot afford the device-wide
+// synchronisation an allocation may cause.  asmv_compare_noalloc serves
+// them: its scratch (the launch plan and the statistics) lives in the
+// file-scope device array below, which every GPU that loads this library
+// holds until the process exits, and host-side staging is a static
+// buffer.  It calls no allocating routine.
+namespace {
+
+constexpr size_t kNoAllocBytes = ASMV_NOALLOC_SCRATCH_BYTES;
+constexpr int kNoAllocMaxDevices = 64;
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+
+alignas(256) unsigned char g_noalloc_host[kNoAllocBytes];   // host image of the same layout
+unsigned char *g_noalloc_dev[kNoAllocMaxDevices];            // scratch address per device
+int g_noalloc_sms[kNoAllocMaxDevices];
+AddrRangeFn g_noalloc_range = nullptr;
+bool g_noalloc_range_looked_up = false;
+std::mutex g_noalloc_mutex;
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Set-up for the current device (under the mutex): the device address of
+// the scratch array, the SM count and the address-range lookup.
+int noalloc_setup(int dev) {
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return ASMV_EINVAL;
+  if (g_noalloc_dev[dev]) return ASMV_OK;
+  void *p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess || p == nullptr) { cudaGetLastError(); return ASMV_ECUDA; }
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return ASMV_ECUDA;
+  }
+  if (!g_noalloc_range_looked_up) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_noalloc_range = (AddrRangeFn)fn;
+    else
+      cudaGetLastError();
+    g_noalloc_range_looked_up = true;
+  }
+  g_noalloc_sms[dev] = sms;
+  g_noalloc_dev[dev] = (unsigned char *)p;
+  return ASMV_OK;
+}
+
+// Device-memory check of one allocation on the current device (no context).
+int noalloc_check_span(int dev, uint64_t alloc, uint64_t total) {
+  if (total == 0) return ASMV_OK;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, (const void *)alloc) != cudaSuccess) {
+    cudaGetLastError();
+    return ASMV_EINVAL;
+  }
+  if (a.type == cudaMemoryTypeDevice) {
+    if (a.device != dev) return ASMV_EINVAL;
+  } else if (a.type != cudaMemoryTypeManaged) {
+    return ASMV_EINVAL;
+  }
+  if (g_noalloc_range) {
+    unsigned long long base = 0;
+    size_t size = 0;
+    if (g_noalloc_range(&base, &size, alloc) != 0) return ASMV_EINVAL;
+    if (alloc + total > base + size) return ASMV_EINVAL;
+  }
+  return ASMV_OK;
+}
+
+size_t noalloc_segments(const asmv_region &r) {
+  return ((size_t)r.guard_lo + kGuardSegBytes - 1) / kGuardSegBytes +
+         ((size_t)r.guard_hi + kGuardSegBytes - 1) / kGuardSegBytes;
+}
+
+// Guard segments of one region written straight into the image.
+size_t noalloc_put_guards(GuardSeg *out, const asmv_region &r, uint8_t kind, uint32_t stats) {
+  uint64_t pb, tot;
+  region_extent(r, &pb, &tot);
+  size_t k = 0;
+  const uint64_t starts[2] = {r.alloc, r.alloc + r.guard_lo + pb};
+  const uint64_t offs[2] = {0, (uint64_t)r.guard_lo + pb};
+  const uint64_t lens[2] = {r.guard_lo, r.guard_hi};
+  for (int side = 0; side < 2; ++side) {
+    for (uint64_t o = 0; o < lens[side]; o += kGuardSegBytes) {
+      GuardSeg &g = out[k++];
+      std::memset(&g, 0, sizeof g);
+      g.ptr = starts[side] + o;
+      g.offset = offs[side] + o;
+      g.len = (uint32_t)std::min<uint64_t>(kGuardSegBytes, lens[side] - o);
+      g.stats = stats;
+      g.canary = r.canary;
+      g.kind = kind;
+    }
+  }
+  return k;
+}
+
+}  // namespace
+
+extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *cand, size_t n,
+                                    const asmv_tol *tol, asmv_stats *out_host,
+                                    asmv_stream_t stream) {
+  if ((n > 0 && (out_host == nullptr || cand == nullptr)) || !tol_ok(tol)) return ASMV_EINVAL;
+  int rc = check_table(ref, n, false);
+  if (rc != ASMV_OK) return rc;
+  if ((rc = check_table(cand, n, false)) != ASMV_OK) return rc;
+  for (size_t i = 0; i < n; ++i)
+    if (cand[i].dtype != ref[i].dtype || cand[i].n_elems != ref[i].n_elems) return ASMV_EINVAL;
+  if (n == 0) return ASMV_OK;
+
+  // sizes of the image: regions (+ sentinel), candidate addresses, guard
+  // segments, statistics (+ the error word)
+  size_t nsegs = 0;
+  for (size_t i = 0; i < n; ++i) nsegs += noalloc_segments(ref[i]) + noalloc_segments(cand[i]);
+  const size_t o_regs = 0;
+  const size_t o_cand = align256(o_regs + (n + 1) * sizeof(CmpRegion));
+  const size_t o_segs = align256(o_cand + n * sizeof(uint64_t));
+  const size_t o_stats = align256(o_segs + nsegs * sizeof(GuardSeg));
+  const size_t total = o_stats + (n + 1) * sizeof(StatsDev);
+  if (total > kNoAllocBytes) return ASMV_EINVAL;      // beyond the fixed scratch
+
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return ASMV_ECUDA; }
+  if ((rc = noalloc_setup(dev)) != ASMV_OK) return rc;
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    region_extent(ref[i], &pb, &tot);
+    if ((rc = noalloc_check_span(dev, ref[i].alloc, tot)) != ASMV_OK) return rc;
+    region_extent(cand[i], &pb, &tot);
+    if ((rc = noalloc_check_span(dev, cand[i].alloc, tot)) != ASMV_OK) return rc;
+  }
+
+  const uint32_t tile_bytes = compare_tile_bytes(1);
+  CmpRegion *cr = (CmpRegion *)(g_noalloc_host + o_regs);
+  uint64_t *caddr = (uint64_t *)(g_noalloc_host + o_cand);
+  GuardSeg *segs = (GuardSeg *)(g_noalloc_host + o_segs);
+  StatsDev *st = (StatsDev *)(g_noalloc_host + o_stats);
+  uint64_t tile = 0;
+  size_t ks = 0;
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    region_extent(ref[i], &pb, &tot);
+    CmpRegion &c = cr[i];
+    std::memset(&c, 0, sizeof c);
+    c.ref = ref[i].alloc + ref[i].guard_lo;
+    c.bytes = pb;
+    c.tile0 = tile;
+    c.dtype = ref[i].dtype;
+    caddr[i] = cand[i].alloc + cand[i].guard_lo;
+    c.vec = (c.ref % 16) == 0 && (caddr[i] % 16) == 0;
+    tile += (pb + tile_bytes - 1) / tile_bytes;
+    ks += noalloc_put_guards(segs + ks, ref[i], kSegRef, (uint32_t)i);
+    ks += noalloc_put_guards(segs + ks, cand[i], kSegCand, (uint32_t)i);
+    st[i] = empty_stats();
+  }
+  std::memset(&cr[n], 0, sizeof(CmpRegion));
+  cr[n].tile0 = tile;
+  std::memset(&st[n], 0, sizeof(StatsDev));          // the error word starts at zero
+
+  unsigned char *dscr = g_noalloc_dev[dev];
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(dscr, g_noalloc_host, total, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return ASMV_ECUDA;
+  CmpParams p;
+  std::memset(&p, 0, sizeof p);
+  p.regions = (const CmpRegion *)(dscr + o_regs);
+  p.cands = (const uint64_t *)(dscr + o_cand);
+  p.segs = (const GuardSeg *)(dscr + o_segs);
+  p.stats = (StatsDev *)(dscr + o_stats);
+  p.seg_stats = p.stats;
+  p.err = (uint32_t *)(p.stats + n);
+  p.ntiles = tile;
+  p.nregions = (uint32_t)n;
+  p.nsegs = (uint32_t)ks;
+  p.K = 1;
+  p.tile_bytes = tile_bytes;
+  for (int d = 0; d <= ASMV_F8E4M3; ++d) p.tol[d] = make_tolf(tol[d]);
+  const uint64_t per_cta = kConsumerWarps + 1;
+  const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(
+      std::max<uint64_t>(tile, (ks + per_cta - 1) / per_cta), (uint64_t)g_noalloc_sms[dev]));
+  if ((e = (cudaError_t)launch_compare(p, grid, s)) != cudaSuccess) return ASMV_ECUDA;
+  if ((e = cudaMemcpyAsync(st, dscr + o_stats, (n + 1) * sizeof(StatsDev), cudaMemcpyDeviceToHost,
+                           s)) != cudaSuccess)
+    return ASMV_ECUDA;
+  if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return ASMV_ECUDA;
+  uint32_t err;
+  std::memcpy(&err, &st[n], sizeof err);
+  if (err) return ASMV_ETIMEOUT;
+  std::memcpy(out_host, st, n * sizeof(asmv_stats));
+  return ASMV_OK;
+}
