@@ -192,16 +192,25 @@ class Setup:
 
 # ------------------------------------------------------------------ CPU oracle
 def _timed_until(budget_s, fn, n0, nmax):
-    """Run fn(n) with n doubling until one run takes >= budget_s (or n hits
-    nmax); return (n, seconds, result) of the last run."""
+    """Run fn(n) (which returns the work it did) with n growing until one
+    run takes >= budget_s; at n == nmax, repeat until the budget is spent.
+    Returns (n, seconds, work) summed over the measured runs."""
     n = n0
     while True:
         t0 = time.perf_counter()
-        res = fn(n)
+        work = fn(n)
         dt = time.perf_counter() - t0
-        if dt >= budget_s or n >= nmax:
-            return n, dt, res
+        if dt >= budget_s:
+            return n, dt, work
+        if n >= nmax:
+            break
         n = min(nmax, n * max(2, int(budget_s / max(dt, 1e-3) * 0.7)))
+    total_t, total_w = dt, work
+    while total_t < budget_s:
+        t0 = time.perf_counter()
+        total_w += fn(n)
+        total_t += time.perf_counter() - t0
+    return n, total_t, total_w
 
 
 def cpu_oracle_sample(setup, budget_s=12.0):

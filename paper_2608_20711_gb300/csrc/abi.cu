@@ -485,6 +485,10 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   p.seed = seed;
   p.nregions = (uint32_t)n;
   p.nsegs = (uint32_t)segs.size();
+  for (uint32_t r = 0; r < 10; ++r) {      // Philox round keys (Weyl sequence from the seed)
+    p.key0[r] = (uint32_t)seed + r * 0x9E3779B9u;
+    p.key1[r] = (uint32_t)(seed >> 32) + r * 0xBB67AE85u;
+  }
   cudaError_t e;
   if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
   if ((e = (cudaError_t)launch_fill(p, grid_for(ctx, tile, segs.size(), ctx->fill_ctas), s)) !=

@@ -60,9 +60,15 @@ struct Hot {
   unsigned long long first;   // lowest mismatching element index seen (~0 if none)
   float m32;             // exact max |c - r| over plain elements (see (3))
   float T;               // relative-error screen threshold
-  double dabs;           // exact max |c - r| over exact-path elements
-  double drel;           // exact max relative error
+  // exact maxima as bit patterns of non-negative doubles (integer order =
+  // numeric order), so that comparing them stays off the fp64 pipe
+  unsigned long long dabs;   // max |c - r| over exact-path elements
+  unsigned long long drel;   // max relative error
 };
+
+__device__ __forceinline__ unsigned long long dbits(double x) {
+  return (unsigned long long)__double_as_longlong(x);
+}
 
 __device__ __forceinline__ float tfloor(double d) {
   return __fmul_rd(__double2float_rd(d), 0x1.ffffcp-1f);    // <= d (1 - 2^-19)
@@ -71,7 +77,8 @@ __device__ __forceinline__ float tfloor(double d) {
 __device__ __forceinline__ void rel_update(Hot &h, double d, double r64) {
   const double ar = fabs(r64);
   const double rel = (ar != 0.0) ? __ddiv_rn(d, ar) : (d == 0.0 ? 0.0 : CUDART_INF);
-  if (rel > h.drel) { h.drel = rel; h.T = tfloor(rel); }
+  const unsigned long long b = dbits(rel);
+  if (b > h.drel) { h.drel = b; h.T = tfloor(rel); }
 }
 
 // Exact fp64 evaluation of one float pair; returns the mismatch bit.
@@ -85,7 +92,7 @@ __device__ __forceinline__ uint32_t exact_float(float r, float c, Hot &h, const 
   const double r64 = (double)r, c64 = (double)c;
   const double d = fabs(__dsub_rn(c64, r64));
   const double bound = __dadd_rn(t.atol, __dmul_rn(t.rtol, fabs(r64)));
-  h.dabs = fmax(h.dabs, d);
+  h.dabs = umax64(h.dabs, dbits(d));
   rel_update(h, d, r64);
   return d > bound ? 1u : 0u;
 }
@@ -94,37 +101,8 @@ __device__ __forceinline__ uint32_t exact_float(float r, float c, Hot &h, const 
 __device__ __forceinline__ void exact_int(int64_t r, int64_t c, Hot &h) {
   const int64_t dd = c - r;
   const double d = (double)(dd < 0 ? -dd : dd);     // exact: |d| < 2^33
-  h.dabs = fmax(h.dabs, d);
+  h.dabs = umax64(h.dabs, dbits(d));
   rel_update(h, d, (double)r);
-}
-
-// A rare element that the screen decided (definite match or mismatch):
-// exact maximum updates.
-__device__ __forceinline__ void decided_update(float r, float c, Hot &h) {
-  const double r64 = (double)r;
-  const double d = fabs(__dsub_rn((double)c, r64));
-  h.dabs = fmax(h.dabs, d);
-  rel_update(h, d, r64);
-}
-
-// Masks of one chunk: bit j for element j.
-struct Masks {
-  uint32_t bad;    // definite mismatches from the screen
-  uint32_t rare;   // elements needing the exact path or a maxima update
-};
-
-__device__ __forceinline__ void screen(float r, float c, int j, Hot &h, const TolF &t, Masks &m) {
-  const float s = __fsub_rn(c, r);
-  const float as = fabsf(s), ar = fabsf(r);
-  const float lo = __fmaf_rn(t.rlo, ar, t.alo);
-  const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
-  const bool ok = as < lo;
-  const bool bad = as > hi;                       // Inf/NaN cases are rare below
-  const bool plain = __fadd_rn(as, as) < ar;      // c - r exact (Sterbenz)
-  const bool rare = !(ok | bad) | !plain | (__fmaf_rn(-h.T, ar, as) > 0.0f);
-  if (plain) h.m32 = fmaxf(h.m32, as);
-  m.bad |= (uint32_t)bad << j;
-  m.rare |= (uint32_t)rare << j;
 }
 
 __device__ __forceinline__ uint32_t word_of(const uint4 &v, int w) {
@@ -158,39 +136,20 @@ __device__ __forceinline__ int64_t elem_int(const uint4 &v, int j) {
   return (int64_t)b;
 }
 
-// Screen one differing 32-bit word of a float chunk.
 template <uint32_t DT>
-__device__ __forceinline__ void screen_word(uint32_t rw, uint32_t cw, int w, Hot &h,
-                                            const TolF &t, Masks &m) {
-  if (DT == kF32) {
-    screen(__uint_as_float(rw), __uint_as_float(cw), w, h, t, m);
-  } else if (DT == kBF16) {
-    const uint32_t d = rw ^ cw;
-    if (d & 0xFFFFu) screen(__uint_as_float(rw << 16), __uint_as_float(cw << 16), 2 * w, h, t, m);
-    if (d >> 16) screen(__uint_as_float(rw & 0xFFFF0000u), __uint_as_float(cw & 0xFFFF0000u), 2 * w + 1, h, t, m);
-  } else if (DT == kF16) {
-    const uint32_t d = rw ^ cw;
-    const float2 rf = f16x2_to_f32(rw), cf = f16x2_to_f32(cw);
-    if (d & 0xFFFFu) screen(rf.x, cf.x, 2 * w, h, t, m);
-    if (d >> 16) screen(rf.y, cf.y, 2 * w + 1, h, t, m);
-  } else {                                      // fp8: four elements
-    const uint32_t d = rw ^ cw;
-    const float2 r0 = f8x2_to_f32(rw), c0 = f8x2_to_f32(cw);
-    const float2 r1 = f8x2_to_f32(rw >> 16), c1 = f8x2_to_f32(cw >> 16);
-    if (d & 0xFFu) screen(r0.x, c0.x, 4 * w, h, t, m);
-    if (d & 0xFF00u) screen(r0.y, c0.y, 4 * w + 1, h, t, m);
-    if (d & 0xFF0000u) screen(r1.x, c1.x, 4 * w + 2, h, t, m);
-    if (d >> 24) screen(r1.y, c1.y, 4 * w + 3, h, t, m);
-  }
+__device__ __forceinline__ uint32_t elem_bits(const uint4 &v, int j) {
+  if (DT == kI32 || DT == kI8 || DT == kU8) return (uint32_t)(int32_t)elem_int<DT>(v, j);
+  return __float_as_uint(elem_f32<DT>(v, j));
 }
 
-// Rare elements are queued per warp in shared memory and evaluated exactly
-// once per tile, lane-parallel, instead of diverging inside the screen.
-constexpr uint32_t kQueue = 256;          // entries per warp
+// Chunks the screen cannot settle are queued per warp in shared memory and
+// re-examined element by element once per tile, lane-parallel, instead of
+// diverging inside the screen.
+constexpr uint32_t kQueue = 64;           // chunk entries per warp
 
 struct QEntry {
-  uint32_t r, c;                          // fp32 bits (floats) or int32 values
-  unsigned long long idx;                 // element index in the region
+  uint4 R, C;                             // the raw 16-byte chunks
+  unsigned long long e0;                  // element index of the chunk's first element
 };
 
 struct Queue {
@@ -198,114 +157,185 @@ struct Queue {
   uint32_t count;
 };
 
-// Exact evaluation of one queued element; returns the mismatch bit.
-template <uint32_t DT>
-__device__ __forceinline__ uint32_t exact_elem(uint32_t rb, uint32_t cb, Hot &h, const TolF &t) {
-  if (DT == kI32 || DT == kI8 || DT == kU8) {
-    exact_int((int64_t)(int32_t)rb, (int64_t)(int32_t)cb, h);
-    return 1u;
-  }
-  const float r = __uint_as_float(rb), c = __uint_as_float(cb);
-  const float as = fabsf(__fsub_rn(c, r)), ar = fabsf(r);
+// 0.5 (1 - 2^-20): below this fraction of |r|, c - r is exact in fp32.
+#define ASMV_HALF_LESS 0x1.fffff8p-2f
+
+// Exact bookkeeping of one differing float element of a queued chunk: the
+// fp32 screen again, with fp64 only for what it cannot settle (ambiguous
+// band, non-finite values, |c-r| >= |r|/2, or a possible new max_rel).
+__device__ __forceinline__ uint32_t settle_float(float r, float c, Hot &h, const TolF &t) {
+  const float s = __fsub_rn(c, r);
+  const float as = fabsf(s), ar = fabsf(r);
   const bool ok = as < __fmaf_rn(t.rlo, ar, t.alo);
-  const bool definite_bad = (as > __fmaf_rn(t.rhi, ar, t.ahi)) & (as <= FLT_MAX);
-  if (ok | definite_bad) {
-    decided_update(r, c, h);
-    return definite_bad ? 1u : 0u;
+  const bool bad = (as > __fmaf_rn(t.rhi, ar, t.ahi)) & (as <= FLT_MAX);
+  const bool plain = as < __fmul_rn(0.5f, ar);          // c - r exact (Sterbenz)
+  if ((ok | bad) && plain) {
+    h.m32 = fmaxf(h.m32, as);
+    if (__fmaf_rn(-h.T, ar, as) > 0.0f) rel_update(h, (double)as, (double)r);
+    return bad ? 1u : 0u;
   }
   return exact_float(r, c, h, t);
 }
 
 template <uint32_t DT>
-__device__ __forceinline__ void record(uint32_t bad, unsigned long long idx, Hot &h) {
-  if (bad) { h.cnt += 1; h.first = umin64(h.first, idx); }
+__device__ __forceinline__ void settle_chunk(const QEntry &e, Hot &h, const TolF &t) {
+  constexpr int E = Fmt<DT>::E;
+  uint32_t bad = 0;
+#pragma unroll 1
+  for (int j = 0; j < E; ++j) {
+    if (DT == kI32 || DT == kI8 || DT == kU8) {
+      const int64_t r = elem_int<DT>(e.R, j), c = elem_int<DT>(e.C, j);
+      if (r != c) { exact_int(r, c, h); bad |= 1u << j; }
+    } else {
+      const uint32_t rb = elem_bits<DT>(e.R, j), cb = elem_bits<DT>(e.C, j);
+      if (rb != cb) bad |= settle_float(__uint_as_float(rb), __uint_as_float(cb), h, t) << j;
+    }
+  }
+  if (bad) {
+    h.cnt += __popc(bad);
+    h.first = umin64(h.first, e.e0 + (unsigned long long)(__ffs(bad) - 1));
+  }
 }
 
-// Drain the warp's queue: lanes take entries in turn; then every lane
+// Drain the warp's queue: lanes take chunks in turn; then every lane
 // adopts the warp's largest exact relative error (only the overall maximum
 // matters, so a shared threshold is as valid as a per-lane one).
 template <uint32_t DT>
 __device__ __noinline__ Hot drain(Queue *q, Hot h, const TolF t) {
   __syncwarp();
   const uint32_t n = min(q->count, kQueue);
-  for (uint32_t j = threadIdx.x & 31; j < n; j += 32) {
-    const QEntry e = q->e[j];
-    record<DT>(exact_elem<DT>(e.r, e.c, h, t), e.idx, h);
-  }
+  for (uint32_t j = threadIdx.x & 31; j < n; j += 32) settle_chunk<DT>(q->e[j], h, t);
   __syncwarp();
   if ((threadIdx.x & 31) == 0) q->count = 0;
-  unsigned long long rb = (unsigned long long)__double_as_longlong(h.drel);
+  unsigned long long rb = h.drel;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) rb = umax64(rb, __shfl_xor_sync(0xFFFFFFFFu, rb, o));
-  const double d = __longlong_as_double((long long)rb);
-  if (d > h.drel) { h.drel = d; h.T = tfloor(d); }
+  if (rb > h.drel) { h.drel = rb; h.T = tfloor(__longlong_as_double((long long)rb)); }
   __syncwarp();
   return h;
 }
 
+// A chunk that found the queue full is settled in its own lane.
 template <uint32_t DT>
-__device__ __forceinline__ uint32_t elem_bits(const uint4 &v, int j) {
-  if (DT == kI32 || DT == kI8 || DT == kU8) return (uint32_t)(int32_t)elem_int<DT>(v, j);
-  return __float_as_uint(elem_f32<DT>(v, j));
+__device__ __noinline__ Hot settle_overflow(const QEntry e, Hot h, const TolF t) {
+  settle_chunk<DT>(e, h, t);
+  return h;
 }
 
-// Queue the flagged elements of one chunk; a full queue falls back to
-// evaluating in this lane.
+// Queue one chunk.
 template <uint32_t DT>
-__device__ __noinline__ Hot push_rare(const uint4 R, const uint4 C, uint32_t rare,
-                                      unsigned long long e0, Queue *q, Hot h, const TolF t) {
-  while (rare) {
-    const int j = __ffs(rare) - 1;
-    rare &= rare - 1;
-    const uint32_t rb = elem_bits<DT>(R, j), cb = elem_bits<DT>(C, j);
-    const uint32_t slot = atomicAdd(&q->count, 1u);
-    if (slot < kQueue) {
-      QEntry e;
-      e.r = rb; e.c = cb; e.idx = e0 + (unsigned long long)j;
-      q->e[slot] = e;
-    } else {
-      record<DT>(exact_elem<DT>(rb, cb, h, t), e0 + (unsigned long long)j, h);
-    }
-  }
-  return h;
+__device__ __forceinline__ void push_chunk(const uint4 &R, const uint4 &C, unsigned long long e0,
+                                           Queue *q, Hot &h, const TolF &t) {
+  const uint32_t slot = atomicAdd(&q->count, 1u);
+  QEntry e;
+  e.R = R; e.C = C; e.e0 = e0;
+  if (slot < kQueue) q->e[slot] = e;
+  else h = settle_overflow<DT>(e, h, t);
+}
+
+// Screen of one element whose difference s is exact when it matters.
+// Returns the definite-mismatch bit; sets `rare` when the element needs the
+// exact path; accumulates the chunk's largest |s|.
+__device__ __forceinline__ uint32_t screen(float r, float s, float Tp, const TolF &t, bool &rare,
+                                          float &cm) {
+  const float as = fabsf(s), ar = fabsf(r);
+  const float lo = __fmaf_rn(t.rlo, ar, t.alo);
+  const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
+  const float y = __fmaf_rn(Tp, ar, 0x1p-149f);
+  const bool ok = as < lo;
+  const bool bad = as > hi;
+  rare |= (!(ok | bad)) | (as >= y);
+  cm = fmaxf(cm, as);
+  return bad ? 1u : 0u;
 }
 
 // One 16-byte chunk whose first element has index e0.
+//  - Equal chunks cost one comparison.
+//  - 16- and 8-bit floats subtract in their own format (one packed
+//    instruction per pair): the result is exact whenever |c-r| < |r|/2
+//    (Sterbenz), and every other element fails |s| < Tp*|r| <= |r|/2.
+//  - A packed s*0 accumulation turns any NaN or Inf into a NaN sentinel.
+//  - A chunk with any element the screen cannot settle is queued whole.
 template <uint32_t DT>
 __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e0, Hot &h,
                                       const TolF &t, Queue *q) {
   if (R.x == C.x && R.y == C.y && R.z == C.z && R.w == C.w) return;
-  uint32_t rare = 0;
   if (DT == kI32 || DT == kI8 || DT == kU8) {
-    // integers: every differing element is a mismatch, evaluated exactly
+    push_chunk<DT>(R, C, e0, q, h, t);          // integer differences are evaluated exactly
+    return;
+  }
+  const float Tp = fminf(h.T, ASMV_HALF_LESS);
+  bool rare = false;
+  float cm = 0.0f;
+  uint32_t bad = 0;
+  if (DT == kF32) {
+    float acc = 0.0f;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
-      const uint32_t d = word_of(R, w) ^ word_of(C, w);
-      if (DT == kI32) rare |= (uint32_t)(d != 0) << w;
-      else
-#pragma unroll
-        for (int qq = 0; qq < 4; ++qq) rare |= (uint32_t)(((d >> (8 * qq)) & 0xFFu) != 0) << (4 * w + qq);
+      const float r = __uint_as_float(word_of(R, w)), c = __uint_as_float(word_of(C, w));
+      const float s = __fsub_rn(c, r);
+      acc = __fmaf_rn(s, 0.0f, acc);
+      bad |= screen(r, s, Tp, t, rare, cm) << w;
     }
-  } else {
-    Masks m = {0u, 0u};
+    rare |= !(acc == 0.0f);
+  } else if (DT == kBF16) {
+    __nv_bfloat162 acc = __float2bfloat162_rn(0.0f);
+    const __nv_bfloat162 zero = acc;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const uint32_t rw = word_of(R, w), cw = word_of(C, w);
-      if (rw != cw) screen_word<DT>(rw, cw, w, h, t, m);
+      const __nv_bfloat162 s2 = __hsub2(*reinterpret_cast<const __nv_bfloat162 *>(&cw),
+                                        *reinterpret_cast<const __nv_bfloat162 *>(&rw));
+      acc = __hfma2(s2, zero, acc);
+      const uint32_t sw = *reinterpret_cast<const uint32_t *>(&s2);
+      bad |= screen(__uint_as_float(rw << 16), __uint_as_float(sw << 16), Tp, t, rare, cm) << (2 * w);
+      bad |= screen(__uint_as_float(rw & 0xFFFF0000u), __uint_as_float(sw & 0xFFFF0000u), Tp, t, rare,
+                    cm) << (2 * w + 1);
     }
-    const uint32_t bad = m.bad & ~m.rare;     // decided here; rare ones are decided exactly
-    if (bad) {
-      h.cnt += __popc(bad);
-      h.first = umin64(h.first, e0 + (uint64_t)(__ffs(bad) - 1));
+    const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
+    rare |= (aw & 0x7FFF7FFFu) != 0u;
+  } else {
+    // fp16, and fp8 widened to fp16 (exact)
+    __half2 acc = __float2half2_rn(0.0f);
+    const __half2 zero = acc;
+    constexpr int WORDS = (DT == kF16) ? 4 : 8;        // half2 pairs per chunk
+#pragma unroll
+    for (int w = 0; w < WORDS; ++w) {
+      uint32_t rw, cw;
+      if (DT == kF16) { rw = word_of(R, w); cw = word_of(C, w); }
+      else {
+        const __half2_raw rh = __nv_cvt_fp8x2_to_halfraw2(
+            (__nv_fp8x2_storage_t)((word_of(R, w >> 1) >> (16 * (w & 1))) & 0xFFFFu), __NV_E4M3);
+        const __half2_raw ch = __nv_cvt_fp8x2_to_halfraw2(
+            (__nv_fp8x2_storage_t)((word_of(C, w >> 1) >> (16 * (w & 1))) & 0xFFFFu), __NV_E4M3);
+        rw = (uint32_t)rh.x | ((uint32_t)rh.y << 16);
+        cw = (uint32_t)ch.x | ((uint32_t)ch.y << 16);
+      }
+      const __half2 s2 = __hsub2(*reinterpret_cast<const __half2 *>(&cw),
+                                 *reinterpret_cast<const __half2 *>(&rw));
+      acc = __hfma2(s2, zero, acc);
+      const float2 rf = f16x2_to_f32(rw);
+      const float2 sf = __half22float2(s2);
+      bad |= screen(rf.x, sf.x, Tp, t, rare, cm) << (2 * w);
+      bad |= screen(rf.y, sf.y, Tp, t, rare, cm) << (2 * w + 1);
     }
-    rare = m.rare;
+    const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
+    rare |= (aw & 0x7FFF7FFFu) != 0u;
   }
-  if (rare) h = push_rare<DT>(R, C, rare, e0, q, h, t);
+  if (rare) {
+    push_chunk<DT>(R, C, e0, q, h, t);
+    return;
+  }
+  h.m32 = fmaxf(h.m32, cm);
+  if (bad) {
+    h.cnt += __popc(bad);
+    h.first = umin64(h.first, e0 + (uint64_t)(__ffs(bad) - 1));
+  }
 }
 
 __device__ __forceinline__ void reset_hot(Hot &h) {
   h.cnt = 0; h.nonfin = 0; h.first = ~0ull;
-  h.m32 = 0.0f; h.T = 0.0f; h.dabs = 0.0; h.drel = 0.0;
+  h.m32 = 0.0f; h.T = 0.0f; h.dabs = 0; h.drel = 0;
 }
 
 // Merge a warp's statistics for region `ri`, candidate k into the global
@@ -313,9 +343,8 @@ __device__ __forceinline__ void reset_hot(Hot &h) {
 __device__ __forceinline__ void flush(Hot &h, const CmpParams &p, uint32_t k, uint32_t ri) {
   unsigned long long cnt = h.cnt, nonfin = h.nonfin;
   unsigned long long first = h.first;
-  const double a = fmax(h.dabs, (double)h.m32);
-  unsigned long long ab = (unsigned long long)__double_as_longlong(a);
-  unsigned long long rb = (unsigned long long)__double_as_longlong(h.drel);
+  unsigned long long ab = umax64(h.dabs, dbits((double)h.m32));
+  unsigned long long rb = h.drel;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
@@ -391,53 +420,107 @@ __device__ __forceinline__ TileInfo tile_info(const CmpRegion &r, uint64_t t, ui
   return ti;
 }
 
-// A warp's share of one tile for its candidate: chunks part*32 + lane +
-// j*32*W; staged chunks come from shared memory, the rest from global.
+// Pipeline position shared by a consumer warp's calls.
+struct Cursor {
+  uint32_t u;          // stage uses consumed so far
+  uint32_t ok;         // every wait succeeded
+};
+
+// The last rows of a short tile: lanes past its end are predicated off and
+// chunks beyond the staged part come from global memory.
 template <uint32_t DT>
-__device__ __noinline__ Hot tile(const CmpRegion r, uint64_t cbase, TileInfo ti, const uint4 *sref,
-                                 const uint4 *scand, uint32_t part, uint32_t W, Hot h, const TolF t,
-                                 Queue *q) {
+__device__ __noinline__ Hot tail_rows(const CmpRegion r, uint64_t cbase, const TileInfo ti,
+                                      const uint4 *sref, const uint4 *scand, uint32_t row,
+                                      uint32_t stride, Hot h, const TolF tol, Queue *q) {
   constexpr int E = Fmt<DT>::E;
-  constexpr int U = 2;
-  const uint64_t c0 = ti.off >> 4;
-  const uint64_t full = r.bytes >> 4;
-  const uint32_t stride = 32 * W;
-  uint32_t i0 = part * 32 + (threadIdx.x & 31);
-  for (; i0 + (U - 1) * stride < ti.nsm; i0 += U * stride) {
-    uint4 R[U], C[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) { R[u] = sref[i0 + u * stride]; C[u] = scand[i0 + u * stride]; }
-#pragma unroll
-    for (int u = 0; u < U; ++u) chunk<DT>(R[u], C[u], (c0 + i0 + u * stride) * E, h, t, q);
-    __syncwarp();
-    if (q->count >= kQueue / 2) h = drain<DT>(q, h, t);
-  }
-  for (uint32_t i = i0; i < ti.nloc; i += stride) {
-    uint4 R, C;
-    if (i < ti.nsm) { R = sref[i]; C = scand[i]; }
-    else {
-      R = load_chunk(r.ref, c0 + i, full, r.bytes, false);
-      C = load_chunk(cbase, c0 + i, full, r.bytes, false);
+  const uint32_t lane = threadIdx.x & 31;
+  const uint64_t c0 = ti.off >> 4, full_chunks = r.bytes >> 4;
+  for (; row < ti.nloc; row += stride) {
+    const uint32_t i = row + lane;
+    if (i < ti.nloc) {
+      uint4 R, C;
+      if (i < ti.nsm) { R = sref[i]; C = scand[i]; }
+      else {
+        R = load_chunk(r.ref, c0 + i, full_chunks, r.bytes, false);
+        C = load_chunk(cbase, c0 + i, full_chunks, r.bytes, false);
+      }
+      chunk<DT>(R, C, (c0 + i) * E, h, tol, q);
     }
-    chunk<DT>(R, C, (c0 + i) * E, h, t, q);
+    __syncwarp();
+    if (q->count >= kQueue / 2) h = drain<DT>(q, h, tol);
   }
-  __syncwarp();
-  if (q->count) h = drain<DT>(q, h, t);
   return h;
 }
 
-__device__ __forceinline__ Hot tile_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
-                                             TileInfo ti, const uint4 *sref, const uint4 *scand,
-                                             uint32_t part, uint32_t W, Hot h, Queue *q) {
-  switch (r.dtype) {
-    case kF32: return tile<kF32>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF32], q);
-    case kBF16: return tile<kBF16>(r, cbase, ti, sref, scand, part, W, h, p.tol[kBF16], q);
-    case kF16: return tile<kF16>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF16], q);
-    case kF8: return tile<kF8>(r, cbase, ti, sref, scand, part, W, h, p.tol[kF8], q);
-    case kI32: return tile<kI32>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
-    case kI8: return tile<kI8>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
-    default: return tile<kU8>(r, cbase, ti, sref, scand, part, W, h, p.tol[0], q);
+// A warp's share of the tiles [t, t_end) of one region for its candidate:
+// for every tile, wait for its stage, check chunks part*32 + lane + j*32*W
+// (staged chunks from shared memory, the rest from global), release the
+// stage.  One call per run of tiles keeps the per-tile cost to the waits.
+template <uint32_t DT>
+__device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, uint64_t t_end,
+                                const unsigned char *bufs, uint32_t stage_bytes, uint32_t cand_off,
+                                uint64_t *full, uint64_t *empty, uint32_t tile_bytes, uint32_t part,
+                                uint32_t W, bool active, Hot h, const TolF tol, Queue *q,
+                                Cursor *cur) {
+  constexpr int E = Fmt<DT>::E;
+  constexpr int U = 2;
+  const uint32_t stride = 32 * W;
+  const uint32_t lane = threadIdx.x & 31;
+  uint32_t u = cur->u;
+  for (; t < t_end; ++t, ++u) {
+    const uint32_t s = u % kStages;
+    if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u)) { cur->ok = 0; break; }
+    if (active) {
+      const TileInfo ti = tile_info(r, t, tile_bytes);
+      const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
+      const uint4 *scand = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes + cand_off);
+      const uint64_t c0 = ti.off >> 4;
+      // Rows of U*32*W chunks; every loop bound below is the same for all
+      // lanes of the warp, so the warp-wide __syncwarp and drain are reached
+      // by every lane.  Whole rows come from shared memory; the last rows of
+      // a short tile go through the predicated tail.
+      uint32_t row = part * 32;
+      for (; row + (U - 1) * stride + 31 < ti.nsm; row += U * stride) {
+        uint4 R[U], C[U];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          R[k] = sref[row + lane + k * stride];
+          C[k] = scand[row + lane + k * stride];
+        }
+#pragma unroll
+        for (int k = 0; k < U; ++k) chunk<DT>(R[k], C[k], (c0 + row + lane + k * stride) * E, h, tol, q);
+        __syncwarp();
+        if (q->count >= kQueue / 2) h = drain<DT>(q, h, tol);
+      }
+      if (row < ti.nloc) h = tail_rows<DT>(r, cbase, ti, sref, scand, row, stride, h, tol, q);
+      __syncwarp();
+      if (q->count) h = drain<DT>(q, h, tol);
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
   }
+  cur->u = u;
+  return h;
+}
+
+__device__ __forceinline__ Hot run_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
+                                            uint64_t t, uint64_t t_end, const unsigned char *bufs,
+                                            uint32_t stage_bytes, uint32_t cand_off, uint64_t *full,
+                                            uint64_t *empty, uint32_t part, uint32_t W, bool active,
+                                            Hot h, Queue *q, Cursor *cur) {
+  const uint32_t TB = p.tile_bytes;
+#define ASMV_RUN(DT, TOL) run<DT>(r, cbase, t, t_end, bufs, stage_bytes, cand_off, full, empty, TB, \
+                                  part, W, active, h, TOL, q, cur)
+  switch (r.dtype) {
+    case kF32: return ASMV_RUN(kF32, p.tol[kF32]);
+    case kBF16: return ASMV_RUN(kBF16, p.tol[kBF16]);
+    case kF16: return ASMV_RUN(kF16, p.tol[kF16]);
+    case kF8: return ASMV_RUN(kF8, p.tol[kF8]);
+    case kI32: return ASMV_RUN(kI32, p.tol[0]);
+    case kI8: return ASMV_RUN(kI8, p.tol[0]);
+    default: return ASMV_RUN(kU8, p.tol[0]);
+  }
+#undef ASMV_RUN
 }
 
 // Guard segments: one warp per segment; bad bytes and the first bad offset.
@@ -526,41 +609,27 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
       }
     }
   } else if (t0 < t1) {
-    // consumers
+    // consumers: one call per run of tiles of the same region
     const uint32_t W = kConsumerWarps / K;                  // warps per candidate
     const bool active = warp < W * K;
     const uint32_t k = warp % K, part = warp / K;
     Hot h;
     reset_hot(h);
+    Cursor cur;
+    cur.u = 0;
+    cur.ok = 1;
     uint32_t ri = find_region(p.regions, p.nregions, t0);
-    uint32_t u = 0;
-    for (uint64_t t = t0; t < t1; ++t, ++u) {
-      if (p.regions[ri + 1].tile0 <= t) {
-        if (active) flush(h, p, k, ri);
-        while (p.regions[ri + 1].tile0 <= t) ++ri;
-      }
-      const uint32_t s = u % kStages;
-      if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u)) {
-        ok = false;
-        break;
-      }
-      if (active) {
-        const CmpRegion r = p.regions[ri];
-        const TileInfo ti = tile_info(r, t, TB);
-        const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
-        const uint4 *scand = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes +
-                                                              (size_t)(1 + k) * TB);
-        h = tile_dispatch(p, r, p.cands[(size_t)k * p.nregions + ri], ti, sref, scand, part, W, h,
-                          &queues[warp]);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
+    uint64_t t = t0;
+    while (t < t1 && cur.ok) {
+      while (p.regions[ri + 1].tile0 <= t) ++ri;
+      const uint64_t t_end = umin64(t1, p.regions[ri + 1].tile0);
+      const CmpRegion r = p.regions[ri];
+      h = run_dispatch(p, r, p.cands[(size_t)k * p.nregions + ri], t, t_end, bufs, stage_bytes,
+                       (1 + k) * TB, full, empty, part, W, active, h, &queues[warp], &cur);
+      t = t_end;
+      if (active && cur.ok) flush(h, p, k, ri);
     }
-    if (!ok) {
-      if (lane == 0) atomicOr(p.err, 1u);
-    } else if (active) {
-      flush(h, p, k, ri);
-    }
+    if (!cur.ok && lane == 0) atomicOr(p.err, 1u);
   }
   guard_phase(p, warp, kConsumerWarps + 1);
 }

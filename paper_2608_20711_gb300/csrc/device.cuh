@@ -17,24 +17,25 @@
 namespace asmv {
 
 // ---------------------------------------------------------------- Philox
-// Round: (x0,x1,x2,x3) -> (hi(B*x2)^x1^k0, B*x2, hi(A*x0)^x3^k1, A*x0) with
-// A = 0xD2511F53, B = 0xCD9E8D57; key bumped by the Weyl increments
-// 0x9E3779B9 / 0xBB67AE85 between rounds (SC'11, Sec. 3).
-__device__ __forceinline__ uint4 philox10(uint4 x, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r) { k0 += 0x9E3779B9u; k1 += 0xBB67AE85u; }
-    const uint32_t a_hi = __umulhi(0xD2511F53u, x.x), a_lo = 0xD2511F53u * x.x;
-    const uint32_t b_hi = __umulhi(0xCD9E8D57u, x.z), b_lo = 0xCD9E8D57u * x.z;
-    x = make_uint4(b_hi ^ x.y ^ k0, b_lo, a_hi ^ x.w ^ k1, a_lo);
-  }
-  return x;
+// Philox4x32-10 round: (x0,x1,x2,x3) -> (hi(B*x2)^x1^k0, lo(B*x2), hi(A*x0)^x3^k1,
+// lo(A*x0)) with A = 0xD2511F53, B = 0xCD9E8D57; round r uses the key
+// (k0 + r*0x9E3779B9, k1 + r*0xBB67AE85) (SC'11, Sec. 3).
+// Ten rounds with the round keys given (one 64-bit product per multiplier;
+// the keys are kernel-parameter operands of the XORs).
+__device__ __forceinline__ void mul_wide(uint32_t a, uint32_t m, uint32_t &hi, uint32_t &lo) {
+  asm("{ .reg .u64 t; mul.wide.u32 t, %2, %3; mov.b64 {%1, %0}, t; }"
+      : "=r"(hi), "=r"(lo) : "r"(a), "r"(m));
 }
 
-// Block `b` of a region's payload stream.
-__device__ __forceinline__ uint4 payload_block(uint64_t seed, uint32_t region_id, uint64_t b) {
-  return philox10(make_uint4((uint32_t)b, (uint32_t)(b >> 32), region_id, 0u),
-                  (uint32_t)seed, (uint32_t)(seed >> 32));
+__device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, const uint32_t *k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    uint32_t ahi, alo, bhi, blo;
+    mul_wide(x.x, 0xD2511F53u, ahi, alo);
+    mul_wide(x.z, 0xCD9E8D57u, bhi, blo);
+    x = make_uint4(bhi ^ x.y ^ k0[r], blo, ahi ^ x.w ^ k1[r], alo);
+  }
+  return x;
 }
 
 // ---------------------------------------------------------------- Box-Muller
@@ -81,7 +82,8 @@ __device__ __forceinline__ float ln_u24(uint32_t k) {
   p = __fmaf_rn(z, p, ASMV_AT3);
   const float s2 = __fadd_rn(s, s);
   const float lnm = __fmaf_rn(__fmul_rn(s2, z), p, s2);
-  const float ef = (float)e;
+  // exact int -> float for |e| < 2^22: 1.5*2^23 + e has unit spacing
+  const float ef = __fsub_rn(__int_as_float(0x4B400000 + e), 12582912.0f);
   return __fmaf_rn(ef, ASMV_LN2_HI, __fmaf_rn(ef, ASMV_LN2_LO, lnm));
 }
 
@@ -90,7 +92,8 @@ __device__ __forceinline__ float ln_u24(uint32_t k) {
 __device__ __forceinline__ void sincos_u24(uint32_t k, float &sn, float &cs) {
   const uint32_t q = (k + (1u << 21)) >> 22;
   const int32_t ri = (int32_t)k - (int32_t)(q << 22);
-  const float r = __fmul_rn((float)ri, 0x1p-22f);
+  // r = ri * 2^-22 exactly: floats in [2, 4) are spaced 2^-22 apart
+  const float r = __fsub_rn(__int_as_float(0x40400000 + ri), 3.0f);
   const float r2 = __fmul_rn(r, r);
   float sp = __fmaf_rn(r2, ASMV_S9, ASMV_S7);
   sp = __fmaf_rn(r2, sp, ASMV_S5);

@@ -40,6 +40,15 @@ __device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span
   return (uint32_t)(lo + (int64_t)(((uint64_t)w * span) >> 32));
 }
 
+// Round keys of a launch.
+struct Keys {
+  const uint32_t *k0, *k1;
+};
+
+__device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id, uint64_t b) {
+  return philox10_keyed(make_uint4((uint32_t)b, (uint32_t)(b >> 32), region_id, 0u), K.k0, K.k1);
+}
+
 // Four fp32 values of one block, per float distribution.
 template <uint32_t DIST>
 __device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, float v[4]) {
@@ -49,18 +58,18 @@ __device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, float v[
 
 // The 16 bytes of chunk c.
 template <uint32_t DIST, uint32_t DT>
-__device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, uint64_t c) {
-  if (DIST == kRaw) return payload_block(seed, r.region_id, c);
+__device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, uint64_t c) {
+  if (DIST == kRaw) return payload_block(K, r.region_id, c);
   if (DIST == kIntRange) {
     if (DT == kI32) {
-      const uint4 w = payload_block(seed, r.region_id, c);
+      const uint4 w = payload_block(K, r.region_id, c);
       return make_uint4(int_of(w.x, r.ilo, r.ispan), int_of(w.y, r.ilo, r.ispan),
                         int_of(w.z, r.ilo, r.ispan), int_of(w.w, r.ilo, r.ispan));
     } else {                                    // 8-bit: 16 elements, blocks 4c..4c+3
       uint32_t out[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint4 w = payload_block(seed, r.region_id, 4 * c + q);
+        const uint4 w = payload_block(K, r.region_id, 4 * c + q);
         out[q] = (int_of(w.x, r.ilo, r.ispan) & 0xFFu) | ((int_of(w.y, r.ilo, r.ispan) & 0xFFu) << 8) |
                  ((int_of(w.z, r.ilo, r.ispan) & 0xFFu) << 16) | (int_of(w.w, r.ilo, r.ispan) << 24);
       }
@@ -70,7 +79,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, 
   // UNIFORM / NORMAL on float dtypes
   if (DT == kF32) {
     float v[4];
-    float4_of<DIST>(payload_block(seed, r.region_id, c), r, v);
+    float4_of<DIST>(payload_block(K, r.region_id, c), r, v);
     return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
                       __float_as_uint(v[3]));
   } else if (DT == kBF16 || DT == kF16) {       // 8 elements: blocks 2c, 2c+1
@@ -78,7 +87,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, 
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
       float v[4];
-      float4_of<DIST>(payload_block(seed, r.region_id, 2 * c + q), r, v);
+      float4_of<DIST>(payload_block(K, r.region_id, 2 * c + q), r, v);
       if (DT == kBF16) { out[2 * q] = pack_bf16x2(v[0], v[1]); out[2 * q + 1] = pack_bf16x2(v[2], v[3]); }
       else { out[2 * q] = pack_f16x2(v[0], v[1]); out[2 * q + 1] = pack_f16x2(v[2], v[3]); }
     }
@@ -88,7 +97,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, 
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       float v[4];
-      float4_of<DIST>(payload_block(seed, r.region_id, 4 * c + q), r, v);
+      float4_of<DIST>(payload_block(K, r.region_id, 4 * c + q), r, v);
       out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
     }
     return make_uint4(out[0], out[1], out[2], out[3]);
@@ -96,41 +105,41 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, uint64_t seed, 
 }
 
 template <uint32_t DIST, uint32_t DT>
-__device__ void fill_tile(const FillRegion &r, uint64_t seed, uint64_t tile_in_region) {
+__device__ void fill_tile(const FillRegion &r, const Keys &K, uint64_t tile_in_region) {
   const uint64_t c0 = tile_in_region * kTileChunks;
   const uint64_t nchunks = (r.bytes + 15) >> 4;
   const uint64_t full = r.bytes >> 4;
   const uint32_t nloc = (uint32_t)umin64(kTileChunks, nchunks - c0);
   for (uint32_t i = threadIdx.x; i < nloc; i += kThreads) {
     const uint64_t c = c0 + i;
-    const uint4 v = make_chunk<DIST, DT>(r, seed, c);
+    const uint4 v = make_chunk<DIST, DT>(r, K, c);
     const uint64_t addr = r.payload + 16 * c;
     if (r.vec && c < full) stg16(addr, v);
     else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * c));
   }
 }
 
-__device__ void fill_tile_dispatch(const FillRegion &r, uint64_t seed, uint64_t t) {
+__device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t t) {
   switch (r.dist) {
-    case kRaw: fill_tile<kRaw, kU8>(r, seed, t); break;
+    case kRaw: fill_tile<kRaw, kU8>(r, K, t); break;
     case kIntRange:
-      if (r.dtype == kI32) fill_tile<kIntRange, kI32>(r, seed, t);
-      else fill_tile<kIntRange, kI8>(r, seed, t);
+      if (r.dtype == kI32) fill_tile<kIntRange, kI32>(r, K, t);
+      else fill_tile<kIntRange, kI8>(r, K, t);
       break;
     case kUniform:
       switch (r.dtype) {
-        case kF32: fill_tile<kUniform, kF32>(r, seed, t); break;
-        case kBF16: fill_tile<kUniform, kBF16>(r, seed, t); break;
-        case kF16: fill_tile<kUniform, kF16>(r, seed, t); break;
-        default: fill_tile<kUniform, kF8>(r, seed, t); break;
+        case kF32: fill_tile<kUniform, kF32>(r, K, t); break;
+        case kBF16: fill_tile<kUniform, kBF16>(r, K, t); break;
+        case kF16: fill_tile<kUniform, kF16>(r, K, t); break;
+        default: fill_tile<kUniform, kF8>(r, K, t); break;
       }
       break;
     case kNormal:
       switch (r.dtype) {
-        case kF32: fill_tile<kNormal, kF32>(r, seed, t); break;
-        case kBF16: fill_tile<kNormal, kBF16>(r, seed, t); break;
-        case kF16: fill_tile<kNormal, kF16>(r, seed, t); break;
-        default: fill_tile<kNormal, kF8>(r, seed, t); break;
+        case kF32: fill_tile<kNormal, kF32>(r, K, t); break;
+        case kBF16: fill_tile<kNormal, kBF16>(r, K, t); break;
+        case kF16: fill_tile<kNormal, kF16>(r, K, t); break;
+        default: fill_tile<kNormal, kF8>(r, K, t); break;
       }
       break;
     default: break;                              // NONE: payload untouched
@@ -141,11 +150,12 @@ __global__ void __launch_bounds__(kThreads) fill_kernel(const FillParams p) {
   const uint64_t G = gridDim.x, b = blockIdx.x;
   const uint64_t t0 = p.ntiles * b / G, t1 = p.ntiles * (b + 1) / G;
   if (t0 < t1) {
+    const Keys K = {p.key0, p.key1};
     uint32_t ri = find_region(p.regions, p.nregions, t0);
     for (uint64_t t = t0; t < t1; ++t) {
       while (p.regions[ri + 1].tile0 <= t) ++ri;
       const FillRegion r = p.regions[ri];
-      fill_tile_dispatch(r, p.seed, t - r.tile0);
+      fill_tile_dispatch(r, K, t - r.tile0);
     }
   }
   // guard bands: one warp per segment

@@ -90,6 +90,9 @@ struct FillParams {
   uint64_t seed;
   uint32_t nregions;
   uint32_t nsegs;
+  // Philox key of each of the 10 rounds: (seed lo, seed hi) advanced by the
+  // Weyl increments, precomputed on the host (kernel-parameter operands)
+  uint32_t key0[10], key1[10];
 };
 
 struct CmpParams {

@@ -248,6 +248,65 @@ def test_compare_screen_boundaries(ctx, oracle, dtype, atol, rtol):
     assert_stats_equal(got, want, dtype)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16", "f8e4m3"])
+def test_compare_subnormal_differences(ctx, oracle, dtype):
+    """Pairs around the smallest normal value whose differences are
+    subnormal: a flush to zero anywhere would lose them."""
+    import torch
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16,
+           "f8e4m3": torch.float8_e4m3fn}[dtype]
+    st = {"f32": torch.int32, "bf16": torch.int16, "f16": torch.int16,
+          "f8e4m3": torch.uint8}[dtype]
+    mn = float(torch.finfo(tdt).tiny)
+    rng = np.random.default_rng(17)
+    n = 4096
+    r = mn * rng.uniform(1.0, 2.0, n) * rng.choice([-1, 1], n)
+    c = r * (1.0 + rng.uniform(-0.3, 0.3, n))
+    c[::7] = r[::7]                                   # some equal pairs
+    c[3::11] = 0.5 * r[3::11]                         # subnormal values themselves
+    R = torch.from_numpy(r).to(tdt).view(st).numpy().view(np.uint8).copy()
+    C = torch.from_numpy(c).to(tdt).view(st).numpy().view(np.uint8).copy()
+    reg = W.Region("s", dtype, n, "raw", 0, 0, 0, 0, 0xA5, 0)
+    reg.offset = 0
+    dref, dcand = to_device(R), to_device(C)
+    for tol in [{dtype: (0.0, 0.0)}, {dtype: (0.0, 1e-3)}]:
+        got = ctx.compare([asmv.make_region(dref.data_ptr(), n, dtype)],
+                          [asmv.make_region(dcand.data_ptr(), n, dtype)], tol)[0]
+        want = oracle_region_stats(oracle, R, reg, C, reg, tol)
+        assert_stats_equal(got, want, dtype)
+        assert want["mismatches"] > n // 2
+
+
+@pytest.mark.parametrize("k", [1, 8])
+def test_partial_tiles_of_every_shape(ctx, oracle, k):
+    """Region sizes that leave the last tile of each region at every
+    fraction of a tile, for the single (16 KiB tiles) and the batched
+    (4 KiB tiles) launch; dense differences keep the exact-path queue busy."""
+    rng = np.random.default_rng(100 + k)
+    regs = []
+    tile = TILE if k == 1 else 4096
+    for i, frac in enumerate(np.linspace(0.02, 0.98, 23)):
+        dt = ["f16", "bf16", "f32", "f8e4m3", "i8"][i % 5]
+        nb = tile * int(rng.integers(1, 4)) + int(frac * tile) + int(rng.integers(0, 16))
+        n = max(1, nb // W.DTYPE_SIZE[dt])
+        dist = "normal" if dt in W.FLOAT_DTYPES else "raw"
+        regs.append(W.Region("p%d" % i, dt, n, dist, 0.0, 1.0, 256, 256, 0xA5, i))
+    size = _place(regs)
+    ref = oracle_fill_arena(oracle, regs, size, 77)
+    cands = [_perturb_host(ref, regs, 300 + j, dense=True) for j in range(k)]
+    dref = to_device(ref)
+    dcs = [to_device(c) for c in cands]
+    rr = asmv.regions_in_arena(regs, dref.data_ptr())
+    if k == 1:
+        got = [ctx.compare(rr, asmv.regions_in_arena(regs, dcs[0].data_ptr()), TOL)]
+    else:
+        got = ctx.compare_batched(rr, [asmv.regions_in_arena(regs, d.data_ptr()) for d in dcs], TOL)
+    for j in range(k):
+        for r, g in zip(regs, got[j]):
+            want = oracle_region_stats(oracle, ref, r, cands[j], r, TOL)
+            assert_stats_equal(g, want, "cand %d %s" % (j, r.name))
+
+
 @pytest.mark.parametrize("k", [2, 8, 11])
 def test_batched_matches_oracle(ctx, oracle, k):
     regs = _cmp_table(31, n_regions=14)
