@@ -216,21 +216,39 @@ uint8_t oracle_f32_to_f8e4m3(float f) {
 }
 
 /* ======================================================================
- * fp32 Box-Muller pieces.  Coefficients are the Taylor coefficients of the
- * stated series, computed here in extended precision and rounded once to
- * fp32; every step below is one IEEE fp32 operation (fmaf where written).
+ * fp32 Box-Muller pieces.  Every step below is one IEEE fp32 operation
+ * (fmaf where written).
+ *
+ * ln(u), u = k 2^-24: u = m 2^e with m in [1, 2) and j = round(128 (m-1));
+ * with inv_j = round(32768/(128+j))/256 (eight significant bits) the
+ * reduction r = m*inv_j - 1 is exact in one fma and |r| < 2^-7; then
+ *   ln u = e ln2 + (-ln inv_j) + log1p(r),
+ * log1p(r) = r + r^2 (-1/2 + r (1/3 - r/4)), ln 2 and -ln inv_j each split
+ * into a head that is a multiple of 2^-9 (so e*head + head is exact) and an
+ * fp32 tail.  The table is computed here, in extended precision, from that
+ * definition.
+ * sin/cos: Taylor coefficients of the stated series, rounded once to fp32.
  * ====================================================================== */
-static float C_LN2_HI, C_LN2_LO, C_AT[5], C_S[5], C_C[6];
+static float C_LN2_HI, C_LN2_LO, C_THIRD, C_S[5], C_C[6];
+static float T_INV[129], T_HI[129], T_LO[129];
 static int consts_ready = 0;
 
 static void init_consts(void) {
   if (consts_ready) return;
   long double ln2 = logl(2.0L);
-  /* Cody-Waite split: a short head (9 significant bits) and the rest. */
+  /* Cody-Waite split of ln 2: a short head (9 significant bits) and the rest */
   C_LN2_HI = 355.0f / 512.0f;
   C_LN2_LO = (float)(ln2 - 355.0L / 512.0L);
-  /* atanh series: ln(m) = 2s (1 + s^2/3 + s^4/5 + ...), s = (m-1)/(m+1) */
-  for (int k = 0; k < 5; ++k) C_AT[k] = (float)(1.0L / (long double)(2 * k + 3));
+  C_THIRD = (float)(1.0L / 3.0L);
+  for (int j = 0; j <= 128; ++j) {
+    int den = 128 + j;
+    int I = (32768 + den / 2) / den;              /* round(32768/den); never a tie */
+    long double nl = logl(256.0L / (long double)I);
+    long double hi = nearbyintl(nl * 512.0L) / 512.0L;
+    T_INV[j] = (float)I / 256.0f;
+    T_HI[j] = (float)hi;
+    T_LO[j] = (float)(nl - hi);
+  }
   /* sin(pi/2 r) and cos(pi/2 r): coefficient of r^j is +-(pi/2)^j / j! */
   long double h = acosl(-1.0L) / 2.0L, p = 1.0L, fact = 1.0L;
   long double coef[12];
@@ -245,12 +263,20 @@ static void init_consts(void) {
   consts_ready = 1;
 }
 
-void oracle_boxmuller_consts(float out[18]) {
+/* [ln2 head, ln2 tail, 1/3, sin r^1..r^9 (5), cos r^0..r^10 (6)] */
+void oracle_boxmuller_consts(float out[14]) {
   init_consts();
-  out[0] = C_LN2_HI; out[1] = C_LN2_LO;
-  for (int k = 0; k < 5; ++k) out[2 + k] = C_AT[k];
-  for (int k = 0; k < 5; ++k) out[7 + k] = C_S[k];
-  for (int k = 0; k < 6; ++k) out[12 + k] = C_C[k];
+  out[0] = C_LN2_HI; out[1] = C_LN2_LO; out[2] = C_THIRD;
+  for (int k = 0; k < 5; ++k) out[3 + k] = C_S[k];
+  for (int k = 0; k < 6; ++k) out[8 + k] = C_C[k];
+}
+
+/* The ln reduction table: out[3j + 0..2] = inv_j, head_j, tail_j. */
+void oracle_ln_table(float out[387]) {
+  init_consts();
+  for (int j = 0; j <= 128; ++j) {
+    out[3 * j] = T_INV[j]; out[3 * j + 1] = T_HI[j]; out[3 * j + 2] = T_LO[j];
+  }
 }
 
 /* ln(k * 2^-24) for k in [1, 2^24], in fp32. */
@@ -259,20 +285,18 @@ float oracle_ln_u24(uint32_t k) {
   float u = (float)k * 0x1p-24f;                 /* exact */
   uint32_t b = f32_bits(u);
   int e = (int)(b >> 23) - 127;
-  float m = bits_f32((b & 0x7FFFFFu) | 0x3F800000u);   /* [1, 2) */
-  if (m > 1.41421356f) { m = m * 0.5f; e += 1; }       /* [sqrt2/2, sqrt2] */
-  float f = m - 1.0f;                              /* exact (Sterbenz) */
-  float s = f / (2.0f + f);
-  float z = s * s;
-  float p = fmaf(z, C_AT[4], C_AT[3]);
-  p = fmaf(z, p, C_AT[2]);
-  p = fmaf(z, p, C_AT[1]);
-  p = fmaf(z, p, C_AT[0]);
-  float s2 = s + s;
-  float lnm = fmaf(s2 * z, p, s2);
+  uint32_t mb = b & 0x7FFFFFu;
+  float m = bits_f32(mb | 0x3F800000u);          /* [1, 2) */
+  uint32_t j = (mb + (1u << 15)) >> 16;          /* round(128 (m - 1)), 0..128 */
+  float r = fmaf(m, T_INV[j], -1.0f);            /* exact */
+  float r2 = r * r;
+  float p = fmaf(r, -0.25f, C_THIRD);
+  p = fmaf(r, p, -0.5f);
+  float lp = fmaf(r2, p, r);
   float ef = (float)e;
-  float r = fmaf(ef, C_LN2_LO, lnm);
-  return fmaf(ef, C_LN2_HI, r);
+  float hi = fmaf(ef, C_LN2_HI, T_HI[j]);        /* exact */
+  float lo = fmaf(ef, C_LN2_LO, T_LO[j]);
+  return hi + (lo + lp);
 }
 
 /* sin and cos of 2*pi*k*2^-24 for k in [0, 2^24), in fp32. */

@@ -68,6 +68,7 @@ def lib():
             L.oracle_sincos_2pi_u24_many.argtypes = [_u32p, c.c_uint64, _f32p, _f32p]
             L.oracle_boxmuller_many.argtypes = [_u32p, _u32p, c.c_uint64, _f32p, _f32p]
             L.oracle_boxmuller_consts.argtypes = [_f32p]
+            L.oracle_ln_table.argtypes = [_f32p]
             L.oracle_encode_many.argtypes = [_f32p, c.c_uint64, c.c_int, _u8p]
             L.oracle_decode_many.argtypes = [_u8p, c.c_uint64, c.c_int, _f64p]
             L.oracle_fill_payload.argtypes = [_u8p, c.c_int, c.c_int, c.c_uint64,
@@ -139,9 +140,17 @@ def boxmuller(w0, w1):
 
 
 def boxmuller_consts():
-    out = np.empty(18, np.float32)
+    """[ln2 head, ln2 tail, 1/3, sin coefficients r^1..r^9, cos r^0..r^10]."""
+    out = np.empty(14, np.float32)
     lib().oracle_boxmuller_consts(_ptr(out, _f32p))
     return out
+
+
+def ln_table():
+    """(129, 3) array: inv_j, head_j, tail_j of the ln reduction."""
+    out = np.empty(129 * 3, np.float32)
+    lib().oracle_ln_table(_ptr(out, _f32p))
+    return out.reshape(129, 3)
 
 
 def encode(x, dtype):

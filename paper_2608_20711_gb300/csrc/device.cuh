@@ -39,19 +39,17 @@ __device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, con
 }
 
 // ---------------------------------------------------------------- Box-Muller
-// Series coefficients, each the fp32 rounding of the exact value:
-//   ln(m) = 2s (1 + s^2/3 + s^4/5 + ... + s^10/11),  s = (m-1)/(m+1)
-//   sin(pi/2 r) = sum_k (-1)^k (pi/2)^(2k+1) r^(2k+1) / (2k+1)!,  k = 0..4
-//   cos(pi/2 r) = sum_k (-1)^k (pi/2)^(2k) r^(2k) / (2k)!,        k = 0..5
-// ln 2 is split Cody-Waite style into 355/512 and the fp32 rounding of the
-// remainder.
+// ln(u), u = k 2^-24: u = m 2^e with m in [1, 2); j = round(128 (m - 1));
+// r = m*inv_j - 1 exactly (fma); ln u = e ln2 + (-ln inv_j) + log1p(r), with
+// ln 2 and -ln inv_j split into a 2^-9-multiple head (exact sum) and an fp32
+// tail, and log1p(r) = r + r^2 (-1/2 + r (1/3 - r/4)) for |r| < 2^-7.  The
+// table lives in shared memory (ln_table.h).
+// sin/cos(2 pi u): nearest quarter turn removed exactly in integers, then the
+// Taylor series of sin(pi/2 r) and cos(pi/2 r) for r in [-1/2, 1/2); each
+// coefficient is the fp32 rounding of +-(pi/2)^j / j!.
 #define ASMV_LN2_HI 0x1.63p-1f
 #define ASMV_LN2_LO (-0x1.bd0106p-13f)
-#define ASMV_AT3 0x1.555556p-2f
-#define ASMV_AT5 0x1.99999ap-3f
-#define ASMV_AT7 0x1.24924ap-3f
-#define ASMV_AT9 0x1.c71c72p-4f
-#define ASMV_AT11 0x1.745d18p-4f
+#define ASMV_THIRD 0x1.555556p-2f
 #define ASMV_S1 0x1.921fb6p+0f
 #define ASMV_S3 (-0x1.4abbcep-1f)
 #define ASMV_S5 0x1.466bc6p-4f
@@ -62,35 +60,29 @@ __device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, con
 #define ASMV_C6 (-0x1.55d3c8p-6f)
 #define ASMV_C8 0x1.e1f506p-11f
 #define ASMV_C10 (-0x1.a6d1f2p-16f)
-// fp32 nearest to sqrt(2): reduction threshold for the mantissa
-#define ASMV_SQRT2 0x1.6a09e6p+0f
 
-// ln(k 2^-24) for k in [1, 2^24]: exponent/mantissa split, mantissa folded
-// into [sqrt2/2, sqrt2], atanh series, e*ln2 added back in two parts.
-__device__ __forceinline__ float ln_u24(uint32_t k) {
+__device__ __forceinline__ float ln_u24(uint32_t k, const float4 *tab) {
   const float u = __fmul_rn(__uint2float_rn(k), 0x1p-24f);   // exact
   const uint32_t bits = __float_as_uint(u);
-  int e = (int)(bits >> 23) - 127;
-  float m = __uint_as_float((bits & 0x7FFFFFu) | 0x3F800000u);
-  if (m > ASMV_SQRT2) { m = __fmul_rn(m, 0.5f); e += 1; }
-  const float f = __fsub_rn(m, 1.0f);
-  const float s = __fdiv_rn(f, __fadd_rn(2.0f, f));
-  const float z = __fmul_rn(s, s);
-  float p = __fmaf_rn(z, ASMV_AT11, ASMV_AT9);
-  p = __fmaf_rn(z, p, ASMV_AT7);
-  p = __fmaf_rn(z, p, ASMV_AT5);
-  p = __fmaf_rn(z, p, ASMV_AT3);
-  const float s2 = __fadd_rn(s, s);
-  const float lnm = __fmaf_rn(__fmul_rn(s2, z), p, s2);
+  const int e = (int)(bits >> 23) - 127;
+  const uint32_t mb = bits & 0x7FFFFFu;
+  const float m = __uint_as_float(mb | 0x3F800000u);
+  const float4 t = tab[(mb + (1u << 15)) >> 16];             // inv, hi, lo
+  const float r = __fmaf_rn(m, t.x, -1.0f);                  // exact
+  const float r2 = __fmul_rn(r, r);
+  float p = __fmaf_rn(r, -0.25f, ASMV_THIRD);
+  p = __fmaf_rn(r, p, -0.5f);
+  const float lp = __fmaf_rn(r2, p, r);
   // exact int -> float for |e| < 2^22: 1.5*2^23 + e has unit spacing
   const float ef = __fsub_rn(__int_as_float(0x4B400000 + e), 12582912.0f);
-  return __fmaf_rn(ef, ASMV_LN2_HI, __fmaf_rn(ef, ASMV_LN2_LO, lnm));
+  const float hi = __fmaf_rn(ef, ASMV_LN2_HI, t.y);           // exact
+  const float lo = __fmaf_rn(ef, ASMV_LN2_LO, t.z);
+  return __fadd_rn(hi, __fadd_rn(lo, lp));
 }
 
-// sin and cos of 2 pi k 2^-24, k in [0, 2^24): nearest quarter turn q
-// removed exactly in integers, the remainder r in [-1/2, 1/2) quarter turns.
+// sin and cos of 2 pi k 2^-24, k in [0, 2^24).
 __device__ __forceinline__ void sincos_u24(uint32_t k, float &sn, float &cs) {
-  const uint32_t q = (k + (1u << 21)) >> 22;
+  const uint32_t q = (k + (1u << 21)) >> 22;                 // nearest quarter turn
   const int32_t ri = (int32_t)k - (int32_t)(q << 22);
   // r = ri * 2^-22 exactly: floats in [2, 4) are spaced 2^-22 apart
   const float r = __fsub_rn(__int_as_float(0x40400000 + ri), 3.0f);
@@ -105,16 +97,16 @@ __device__ __forceinline__ void sincos_u24(uint32_t k, float &sn, float &cs) {
   cp = __fmaf_rn(r2, cp, ASMV_C4);
   cp = __fmaf_rn(r2, cp, ASMV_C2);
   const float c = __fmaf_rn(r2, cp, 1.0f);
-  switch (q & 3u) {
-    case 0: sn = s; cs = c; break;
-    case 1: sn = c; cs = -s; break;
-    case 2: sn = -s; cs = -c; break;
-    default: sn = -c; cs = s; break;
-  }
+  // quarter turn q: (sin, cos) = (s, c), (c, -s), (-s, -c), (-c, s)
+  const bool odd = q & 1u;
+  const float a = odd ? c : s, b = odd ? s : c;
+  sn = __uint_as_float(__float_as_uint(a) ^ ((q & 2u) << 30));
+  cs = __uint_as_float(__float_as_uint(b) ^ (((q + 1u) & 2u) << 30));
 }
 
-__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, float &z0, float &z1) {
-  const float l = ln_u24((w0 >> 8) + 1u);
+__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const float4 *tab, float &z0,
+                                           float &z1) {
+  const float l = ln_u24((w0 >> 8) + 1u, tab);
   const float rho = __fsqrt_rn(__fmul_rn(-2.0f, l));
   float sn, cs;
   sincos_u24(w1 >> 8, sn, cs);

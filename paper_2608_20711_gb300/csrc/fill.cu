@@ -12,6 +12,7 @@
 // operations per 16-byte block) and Box-Muller for NORMAL also load the
 // ALUs, so 16-bit and 8-bit NORMAL fills are arithmetic-bound.
 #include "device.cuh"
+#include "ln_table.h"
 
 namespace asmv {
 namespace {
@@ -21,10 +22,10 @@ __device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
   return __fadd_rn(lo, __fmul_rn(f, width));
 }
 
-__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, float v[4]) {
+__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const float4 *tab, float v[4]) {
   float z[4];
-  box_muller(w.x, w.y, z[0], z[1]);
-  box_muller(w.z, w.w, z[2], z[3]);
+  box_muller(w.x, w.y, tab, z[0], z[1]);
+  box_muller(w.z, w.w, tab, z[2], z[3]);
 #pragma unroll
   for (int j = 0; j < 4; ++j) v[j] = __fadd_rn(mean, __fmul_rn(sd, z[j]));
 }
@@ -40,9 +41,10 @@ __device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span
   return (uint32_t)(lo + (int64_t)(((uint64_t)w * span) >> 32));
 }
 
-// Round keys of a launch.
+// Round keys of a launch and the ln table (in shared memory).
 struct Keys {
   const uint32_t *k0, *k1;
+  const float4 *lntab;
 };
 
 __device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id, uint64_t b) {
@@ -51,8 +53,8 @@ __device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id
 
 // Four fp32 values of one block, per float distribution.
 template <uint32_t DIST>
-__device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, float v[4]) {
-  if (DIST == kNormal) normal4(w, r.f0, r.f1, v);
+__device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, const Keys &K, float v[4]) {
+  if (DIST == kNormal) normal4(w, r.f0, r.f1, K.lntab, v);
   else uniform4(w, r.f0, r.f1, v);
 }
 
@@ -79,7 +81,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
   // UNIFORM / NORMAL on float dtypes
   if (DT == kF32) {
     float v[4];
-    float4_of<DIST>(payload_block(K, r.region_id, c), r, v);
+    float4_of<DIST>(payload_block(K, r.region_id, c), r, K, v);
     return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
                       __float_as_uint(v[3]));
   } else if (DT == kBF16 || DT == kF16) {       // 8 elements: blocks 2c, 2c+1
@@ -87,7 +89,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
       float v[4];
-      float4_of<DIST>(payload_block(K, r.region_id, 2 * c + q), r, v);
+      float4_of<DIST>(payload_block(K, r.region_id, 2 * c + q), r, K, v);
       if (DT == kBF16) { out[2 * q] = pack_bf16x2(v[0], v[1]); out[2 * q + 1] = pack_bf16x2(v[2], v[3]); }
       else { out[2 * q] = pack_f16x2(v[0], v[1]); out[2 * q + 1] = pack_f16x2(v[2], v[3]); }
     }
@@ -97,7 +99,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       float v[4];
-      float4_of<DIST>(payload_block(K, r.region_id, 4 * c + q), r, v);
+      float4_of<DIST>(payload_block(K, r.region_id, 4 * c + q), r, K, v);
       out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
     }
     return make_uint4(out[0], out[1], out[2], out[3]);
@@ -147,10 +149,13 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
 }
 
 __global__ void __launch_bounds__(kThreads) fill_kernel(const FillParams p) {
+  __shared__ float4 lntab[ASMV_LN_TABLE_ROWS];
+  for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS; i += kThreads) lntab[i] = kLnTableInit[i];
+  __syncthreads();
   const uint64_t G = gridDim.x, b = blockIdx.x;
   const uint64_t t0 = p.ntiles * b / G, t1 = p.ntiles * (b + 1) / G;
   if (t0 < t1) {
-    const Keys K = {p.key0, p.key1};
+    const Keys K = {p.key0, p.key1, lntab};
     uint32_t ri = find_region(p.regions, p.nregions, t0);
     for (uint64_t t = t0; t < t1; ++t) {
       while (p.regions[ri + 1].tile0 <= t) ++ri;

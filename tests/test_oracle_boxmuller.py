@@ -35,30 +35,49 @@ def test_sincos_2pi_u24_all_inputs(oracle):
     assert (sn[3 * q], cs[3 * q]) == (-1.0, 0.0)
 
 
+def _rn32(mpmath, x):
+    """Correctly rounded fp32 of a 50-digit value."""
+    f = np.float32(float(x))
+    cands = [np.nextafter(f, np.float32(-np.inf)), f, np.nextafter(f, np.float32(np.inf))]
+    return min(cands, key=lambda c: abs(mpmath.mpf(float(c)) - x))
+
+
 def test_series_coefficients_are_correctly_rounded(oracle):
     mpmath = pytest.importorskip("mpmath")
     mpmath.mp.dps = 50
-
-    def rn32(x):
-        # correctly rounded fp32 of a 50-digit value: nearest of the two
-        # fp32 neighbours of the float64 approximation
-        f = np.float32(float(x))
-        cands = [np.nextafter(f, np.float32(-np.inf)), f, np.nextafter(f, np.float32(np.inf))]
-        return min(cands, key=lambda c: abs(mpmath.mpf(float(c)) - x))
-
     c = oracle.boxmuller_consts()
     ln2 = mpmath.log(2)
     assert c[0] == np.float32(355.0 / 512.0)
-    assert c[1] == rn32(ln2 - mpmath.mpf(355) / 512)
-    for k in range(5):
-        assert c[2 + k] == rn32(mpmath.mpf(1) / (2 * k + 3))
+    assert c[1] == _rn32(mpmath, ln2 - mpmath.mpf(355) / 512)
+    assert c[2] == _rn32(mpmath, mpmath.mpf(1) / 3)
     h = mpmath.pi / 2
     for k in range(5):                       # sin: r^1, r^3, ..., r^9
         j = 2 * k + 1
-        assert c[7 + k] == rn32((-1) ** k * h ** j / mpmath.factorial(j))
+        assert c[3 + k] == _rn32(mpmath, (-1) ** k * h ** j / mpmath.factorial(j))
     for k in range(6):                       # cos: r^0, r^2, ..., r^10
         j = 2 * k
-        assert c[12 + k] == rn32((-1) ** k * h ** j / mpmath.factorial(j))
+        assert c[8 + k] == _rn32(mpmath, (-1) ** k * h ** j / mpmath.factorial(j))
+
+
+def test_ln_table_entries_and_exact_reduction(oracle):
+    """Each row: inv_j = round(32768/(128+j))/256, head = -ln(inv_j) rounded
+    to a multiple of 2^-9, tail = fp32 of the rest; every mantissa of a
+    bucket gives |m*inv_j - 1| < 2^-7 (so one fma is exact)."""
+    mpmath = pytest.importorskip("mpmath")
+    mpmath.mp.dps = 50
+    t = oracle.ln_table()
+    for j in range(129):
+        I = int(mpmath.nint(mpmath.mpf(32768) / (128 + j)))
+        assert t[j, 0] == np.float32(I / 256.0)
+        nl = mpmath.log(mpmath.mpf(256) / I)
+        hi = mpmath.nint(nl * 512) / 512
+        assert t[j, 1] == np.float32(float(hi))
+        assert t[j, 2] == _rn32(mpmath, nl - hi)
+        lo_m = max(1.0, 1 + (j - 0.5) / 128)
+        hi_m = min(2 - 2.0 ** -23, 1 + (j + 0.5) / 128)
+        for m in (lo_m, hi_m):
+            assert abs(m * float(t[j, 0]) - 1) < 2.0 ** -7
+    assert (t[128, 1], t[128, 2]) == (oracle.boxmuller_consts()[0], oracle.boxmuller_consts()[1])
 
 
 def test_boxmuller_is_standard_normal(oracle):
