@@ -116,13 +116,14 @@ __device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const float
 
 // ---------------------------------------------------------------- encoders
 // Hardware round-to-nearest-even conversions (fp8: saturating to +-448).
+// (one packed conversion per pair; a goes to the low half)
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-  const __nv_bfloat16 x = __float2bfloat16_rn(a), y = __float2bfloat16_rn(b);
-  return (uint32_t)__bfloat16_as_ushort(x) | ((uint32_t)__bfloat16_as_ushort(y) << 16);
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t *>(&v);
 }
 __device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
-  const __half x = __float2half_rn(a), y = __float2half_rn(b);
-  return (uint32_t)__half_as_ushort(x) | ((uint32_t)__half_as_ushort(y) << 16);
+  const __half2 v = __floats2half2_rn(a, b);
+  return *reinterpret_cast<const uint32_t *>(&v);
 }
 __device__ __forceinline__ uint32_t pack_f8x4(float a, float b, float c, float d) {
   const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
