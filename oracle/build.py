@@ -13,14 +13,20 @@ SRC = os.path.join(HERE, "asmv_oracle.c")
 LIB = os.path.join(HERE, "liboracle.so")
 
 
+def compile_library(src: str, out: str) -> str:
+    """Compile an oracle source file (this one, or an edited copy) to `out`."""
+    cmd = ["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fno-fast-math",
+           "-fPIC", "-shared", "-Wall", "-Wextra", "-o", out, src, "-lm"]
+    subprocess.check_call(cmd)
+    return out
+
+
 def build(force: bool = False) -> str:
     if (not force and os.path.exists(LIB)
             and os.path.getmtime(LIB) >= os.path.getmtime(SRC)):
         return LIB
     tmp = LIB + ".tmp.%d" % os.getpid()
-    cmd = ["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fno-fast-math",
-           "-fPIC", "-shared", "-Wall", "-Wextra", "-o", tmp, SRC, "-lm"]
-    subprocess.check_call(cmd)
+    compile_library(SRC, tmp)
     os.replace(tmp, LIB)
     return LIB
 

@@ -59,7 +59,33 @@ def lib():
     global _lib
     with _lock:
         if _lib is None:
-            path = _build.build()
+            _lib = _load(_build.build())
+    return _lib
+
+
+class use_library:
+    """Context manager: route this module's calls to another build of the
+    oracle (the tests use it to run the pins against planted mistakes)."""
+
+    def __init__(self, path):
+        self.path = path
+
+    def __enter__(self):
+        global _lib
+        with _lock:
+            self.saved = _lib
+            _lib = _load(self.path)
+        return self
+
+    def __exit__(self, *exc):
+        global _lib
+        with _lock:
+            _lib = self.saved
+
+
+def _load(path):
+    if True:
+        if True:
             L = ctypes.CDLL(path)
             c = ctypes
             L.oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
@@ -87,8 +113,7 @@ def lib():
                 _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
                 c.c_uint64, c.c_int, c.c_double, c.c_double,
                 c.POINTER(_RegionStats)]
-            _lib = L
-    return _lib
+    return L
 
 
 def _ptr(a, t):

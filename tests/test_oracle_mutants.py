@@ -1,0 +1,186 @@
+"""Planted mistakes in the oracle must each fail at least one of its pins.
+
+Each mutant below is one plausible slip in oracle/asmv_oracle.c: a dropped
+term, a wrong sign, index or operand, a wrong rounding or tie rule, an
+off-by-one scale.  The test compiles the edited source with the oracle's
+own flags into a temporary library, routes the oracle module to it, and
+runs the oracle's pin tests (every test_oracle_* function and every
+parametrisation of it) from cheapest to dearest until one fails.  A mutant
+that passes every pin would mean the pins do not fix that part of the
+oracle, so it fails this test.  All of it runs on the CPU.
+"""
+import importlib
+import itertools
+import os
+
+import pytest
+
+from oracle import build as oracle_build
+from oracle import oracle as O
+
+PIN_MODULES = ("tests.test_oracle_codecs", "tests.test_oracle_philox",
+               "tests.test_oracle_fill", "tests.test_oracle_compare",
+               "tests.test_oracle_boxmuller")
+# pins that take seconds run last, in this order
+EXPENSIVE = ("test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
+             "test_ln_u24_all_inputs")
+
+# (name, text in the oracle source, replacement): each text occurs once
+MUTANTS = [
+    # Philox4x32-10 (Salmon et al., SC'11)
+    ("philox_key_bump_dropped", "k0 += PHILOX_W_0; k1 += PHILOX_W_1;", "k0 += PHILOX_W_0;"),
+    ("philox_bump_before_first_round", "if (round > 0) {", "if (round >= 0) {"),
+    ("philox_xor_wrong_word", "uint32_t y0 = pb_hi ^ x1 ^ k0;", "uint32_t y0 = pb_hi ^ x3 ^ k0;"),
+    ("philox_same_multiplier",
+     "uint64_t pa = (uint64_t)PHILOX_M_A * (uint64_t)x0;",
+     "uint64_t pa = (uint64_t)PHILOX_M_B * (uint64_t)x0;"),
+    ("philox_low_halves_swapped", "uint32_t y1 = pb_lo;", "uint32_t y1 = pa_lo;"),
+    ("counter_words_transposed",
+     "{(uint32_t)b, (uint32_t)(b >> 32), region_id, 0u}",
+     "{(uint32_t)b, region_id, (uint32_t)(b >> 32), 0u}"),
+    # storage formats
+    ("f16_subnormal_scale", "else if (ex == 0) v = ldexp((double)man, -24);",
+     "else if (ex == 0) v = ldexp((double)man, -25);"),
+    ("f16_exponent_bias", "ldexp((double)(1024 + man), ex - 25)",
+     "ldexp((double)(1024 + man), ex - 24)"),
+    ("f8_subnormal_scale", "ldexp((double)man, -9)", "ldexp((double)man, -10)"),
+    ("bf16_round_half_up", "u += 0x7FFFu + lsb;", "u += 0x8000u;"),
+    ("rne_ties_away", "(rem == half && (q & 1u))", "(rem == half)"),
+    ("f8_overflow_to_nan", "if (bits_f32(a) >= 448.0f) return (uint8_t)(sign | 0x7Eu);",
+     "if (bits_f32(a) >= 448.0f) return (uint8_t)(sign | 0x7Fu);"),
+    ("f16_underflow_cut", "if (e < -25) return sign;", "if (e < -24) return sign;"),
+    # Box-Muller in fp32
+    ("log1p_quartic_sign", "fmaf(r, -0.25f, C_THIRD)", "fmaf(r, 0.25f, C_THIRD)"),
+    ("ln2_tail_dropped", "float lo = fmaf(ef, C_LN2_LO, T_LO[j]);", "float lo = T_LO[j];"),
+    ("ln_table_truncated", "int I = (32768 + den / 2) / den;", "int I = 32768 / den;"),
+    ("series_sign_pattern", "if ((j / 2) % 2 == 1) c = -c;", "if (j % 2 == 1) c = -c;"),
+    ("quarter_turn_truncated", "uint32_t q = (k + (1u << 21)) >> 22;", "uint32_t q = k >> 22;"),
+    ("quadrant_sign", "case 1: *sn_out = cs;  *cs_out = -sn; break;",
+     "case 1: *sn_out = cs;  *cs_out = sn; break;"),
+    ("radius_factor_dropped", "float rho = sqrtf(-2.0f * l);", "float rho = sqrtf(-l);"),
+    ("u1_offset_dropped", "oracle_ln_u24((w0 >> 8) + 1u)", "oracle_ln_u24(w0 >> 8)"),
+    ("cos_sin_outputs_swapped", "*z0 = rho * cs;\n  *z1 = rho * sn;",
+     "*z0 = rho * sn;\n  *z1 = rho * cs;"),
+    # Tier-1 fill
+    ("raw_big_endian", "(uint8_t)(word >> (8 * (j % 4)))", "(uint8_t)(word >> (8 * (3 - j % 4)))"),
+    ("int_range_modulo", "uint64_t off = ((uint64_t)w[i % 4] * span) >> 32;",
+     "uint64_t off = (uint64_t)w[i % 4] % span;"),
+    ("uniform_sign", "float v = lo + f * width;", "float v = lo - f * width;"),
+    ("uniform_fraction_bits", "float f = (float)(w[i % 4] >> 8) * 0x1p-24f;",
+     "float f = (float)(w[i % 4] >> 9) * 0x1p-23f;"),
+    ("normal_pair_index", "unsigned pair = (unsigned)((i % 4) / 2);",
+     "unsigned pair = (unsigned)((i % 4) % 2);"),
+    ("normal_affine_order", "float v = mean + sd * z;", "float v = sd + mean * z;"),
+    ("guard_band_misplaced", "uint8_t *hi = alloc + glo + payload_bytes;",
+     "uint8_t *hi = alloc + payload_bytes;"),
+    # guard check and the equivalence predicate
+    ("guard_first_relative", "first = base + j;", "first = j;"),
+    ("guard_hi_base", "uint64_t base = (uint64_t)glo + payload_bytes;",
+     "uint64_t base = payload_bytes;"),
+    ("guards_of_reference_reported",
+     "oracle_guard_check(cand_alloc, bytes, cand_glo, cand_ghi, cand_canary, &gbad, &gfirst);",
+     "oracle_guard_check(ref_alloc, bytes, cand_glo, cand_ghi, cand_canary, &gbad, &gfirst);"),
+    ("nan_pair_mismatch", "if (isnan(r) && isnan(c)) mismatch = 0;", "if (0) mismatch = 0;"),
+    ("inf_sign_ignored", "isinf(r) && isinf(c) && (signbit(r) == signbit(c))",
+     "isinf(r) && isinf(c)"),
+    ("bound_on_candidate", "double bound = atol + rtol * fabs(r);",
+     "double bound = atol + rtol * fabs(c);"),
+    ("bound_inclusive", "mismatch = d > bound;", "mismatch = d >= bound;"),
+    ("rel_on_candidate", "if (r != 0.0) rel_err = d / fabs(r);",
+     "if (r != 0.0) rel_err = d / fabs(c);"),
+    ("rel_zero_reference", "else rel_err = (d == 0.0) ? 0.0 : INFINITY;",
+     "else rel_err = d;"),
+    ("last_mismatch_kept", "if (st.first_mismatch == UINT64_MAX) st.first_mismatch = i;",
+     "st.first_mismatch = i;"),
+    ("int_compare_one_sided", "(size_t)sz) != 0;", "(size_t)sz) > 0;"),
+    ("nonfinite_not_counted", "else { mismatch = 1; st.nonfinite_mismatches += 1; }",
+     "else { mismatch = 1; }"),
+]
+
+
+def _params(fn):
+    """Every argument binding of a test function's parametrize marks."""
+    axes = []
+    for m in getattr(fn, "pytestmark", []):
+        if m.name != "parametrize":
+            continue
+        names, values = m.args[0], m.args[1]
+        names = [n.strip() for n in names.split(",")] if isinstance(names, str) else list(names)
+        rows = []
+        for v in values:
+            if hasattr(v, "values") and hasattr(v, "marks"):     # pytest.param(...)
+                v = tuple(v.values)
+            elif len(names) == 1:
+                v = (v,)
+            rows.append(dict(zip(names, v)))
+        axes.append(rows)
+    for combo in itertools.product(*axes):
+        kw = {}
+        for d in combo:
+            kw.update(d)
+        yield kw
+
+
+def _pins(torch_philox, cheap_only=False):
+    """(label, zero-argument callable) for every pin, cheapest first."""
+    found = []
+    for modname in PIN_MODULES:
+        mod = importlib.import_module(modname)
+        for name, fn in vars(mod).items():
+            if not name.startswith("test_") or not callable(fn):
+                continue
+            if cheap_only and name in EXPENSIVE:
+                continue
+            argnames = fn.__code__.co_varnames[:fn.__code__.co_argcount]
+            for kw in _params(fn):
+                call = dict(kw)
+                if "oracle" in argnames:
+                    call["oracle"] = O
+                if "torch_philox" in argnames:
+                    call["torch_philox"] = torch_philox
+                label = "%s::%s%s" % (modname.split(".")[-1], name,
+                                      sorted(kw.items()) if kw else "")
+                rank = EXPENSIVE.index(name) + 1 if name in EXPENSIVE else 0
+                found.append((rank, len(found), label, fn, call))
+    found.sort(key=lambda t: (t[0], t[1]))
+    return [(label, (lambda f=fn, c=call: f(**c))) for _, _, label, fn, call in found]
+
+
+def _first_failing_pin(pins):
+    for label, run in pins:
+        try:
+            run()
+        except Exception as e:                      # an assertion, or a raise
+            return label, type(e).__name__
+    return None
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(oracle_build.SRC) as f:
+        return f.read()
+
+
+def _compile(tmp_path, text, name):
+    src = tmp_path / (name + ".c")
+    src.write_text(text)
+    return oracle_build.compile_library(str(src), str(tmp_path / ("lib" + name + ".so")))
+
+
+def test_runner_passes_the_unmodified_oracle(tmp_path, source, torch_philox):
+    """The same runner on an unmodified copy: every (cheap) pin passes, so a
+    failure below is the planted mistake's doing."""
+    pins = _pins(torch_philox, cheap_only=True)
+    assert len(pins) > 60
+    with O.use_library(_compile(tmp_path, source, "pristine")):
+        assert _first_failing_pin(pins) is None
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_fails_a_pin(tmp_path, source, torch_philox, name, old, new):
+    assert source.count(old) == 1, "mutation site of %s not unique" % name
+    path = _compile(tmp_path, source.replace(old, new), name)
+    with O.use_library(path):
+        caught = _first_failing_pin(_pins(torch_philox))
+    assert caught is not None, "no pin fails with the mutant %s" % name
+    os.remove(path)
