@@ -538,6 +538,81 @@ void oracle_compare_region(const uint8_t *ref_alloc, uint32_t ref_glo,
 }
 
 /* ======================================================================
+ * Eq. 1 aggregate terms.  The cosine c_x = cos(K'(x), O(x)) of a float
+ * region is built from three sums over its elements:
+ *   S_rc = sum r*c,   S_rr = sum r*r,   S_cc = sum c*c.
+ * Readings (the paper gives the formula only):
+ *   R8 The sums run over the finite pairs; a pair with a NaN or an Inf on
+ *      either side is judged by the NaN/Inf rule (R4) instead.
+ *   R9 The sums are exact, then rounded once to fp64 (nearest, ties to
+ *      even): every decoded value has at most 24 significant bits, so each
+ *      product is exact in fp64, and the products are added here without
+ *      rounding, into a fixed-point integer of OEQ_DIGITS signed 64-bit
+ *      digits, digit k weighing 2^(32 k + OEQ_BASE).  The final rounding is
+ *      done by the caller from the digits.
+ * The range covers every product of two fp32 values (2^-298 .. 2^256) with
+ * 2^64 of headroom for the sum.
+ * ====================================================================== */
+#define OEQ_DIGITS 20
+#define OEQ_BASE (-320)
+
+/* Carry-propagate: digits 0 .. OEQ_DIGITS-2 end in [0, 2^32), the top digit
+ * keeps the sign. */
+static void eq_normalize(int64_t *acc) {
+  for (int k = 0; k < OEQ_DIGITS - 1; ++k) {
+    int64_t carry = acc[k] >> 32;          /* floor division by 2^32 */
+    acc[k] -= carry * 4294967296LL;
+    acc[k + 1] += carry;
+  }
+}
+
+/* acc += p, for p an exact fp64 product; returns nothing, exact. */
+static void eq_add(int64_t *acc, double p) {
+  if (p == 0.0) return;
+  int e;
+  double f = frexp(fabs(p), &e);                   /* |p| = f 2^e, f in [0.5, 1) */
+  uint64_t m = (uint64_t)ldexp(f, 53);             /* exact: 53-bit integer */
+  int lsb = e - 53;                                /* |p| = m 2^lsb */
+  while ((m & 1u) == 0) { m >>= 1; ++lsb; }
+  int pos = lsb - OEQ_BASE;                        /* >= 22 for any fp32 product */
+  int q = pos / 32, b = pos % 32;
+  /* m 2^b spans at most three 32-bit digits */
+  uint64_t lo = (m << b) & 0xFFFFFFFFu;
+  uint64_t mid = (b == 0) ? (m >> 32) : ((m >> (32 - b)) & 0xFFFFFFFFu);
+  uint64_t hi = (b == 0) ? 0 : (m >> (64 - b));
+  int64_t sg = (p < 0.0) ? -1 : 1;
+  acc[q] += sg * (int64_t)lo;
+  acc[q + 1] += sg * (int64_t)mid;
+  acc[q + 2] += sg * (int64_t)hi;
+}
+
+/* The three sums over elements [i0, i1) of two payloads of float dtype dt,
+ * as normalized digits: out[0..D) = S_rc, out[D..2D) = S_rr,
+ * out[2D..3D) = S_cc.  Integer and opaque dtypes give zeros. */
+void oracle_eq_sums_range(const uint8_t *ref, const uint8_t *cand, int dt,
+                          uint64_t i0, uint64_t i1, int64_t *out) {
+  int64_t *rc = out, *rr = out + OEQ_DIGITS, *cc = out + 2 * OEQ_DIGITS;
+  for (int k = 0; k < 3 * OEQ_DIGITS; ++k) out[k] = 0;
+  if (!is_float_dtype(dt)) return;
+  uint64_t since = 0;
+  for (uint64_t i = i0; i < i1; ++i) {
+    double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);
+    if (!isfinite(r) || !isfinite(c)) continue;
+    eq_add(rc, r * c);
+    eq_add(rr, r * r);
+    eq_add(cc, c * c);
+    if (++since == (1u << 20)) {     /* each digit grows by < 2^32 per add */
+      eq_normalize(rc); eq_normalize(rr); eq_normalize(cc);
+      since = 0;
+    }
+  }
+  eq_normalize(rc); eq_normalize(rr); eq_normalize(cc);
+}
+
+int oracle_eq_digits(void) { return OEQ_DIGITS; }
+int oracle_eq_base(void) { return OEQ_BASE; }
+
+/* ======================================================================
  * Batch entry points for the tests (plain loops over the functions above).
  * ====================================================================== */
 void oracle_philox_many(const uint32_t *ctr, const uint32_t *key, uint64_t n,

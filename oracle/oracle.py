@@ -28,6 +28,7 @@ CODE_OF_DTYPE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": 
 CODE_OF_DIST = {"raw": RAW, "uniform": UNIFORM, "normal": NORMAL, "int_range": INT_RANGE,
                 "none": NONE}
 
+_i64p = ctypes.POINTER(ctypes.c_int64)
 _u8p = ctypes.POINTER(ctypes.c_uint8)
 _u32p = ctypes.POINTER(ctypes.c_uint32)
 _f32p = ctypes.POINTER(ctypes.c_float)
@@ -113,6 +114,8 @@ def _load(path):
                 _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
                 c.c_uint64, c.c_int, c.c_double, c.c_double,
                 c.POINTER(_RegionStats)]
+            L.oracle_eq_sums_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
+                                               c.c_uint64, _i64p]
     return L
 
 
@@ -300,3 +303,75 @@ def host_threads():
         return len(os.sched_getaffinity(0))
     except AttributeError:
         return os.cpu_count() or 1
+
+
+# ------------------------------------------- Eq. 1 aggregate (cosine) terms
+EQ_DIGITS, EQ_BASE = 20, -320
+EQ_COS, EQ_LINF, EQ_INT, EQ_GUARD = 1, 2, 4, 8
+THETA, TAU = 0.9999, 1e-3          # the paper's thresholds for Eq. 1 (Sec. 5)
+
+
+def eq_sums_range(ref_payload, cand_payload, dtype, i0, i1):
+    """Exact S_rc, S_rr, S_cc over elements [i0, i1), as Python integers
+    scaled by 2^-EQ_BASE (value = integer * 2^EQ_BASE)."""
+    out = np.zeros(3 * EQ_DIGITS, np.int64)
+    lib().oracle_eq_sums_range(_ptr(ref_payload, _u8p), _ptr(cand_payload, _u8p),
+                               dtype, i0, i1, _ptr(out, _i64p))
+    vals = []
+    for s in range(3):
+        d = out[s * EQ_DIGITS:(s + 1) * EQ_DIGITS]
+        vals.append(sum(int(d[k]) << (32 * k) for k in range(EQ_DIGITS)))
+    return tuple(vals)
+
+
+def exact_to_double(v):
+    """The integer v * 2^EQ_BASE rounded to the nearest fp64, ties to even
+    (Python's int / int true division rounds correctly)."""
+    return v / (1 << -EQ_BASE)
+
+
+def eq_cos(s_rc, s_rr, s_cc):
+    """c_x of Eq. 1 from the rounded sums, in fp64: S_rc / (sqrt(S_rr) *
+    sqrt(S_cc)); 1 when both vectors are zero, 0 when exactly one is."""
+    import math
+    if s_rr == 0.0 and s_cc == 0.0:
+        return 1.0
+    if s_rr == 0.0 or s_cc == 0.0:
+        return 0.0
+    return s_rc / (math.sqrt(s_rr) * math.sqrt(s_cc))
+
+
+def eq_sums(ref_payload, cand_payload, dtype, n_elems, threads=1):
+    """The three sums of one float region, each exact then rounded to fp64."""
+    spans = _split(n_elems, threads)
+    parts = [None] * len(spans)
+
+    def job(k, a, b):
+        parts[k] = eq_sums_range(ref_payload, cand_payload, dtype, a, b)
+    _run_threads([lambda k=k, a=a, b=b: job(k, a, b) for k, (a, b) in enumerate(spans)])
+    tot = [sum(p[j] for p in parts) for j in range(3)]
+    return {"sum_rc": exact_to_double(tot[0]), "sum_rr": exact_to_double(tot[1]),
+            "sum_cc": exact_to_double(tot[2])}
+
+
+def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
+    """Eq. 1 for one region: c_x >= theta, ||Delta||_inf <= tau, and iota
+    (bit-exact integer and opaque buffers, intact candidate guard bands).
+    Float regions: the L-infinity term is the exact max |c - r| over finite
+    pairs and fails on any NaN/Inf-position mismatch.  Integer and opaque
+    regions have no cosine (NaN) and pass the two float terms."""
+    flt = dtype in (F32, BF16, F16, F8E4M3)
+    out = dict(sums) if flt else {"sum_rc": 0.0, "sum_rr": 0.0, "sum_cc": 0.0}
+    out["cos"] = eq_cos(out["sum_rc"], out["sum_rr"], out["sum_cc"]) if flt else float("nan")
+    flags = 0
+    if not flt or out["cos"] >= theta:
+        flags |= EQ_COS
+    if not flt or (stats["max_abs_err"] <= tau and stats["nonfinite_mismatches"] == 0):
+        flags |= EQ_LINF
+    if flt or stats["mismatches"] == 0:
+        flags |= EQ_INT
+    if stats["guard_bad_bytes"] == 0:
+        flags |= EQ_GUARD
+    out["flags"] = flags
+    out["eq"] = int(flags == EQ_COS | EQ_LINF | EQ_INT | EQ_GUARD)
+    return out

@@ -20,7 +20,7 @@ from oracle import oracle as O
 
 PIN_MODULES = ("tests.test_oracle_codecs", "tests.test_oracle_philox",
                "tests.test_oracle_fill", "tests.test_oracle_compare",
-               "tests.test_oracle_boxmuller")
+               "tests.test_oracle_eq", "tests.test_oracle_boxmuller")
 # pins that take seconds run last, in this order
 EXPENSIVE = ("test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
              "test_ln_u24_all_inputs")
@@ -95,6 +95,13 @@ MUTANTS = [
     ("int_compare_one_sided", "(size_t)sz) != 0;", "(size_t)sz) > 0;"),
     ("nonfinite_not_counted", "else { mismatch = 1; st.nonfinite_mismatches += 1; }",
      "else { mismatch = 1; }"),
+    # the exact sums of the Eq. 1 cosine
+    ("eq_cc_uses_cross_product", "eq_add(cc, c * c);", "eq_add(cc, r * c);"),
+    ("eq_rr_uses_cross_product", "eq_add(rr, r * r);", "eq_add(rr, r * c);"),
+    ("eq_top_digit_dropped", "acc[q + 2] += sg * (int64_t)hi;", ""),
+    ("eq_sign_dropped", "int64_t sg = (p < 0.0) ? -1 : 1;", "int64_t sg = 1;"),
+    ("eq_lsb_off_by_one", "int lsb = e - 53;", "int lsb = e - 52;"),
+    ("eq_mid_digit_shift", "((m >> (32 - b)) & 0xFFFFFFFFu)", "((m >> (31 - b)) & 0xFFFFFFFFu)"),
 ]
 
 
