@@ -542,8 +542,10 @@ void oracle_compare_region(const uint8_t *ref_alloc, uint32_t ref_glo,
  * region is built from three sums over its elements:
  *   S_rc = sum r*c,   S_rr = sum r*r,   S_cc = sum c*c.
  * Readings (the paper gives the formula only):
- *   R8 The sums run over the finite pairs; a pair with a NaN or an Inf on
- *      either side is judged by the NaN/Inf rule (R4) instead.
+ *   R8 Each sum takes the elements whose own term is finite: S_rc the
+ *      pairs with both values finite, S_rr the finite r, S_cc the finite c.
+ *      (Non-finite values are judged by the NaN/Inf rule R4; wherever their
+ *      positions agree, the three index sets coincide.)
  *   R9 The sums are exact, then rounded once to fp64 (nearest, ties to
  *      even): every decoded value has at most 24 significant bits, so each
  *      product is exact in fp64, and the products are added here without
@@ -597,10 +599,9 @@ void oracle_eq_sums_range(const uint8_t *ref, const uint8_t *cand, int dt,
   uint64_t since = 0;
   for (uint64_t i = i0; i < i1; ++i) {
     double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);
-    if (!isfinite(r) || !isfinite(c)) continue;
-    eq_add(rc, r * c);
-    eq_add(rr, r * r);
-    eq_add(cc, c * c);
+    if (isfinite(r) && isfinite(c)) eq_add(rc, r * c);
+    if (isfinite(r)) eq_add(rr, r * r);
+    if (isfinite(c)) eq_add(cc, c * c);
     if (++since == (1u << 20)) {     /* each digit grows by < 2^32 per add */
       eq_normalize(rc); eq_normalize(rr); eq_normalize(cc);
       since = 0;

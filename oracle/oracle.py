@@ -358,7 +358,8 @@ def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
     """Eq. 1 for one region: c_x >= theta, ||Delta||_inf <= tau, and iota
     (bit-exact integer and opaque buffers, intact candidate guard bands).
     Float regions: the L-infinity term is the exact max |c - r| over finite
-    pairs and fails on any NaN/Inf-position mismatch.  Integer and opaque
+    pairs and fails on any NaN/Inf-position mismatch.  S_rc sums over pairs
+    with both values finite, S_rr over finite r, S_cc over finite c.  Integer and opaque
     regions have no cosine (NaN) and pass the two float terms."""
     flt = dtype in (F32, BF16, F16, F8E4M3)
     out = dict(sums) if flt else {"sum_rc": 0.0, "sum_rr": 0.0, "sum_cc": 0.0}

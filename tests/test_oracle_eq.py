@@ -33,10 +33,10 @@ def _random_bits(name, n, rng):
 
 
 def _fsum_terms(r, c):
-    ok = np.isfinite(r) & np.isfinite(c)
-    r, c = r[ok], c[ok]
-    return (math.fsum((r * c).tolist()), math.fsum((r * r).tolist()),
-            math.fsum((c * c).tolist()))
+    fr, fc = np.isfinite(r), np.isfinite(c)
+    both = fr & fc
+    return (math.fsum((r[both] * c[both]).tolist()), math.fsum((r[fr] * r[fr]).tolist()),
+            math.fsum((c[fc] * c[fc]).tolist()))
 
 
 def _sums(o, ref, cand, name, n, threads=1):
@@ -145,20 +145,34 @@ def test_closed_forms(oracle):
     assert abs(oracle.eq_cos(rc, rr, cc) - 2 ** -0.5) <= 2 * 2.0 ** -53   # two roundings
 
 
-def test_nonfinite_pairs_are_left_out(oracle):
+def test_nonfinite_terms_are_left_out(oracle):
+    """Each sum drops exactly the elements whose own term is not finite."""
     rng = np.random.default_rng(14)
     r = rng.standard_normal(100).astype(np.float32)
     c = r + np.float32(1e-3)
-    base = _sums(oracle, r.view(np.uint8), c.view(np.uint8), "F32", 100)
     r2, c2 = r.copy(), c.copy()
     r2[[3, 50]] = np.nan
     c2[[7]] = np.inf
     c2[[50]] = np.nan
-    got = _sums(oracle, r2.view(np.uint8), c2.view(np.uint8), "F32", 100)
-    keep = np.ones(100, bool)
-    keep[[3, 7, 50]] = False
-    want = _sums(oracle, r[keep].view(np.uint8), c[keep].view(np.uint8), "F32", 97)
-    assert got == want and got != base
+    rc, rr, cc = _sums(oracle, r2.view(np.uint8), c2.view(np.uint8), "F32", 100)
+
+    def keep(*drop):
+        k = np.ones(100, bool)
+        k[list(drop)] = False
+        return k
+    k = keep(3, 7, 50)
+    assert rc == _sums(oracle, r[k].view(np.uint8), c[k].view(np.uint8), "F32", 97)[0]
+    k = keep(3, 50)
+    assert rr == _sums(oracle, r[k].view(np.uint8), r[k].view(np.uint8), "F32", 98)[1]
+    k = keep(7, 50)
+    assert cc == _sums(oracle, c[k].view(np.uint8), c[k].view(np.uint8), "F32", 98)[2]
+    # matching non-finite positions: all three sums are those of the finite part
+    r3, c3 = r.copy(), c.copy()
+    r3[[5, 9]] = [np.nan, -np.inf]
+    c3[[5, 9]] = [np.nan, -np.inf]
+    k = keep(5, 9)
+    assert _sums(oracle, r3.view(np.uint8), c3.view(np.uint8), "F32", 100) == \
+        _sums(oracle, r[k].view(np.uint8), c[k].view(np.uint8), "F32", 98)
 
 
 def test_order_and_split_invariance(oracle):

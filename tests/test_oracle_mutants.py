@@ -98,6 +98,8 @@ MUTANTS = [
     # the exact sums of the Eq. 1 cosine
     ("eq_cc_uses_cross_product", "eq_add(cc, c * c);", "eq_add(cc, r * c);"),
     ("eq_rr_uses_cross_product", "eq_add(rr, r * r);", "eq_add(rr, r * c);"),
+    ("eq_rr_needs_finite_pair", "if (isfinite(r)) eq_add(rr, r * r);",
+     "if (isfinite(r) && isfinite(c)) eq_add(rr, r * r);"),
     ("eq_top_digit_dropped", "acc[q + 2] += sg * (int64_t)hi;", ""),
     ("eq_sign_dropped", "int64_t sg = (p < 0.0) ? -1 : 1;", "int64_t sg = 1;"),
     ("eq_lsb_off_by_one", "int lsb = e - 53;", "int lsb = e - 52;"),
