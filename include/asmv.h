@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define ASMV_ABI_VERSION 1
+#define ASMV_ABI_VERSION 2
 
 /* A CUDA stream (the same type as cudaStream_t); NULL is the legacy
  * default stream. */
@@ -187,6 +187,56 @@ int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref,
                          const asmv_region *const *cands, size_t k, size_t n,
                          const asmv_tol *tol, asmv_stats *out_host,
                          asmv_stream_t stream);
+
+/* ---------------------------------------------------------------------
+ * Eq. 1 as a whole (Sec. 3.2): eq(K', x) = c_x >= theta AND
+ * ||K'(x) - O(x)||_inf <= tau AND iota(K', x), with c_x the cosine of the
+ * candidate and reference outputs and iota requiring bit-exact integer and
+ * opaque buffers and intact guard bands.  The paper uses theta = 0.9999 and
+ * tau = 1e-3 (Sec. 5).  Per region:
+ *   - float regions: sum_rc = sum of r*c over pairs with both values finite,
+ *     sum_rr = sum of r*r over finite r, sum_cc = sum of c*c over finite c;
+ *     each is the exact sum rounded once to the nearest double (ties to
+ *     even), so it does not depend on the grid or the order of elements.
+ *     cos = sum_rc / (sqrt(sum_rr) * sqrt(sum_cc)) in double, 1 when both
+ *     sums of squares are 0, 0 when exactly one is.  The L-infinity term is
+ *     max_abs_err of asmv_stats (exact, finite pairs) <= tau together with
+ *     no NaN/Inf-position mismatch.
+ *   - integer and opaque regions: sums 0, cos NaN; the cosine and
+ *     L-infinity terms hold, the integer term needs mismatches == 0.
+ *   - every region: the guard term needs guard_bad_bytes == 0 (the
+ *     candidate's bands; the reference's are reported, not judged).
+ * ------------------------------------------------------------------- */
+#define ASMV_EQ_COS   1u   /* c_x >= theta */
+#define ASMV_EQ_LINF  2u   /* ||Delta||_inf <= tau and no NaN/Inf-position mismatch */
+#define ASMV_EQ_INT   4u   /* integer / opaque payload bit-exact */
+#define ASMV_EQ_GUARD 8u   /* candidate guard bands intact */
+
+typedef struct {
+  double sum_rc, sum_rr, sum_cc;
+  double cos;
+  uint32_t flags;       /* the ASMV_EQ_* terms that hold */
+  uint32_t eq;          /* 1 iff all four hold */
+} asmv_eq;              /* 40 bytes */
+
+/* asmv_compare_batched plus the Eq. 1 terms: stats_host[j*n + i] as there,
+ * eq_host[j*n + i] the Eq. 1 result of candidate j on region i (k*n entries
+ * each, caller-owned).  theta is any finite double; tau a finite double
+ * >= 0.  Float regions of more than 2^31 elements are rejected (the exact
+ * sums keep per-digit counts below 2^31).  Synchronous.  Errors as
+ * asmv_compare_batched, plus EINVAL for a null eq_host, a non-finite theta
+ * or tau, a negative tau, or a float region over that size. */
+int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                    size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
+                    asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream);
+
+/* The integer sum_k digits[k] * 2^(32 k + base_exp) (k < ndigits, each
+ * digit a signed 64-bit value) rounded to the nearest double, ties to even;
+ * the conversion asmv_compare_eq applies to its exact sums.  Host only,
+ * makes no CUDA call.  EINVAL for a null pointer, ndigits outside
+ * [1, 64], or a result outside the normal double range (which the sums of
+ * asmv_compare_eq never reach). */
+int asmv_exact_to_double(const int64_t *digits, int ndigits, int base_exp, double *out);
 
 /* Host-only validation of a region table, the checks every call above
  * makes before touching the device, except the device-memory checks.

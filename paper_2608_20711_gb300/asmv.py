@@ -50,14 +50,25 @@ class Stats(ctypes.Structure):
                 ("first_guard_bad", ctypes.c_uint64), ("ref_guard_bad_bytes", ctypes.c_uint64)]
 
 
+class EqResult(ctypes.Structure):
+    """asmv_eq (40 bytes): the Eq. 1 terms of one region."""
+    _fields_ = [("sum_rc", ctypes.c_double), ("sum_rr", ctypes.c_double),
+                ("sum_cc", ctypes.c_double), ("cos", ctypes.c_double),
+                ("flags", ctypes.c_uint32), ("eq", ctypes.c_uint32)]
+
+
 STATS_FIELDS = [f for f, _ in Stats._fields_]
+EQ_FIELDS = [f for f, _ in EqResult._fields_]
+EQ_COS, EQ_LINF, EQ_INT, EQ_GUARD = 1, 2, 4, 8
+THETA, TAU = 0.9999, 1e-3          # Eq. 1 thresholds used in the paper (Sec. 5)
 assert ctypes.sizeof(Region) == 56 and ctypes.sizeof(Stats) == 64
+assert ctypes.sizeof(EqResult) == 40
 
 ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard_check",
                  "asmv_compare", "asmv_compare_batched", "asmv_check_regions",
                  "asmv_ctx_set_timing", "asmv_ctx_kernel_ms", "asmv_ctx_cuda_error",
                  "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version",
-                 "asmv_compare_noalloc")
+                 "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double")
 NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -98,6 +109,10 @@ def lib():
         L.asmv_strerror.restype = ctypes.c_char_p
         L.asmv_abi_version.argtypes = []
         L.asmv_compare_noalloc.argtypes = [RP, RP, sz, TP, SP, vp]
+        L.asmv_compare_eq.argtypes = [vp, RP, ctypes.POINTER(RP), sz, sz, TP, ctypes.c_double,
+                                      ctypes.c_double, SP, ctypes.POINTER(EqResult), vp]
+        L.asmv_exact_to_double.argtypes = [ctypes.POINTER(ctypes.c_int64), ctypes.c_int,
+                                           ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
         _lib = L
     return _lib
 
@@ -254,6 +269,37 @@ class Context:
             _stream_handle(stream)))
         flat = stats_dicts(out, k * n)
         return [flat[j * n:(j + 1) * n] for j in range(k)]
+
+    def compare_eq(self, ref: Sequence, cands: Sequence[Sequence], tol, theta: float = THETA,
+                   tau: float = TAU, stream=None):
+        """asmv_compare_eq: (stats, eq) with stats[j][i] as compare_batched
+        and eq[j][i] the Eq. 1 terms of candidate j on region i."""
+        n, k = len(ref), len(cands)
+        ra = region_array(ref)
+        cas = [region_array(c) for c in cands]
+        ptrs = (ctypes.POINTER(Region) * max(1, k))(*[ctypes.cast(c, ctypes.POINTER(Region))
+                                                      for c in cas])
+        st = (Stats * max(1, k * n))()
+        eq = (EqResult * max(1, k * n))()
+        self._check(self._lib.asmv_compare_eq(
+            self._h, ra, ptrs, k, n,
+            tol_array(tol) if not isinstance(tol, ctypes.Array) else tol,
+            float(theta), float(tau), st, eq, _stream_handle(stream)))
+        flat = stats_dicts(st, k * n)
+        eqs = [{f: getattr(eq[x], f) for f in EQ_FIELDS} for x in range(k * n)]
+        return ([flat[j * n:(j + 1) * n] for j in range(k)],
+                [eqs[j * n:(j + 1) * n] for j in range(k)])
+
+
+def exact_to_double(digits: Sequence[int], base_exp: int) -> float:
+    """asmv_exact_to_double: sum_k digits[k] 2^(32k + base_exp), rounded to
+    the nearest double (host only)."""
+    arr = (ctypes.c_int64 * max(1, len(digits)))(*[int(d) for d in digits])
+    out = ctypes.c_double()
+    rc = lib().asmv_exact_to_double(arr, len(digits), int(base_exp), ctypes.byref(out))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return out.value
 
 
 def compare_noalloc(ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:

@@ -24,6 +24,7 @@ using namespace asmv;
 
 static_assert(sizeof(asmv_region) == 56, "asmv_region layout");
 static_assert(sizeof(asmv_stats) == 64, "asmv_stats layout");
+static_assert(sizeof(asmv_eq) == 40, "asmv_eq layout");
 static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
 static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
               "plan layouts");
@@ -197,6 +198,7 @@ struct asmv_ctx {
   int device = 0;
   int sms = 0;
   int fill_ctas = 1;
+  int eq_ctas = 1;
   void *dws = nullptr;
   size_t dws_cap = 0;
   unsigned char *hst = nullptr;
@@ -255,9 +257,12 @@ int check_device_table(asmv_ctx *ctx, const asmv_region *regs, size_t n,
 }
 
 // Upload `img` (and reserve `readback` bytes of staging after it) to the
-// workspace on `s`; returns the device base in *dev.
-int stage(asmv_ctx *ctx, const Image &img, size_t readback, cudaStream_t s, unsigned char **dev) {
-  const size_t need_dev = std::max<size_t>(img.bytes.size(), 256);
+// workspace on `s`; returns the device base in *dev.  `dev_extra` more
+// bytes of workspace follow the image (at its size rounded up to 256),
+// uninitialised.
+int stage(asmv_ctx *ctx, const Image &img, size_t readback, cudaStream_t s, unsigned char **dev,
+          size_t dev_extra = 0) {
+  const size_t need_dev = std::max<size_t>(((img.bytes.size() + 255) & ~(size_t)255) + dev_extra, 256);
   const size_t need_host = ((img.bytes.size() + 255) & ~(size_t)255) + readback;
   cudaError_t e;
   if (ctx->staged_pending) {
@@ -341,6 +346,63 @@ int readback(asmv_ctx *ctx, size_t stats_off, size_t img_bytes, size_t count, cu
   return ASMV_OK;
 }
 
+// The integer sum_k d[k] 2^(32k + base) rounded to the nearest double (ties
+// to even).  The digits are first carried into nd + 2 limbs of 32 bits in
+// two's complement; the magnitude's leading 64 bits and a sticky bit then
+// decide the rounding.
+int exact_to_double_impl(const int64_t *d, int nd, int base, double *out) {
+  if (d == nullptr || out == nullptr || nd < 1 || nd > 64) return ASMV_EINVAL;
+  const int nl = nd + 2;
+  uint32_t L[66];
+  __int128 c = 0;
+  for (int k = 0; k < nl; ++k) {
+    const __int128 x = c + (k < nd ? (__int128)d[k] : (__int128)0);
+    L[k] = (uint32_t)(x & 0xFFFFFFFF);
+    c = x >> 32;                                   // floor: arithmetic shift
+  }
+  const bool neg = c < 0;                          // c is 0 or -1 here
+  if (neg) {
+    uint64_t carry = 1;
+    for (int k = 0; k < nl; ++k) {
+      const uint64_t x = (uint64_t)(uint32_t)~L[k] + carry;
+      L[k] = (uint32_t)x;
+      carry = x >> 32;
+    }
+  }
+  int top = nl - 1;
+  while (top >= 0 && L[top] == 0) --top;
+  if (top < 0) { *out = 0.0; return ASMV_OK; }
+  int msb = 32 * top;
+  for (uint32_t v = L[top]; v > 1; v >>= 1) ++msb;
+  auto bit = [&](int pos) -> uint64_t {
+    return pos < 0 ? 0u : (uint64_t)((L[pos >> 5] >> (pos & 31)) & 1u);
+  };
+  uint64_t m = 0;
+  for (int b = 0; b < 64; ++b) m = (m << 1) | bit(msb - b);
+  bool sticky = false;
+  const int below = msb - 64;                      // highest bit not in m
+  if (below >= 0) {
+    const int lim = below >> 5;
+    const uint32_t mask = (below & 31) == 31 ? 0xFFFFFFFFu : ((1u << ((below & 31) + 1)) - 1u);
+    sticky = (L[lim] & mask) != 0;
+    for (int k = 0; k < lim && !sticky; ++k) sticky = L[k] != 0;
+  }
+  uint64_t keep = m >> 11;                         // 53 bits
+  const uint64_t rem = m & 0x7FFu, half = 0x400u;
+  if (rem > half || (rem == half && (sticky || (keep & 1u)))) keep += 1;
+  const int e = msb - 52 + base;                   // weight of keep's last bit
+  if (e + 52 < -1022 || e + 53 > 1024) return ASMV_EINVAL;
+  const double v = std::ldexp((double)keep, e);
+  *out = neg ? -v : v;
+  return ASMV_OK;
+}
+
+double eq_cosine(double rc, double rr, double cc) {
+  if (rr == 0.0 && cc == 0.0) return 1.0;
+  if (rr == 0.0 || cc == 0.0) return 0.0;
+  return rc / (std::sqrt(rr) * std::sqrt(cc));
+}
+
 }  // namespace
 
 // ====================================================================== ABI
@@ -385,6 +447,7 @@ int asmv_ctx_create(asmv_ctx **out, int device) {
     return ASMV_ECUDA;
   }
   ctx->fill_ctas = fill_max_ctas_per_sm();
+  ctx->eq_ctas = eq_max_ctas_per_sm();
   void *fn = nullptr;
   cudaDriverEntryPointQueryResult q;
   if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &fn, 12000, cudaEnableDefault, &q) ==
@@ -644,6 +707,139 @@ int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref, const asmv_regio
   DeviceScope ds(ctx->device);
   if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
   return run_compare(ctx, ref, cands, k, n, tol, out_host, (cudaStream_t)stream, false);
+}
+
+// The exact Eq. 1 sums of k candidates: fills digits[n][1 + 2k][kEqDigits].
+static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                  size_t k, size_t n, cudaStream_t s, std::vector<long long> &digits) {
+  const size_t nslots = 1 + 2 * k;
+  digits.assign(n * nslots * kEqDigits, 0);
+  std::vector<CmpRegion> cr(n + 1);
+  std::vector<uint64_t> caddr(k * n);
+  uint64_t tile = 0;
+  for (size_t i = 0; i < n; ++i) {
+    const asmv_region &r = ref[i];
+    uint64_t pb, tot;
+    region_extent(r, &pb, &tot);
+    CmpRegion &c = cr[i];
+    std::memset(&c, 0, sizeof c);
+    c.ref = r.alloc + r.guard_lo;
+    c.bytes = is_float(r.dtype) ? pb : 0;
+    c.tile0 = tile;
+    c.dtype = r.dtype;
+    bool vec = (c.ref % 16) == 0;
+    for (size_t j = 0; j < k; ++j) {
+      const uint64_t a = cands[j][i].alloc + cands[j][i].guard_lo;
+      caddr[j * n + i] = a;
+      vec = vec && (a % 16) == 0;
+    }
+    c.vec = vec;
+    tile += tiles_of(c.bytes);
+  }
+  std::memset(&cr[n], 0, sizeof(CmpRegion));
+  cr[n].tile0 = tile;
+  if (tile == 0) return ASMV_OK;                    // no float payload: all sums are zero
+  const size_t dig_bytes = digits.size() * sizeof(long long);
+
+  Image img;
+  const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CmpRegion));
+  const size_t o_cand = img.add(caddr.data(), caddr.size() * sizeof(uint64_t));
+  const size_t o_dig = (img.bytes.size() + 255) & ~(size_t)255;
+  unsigned char *dev = nullptr;
+  int rc;
+  if ((rc = stage(ctx, img, dig_bytes, s, &dev, dig_bytes)) != ASMV_OK) return rc;
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(dev + o_dig, 0, dig_bytes, s)) != cudaSuccess) return fail_cuda(ctx, e);
+
+  EqParams p;
+  std::memset(&p, 0, sizeof p);
+  p.regions = (const CmpRegion *)(dev + o_regs);
+  p.digits = (long long *)(dev + o_dig);
+  p.ntiles = tile;
+  p.nregions = (uint32_t)n;
+  p.nslots = (uint32_t)nslots;
+  const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tile, (uint64_t)ctx->sms * ctx->eq_ctas));
+  if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  for (size_t g = 0; g * kMaxCands < k; ++g) {
+    p.K = (uint32_t)std::min<size_t>(kMaxCands, k - g * kMaxCands);
+    p.j0 = (uint32_t)(g * kMaxCands);
+    p.do_rr = g == 0;
+    p.cands = (const uint64_t *)(dev + o_cand) + g * kMaxCands * n;
+    if ((e = (cudaError_t)launch_eq(p, grid, s)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->launches += 1;
+  }
+  if (ctx->timing) {
+    if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->timed = true;
+  }
+  if ((rc = after_launch(ctx, s)) != ASMV_OK) return rc;
+  unsigned char *host = ctx->hst + ((img.bytes.size() + 255) & ~(size_t)255);
+  if ((e = cudaMemcpyAsync(host, dev + o_dig, dig_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+    return fail_cuda(ctx, e);
+  if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return fail_cuda(ctx, e);
+  ctx->staged_pending = false;
+  ctx->ws_pending = false;
+  std::memcpy(digits.data(), host, dig_bytes);
+  return ASMV_OK;
+}
+
+int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                    size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
+                    asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream) {
+  if (ctx == nullptr || k == 0 || cands == nullptr || !tol_ok(tol) ||
+      (n > 0 && (stats_host == nullptr || eq_host == nullptr)))
+    return ASMV_EINVAL;
+  if (!std::isfinite(theta) || !std::isfinite(tau) || tau < 0.0) return ASMV_EINVAL;
+  if (k > (size_t)0x7FFFFFFF / (n ? n : 1)) return ASMV_EINVAL;
+  int rc = check_pairs(ref, cands, k, n);
+  if (rc != ASMV_OK) return rc;
+  for (size_t i = 0; i < n; ++i)
+    if (is_float(ref[i].dtype) && ref[i].n_elems > ((uint64_t)1 << 31)) return ASMV_EINVAL;
+  if (n == 0) return ASMV_OK;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  const cudaStream_t s = (cudaStream_t)stream;
+  std::vector<asmv_stats> stats(k * n);
+  if ((rc = run_compare(ctx, ref, cands, k, n, tol, stats.data(), s, false)) != ASMV_OK) return rc;
+  std::vector<long long> digits;
+  if ((rc = run_eq(ctx, ref, cands, k, n, s, digits)) != ASMV_OK) return rc;
+  std::vector<asmv_eq> res(k * n);
+  const size_t nslots = 1 + 2 * k;
+  for (size_t j = 0; j < k; ++j) {
+    for (size_t i = 0; i < n; ++i) {
+      const asmv_stats &st = stats[j * n + i];
+      asmv_eq &q = res[j * n + i];
+      std::memset(&q, 0, sizeof q);
+      const bool flt = is_float(ref[i].dtype);
+      if (flt) {
+        const long long *d = digits.data() + i * nslots * kEqDigits;
+        const int base = eq_digit_base(ref[i].dtype);
+        if (exact_to_double_impl((const int64_t *)(d + (1 + 2 * j) * kEqDigits), kEqDigits, base,
+                                 &q.sum_rc) != ASMV_OK ||
+            exact_to_double_impl((const int64_t *)d, kEqDigits, base, &q.sum_rr) != ASMV_OK ||
+            exact_to_double_impl((const int64_t *)(d + (2 + 2 * j) * kEqDigits), kEqDigits, base,
+                                 &q.sum_cc) != ASMV_OK)
+          return ASMV_ECUDA;                         // digits out of range: a device fault
+        q.cos = eq_cosine(q.sum_rc, q.sum_rr, q.sum_cc);
+      } else {
+        q.cos = NAN;
+      }
+      uint32_t f = 0;
+      if (!flt || q.cos >= theta) f |= ASMV_EQ_COS;
+      if (!flt || (st.max_abs_err <= tau && st.nonfinite_mismatches == 0)) f |= ASMV_EQ_LINF;
+      if (flt || st.mismatches == 0) f |= ASMV_EQ_INT;
+      if (st.guard_bad_bytes == 0) f |= ASMV_EQ_GUARD;
+      q.flags = f;
+      q.eq = f == (ASMV_EQ_COS | ASMV_EQ_LINF | ASMV_EQ_INT | ASMV_EQ_GUARD);
+    }
+  }
+  std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
+  std::memcpy(eq_host, res.data(), res.size() * sizeof(asmv_eq));
+  return ASMV_OK;
+}
+
+int asmv_exact_to_double(const int64_t *digits, int ndigits, int base_exp, double *out) {
+  return exact_to_double_impl(digits, ndigits, base_exp, out);
 }
 
 }  // extern "C"

@@ -1,0 +1,301 @@
+// eqsum.cu -- the three sums behind the cosine of Eq. 1 (AsmEvo Sec. 3.2):
+//   S_rc = sum r*c over pairs with both values finite,
+//   S_rr = sum r*r over finite r,   S_cc = sum c*c over finite c,
+// for every float region of a reference and K candidates, added exactly.
+//
+// Exactness.  A decoded element is +-m 2^e with an integer significand m
+// (< 2^24 fp32, 2^8 bf16, 2^11 fp16, 2^4 fp8) and e the weight of its last
+// bit; a product is +-P 2^s with P = m_r m_c and s = e_r + e_c.  Each thread
+// adds its products at a fixed binary point 2^L into NACC signed 64-bit
+// accumulators 32 bits apart (accumulator q weighs 2^(L + 32q)):
+//   P 2^s = (P << (t & 31)) 2^(L + 32 (t >> 5)),  t = s - L,
+// (fp32 products are split into two 24-bit pieces first).  Integer additions
+// are exact and commute, so the sums do not depend on the order of the
+// elements or on the grid.  A product outside the window [L, L + 32 NACC)
+// goes straight to the region's global digits with 64-bit atomics: fp16 and
+// fp8 products always fit; bf16 and fp32 ones do for values between about
+// 2^-24 and 2^24.
+//
+// Reduction.  Every tile, each warp carries its lanes' accumulators into
+// 32-bit digits, sums them over the warp with shuffles and adds them to the
+// CTA's shared digits; the CTA adds those to the region's global digits when
+// it leaves the region.  Global digit k of a sum weighs 2^(32k + base), base
+// = eq_digit_base(dtype); the host rounds the digits to fp64.
+//
+// Work split: like the compare, a persistent grid over 16 KiB tiles of the
+// reference payloads.  Within a tile, warp w takes a contiguous run of at
+// most 128 chunks of 16 bytes (four per lane).  The K candidates are read
+// one after another; the reference tile is re-read through L1 for each, so
+// it comes from memory once per tile.
+#include <cuda_runtime.h>
+#include "device.cuh"
+#include "plan.h"
+
+namespace asmv {
+namespace {
+
+constexpr int kWin = 5;                 // shared digits per sum: NACC + 1 <= 5
+constexpr int kMaxRounds = 4;           // chunks per lane per tile (16 KiB / 8 warps / 32 lanes / 16 B)
+static_assert(kTileBytes == (uint64_t)kMaxRounds * 16 * 32 * kWarps, "eq tile split");
+
+template <int DT> struct Fmt;
+// kL: binary point of the window; kDig: index of the global digit at 2^kL
+template <> struct Fmt<kF32>  { static constexpr int kBytes = 4, kNacc = 4, kL = -94, kDig = 7; };
+template <> struct Fmt<kBF16> { static constexpr int kBytes = 2, kNacc = 3, kL = -62, kDig = 7; };
+template <> struct Fmt<kF16>  { static constexpr int kBytes = 2, kNacc = 2, kL = -48, kDig = 2; };
+template <> struct Fmt<kF8>   { static constexpr int kBytes = 1, kNacc = 1, kL = -18, kDig = 2; };
+
+static_assert(Fmt<kF32>::kL - 32 * Fmt<kF32>::kDig == eq_digit_base(kF32), "fp32 digits");
+static_assert(Fmt<kBF16>::kL - 32 * Fmt<kBF16>::kDig == eq_digit_base(kBF16), "bf16 digits");
+static_assert(Fmt<kF16>::kL - 32 * Fmt<kF16>::kDig == eq_digit_base(kF16), "fp16 digits");
+static_assert(Fmt<kF8>::kL - 32 * Fmt<kF8>::kDig == eq_digit_base(kF8), "fp8 digits");
+
+struct Elem {
+  uint32_t m;      // significand (integer)
+  int e;           // weight of its last bit: |x| = m 2^e
+  bool neg, fin;
+};
+
+// Element k of a 16-byte chunk.
+template <int DT>
+__device__ __forceinline__ Elem decode(const uint4 &v, int k) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  Elem x;
+  if (DT == kF32) {
+    const uint32_t b = w[k];
+    const uint32_t E = (b >> 23) & 255u, f = b & 0x7FFFFFu;
+    x.fin = E != 255u;
+    x.m = E ? (f | 0x800000u) : f;
+    x.e = (int)max(E, 1u) - 150;
+    x.neg = (b >> 31) != 0;
+  } else if (DT == kBF16 || DT == kF16) {
+    const uint32_t b = (w[k >> 1] >> (16 * (k & 1))) & 0xFFFFu;
+    if (DT == kBF16) {
+      const uint32_t E = (b >> 7) & 255u, f = b & 127u;
+      x.fin = E != 255u;
+      x.m = E ? (f | 128u) : f;
+      x.e = (int)max(E, 1u) - 134;
+    } else {
+      const uint32_t E = (b >> 10) & 31u, f = b & 1023u;
+      x.fin = E != 31u;
+      x.m = E ? (f | 1024u) : f;
+      x.e = (int)max(E, 1u) - 25;
+    }
+    x.neg = (b >> 15) != 0;
+  } else {
+    const uint32_t b = (w[k >> 2] >> (8 * (k & 3))) & 0xFFu;
+    const uint32_t E = (b >> 3) & 15u, f = b & 7u;
+    x.fin = (b & 0x7Fu) != 0x7Fu;
+    x.m = E ? (f | 8u) : f;
+    x.e = (int)max(E, 1u) - 10;
+    x.neg = (b >> 7) != 0;
+  }
+  return x;
+}
+
+// One product outside the window: three digit atomics.  pos = s - base >= 0.
+__device__ __noinline__ void rare_add(long long *dig, unsigned long long P, int pos, bool neg) {
+  const int q = pos >> 5, b = pos & 31;
+  const unsigned long long lo = P << b;
+  const unsigned long long hi = b ? (P >> (64 - b)) : 0ull;
+  const unsigned long long d[3] = {lo & 0xFFFFFFFFull, lo >> 32, hi};
+#pragma unroll
+  for (int k = 0; k < 3; ++k)
+    if (d[k]) atomicAdd(reinterpret_cast<unsigned long long *>(dig + q + k),
+                        neg ? (unsigned long long)(-(long long)d[k]) : d[k]);
+}
+
+template <int N>
+__device__ __forceinline__ void add_piece(long long (&a)[N], int t, unsigned long long piece, bool neg) {
+  long long v = (long long)(piece << (t & 31));
+  v = neg ? -v : v;
+  const int q = t >> 5;
+#pragma unroll
+  for (int k = 0; k < N; ++k)
+    if (q == k) a[k] += v;
+}
+
+// acc += x*y (exact); `dig` is the sum's global digits (for the rare path).
+template <int DT>
+__device__ __forceinline__ void add_product(long long (&a)[Fmt<DT>::kNacc], const Elem &x,
+                                            const Elem &y, long long *dig) {
+  using F = Fmt<DT>;
+  const unsigned long long P = (unsigned long long)x.m * y.m;
+  if (P == 0ull) return;
+  const int t = x.e + y.e - F::kL;
+  const bool neg = x.neg != y.neg;
+  if (DT == kF32) {
+    if ((unsigned)t < (unsigned)(32 * F::kNacc - 24)) {
+      add_piece(a, t, P & 0xFFFFFFull, neg);
+      add_piece(a, t + 24, P >> 24, neg);
+    } else {
+      rare_add(dig, P, t + 32 * F::kDig, neg);
+    }
+  } else {
+    if ((unsigned)t < (unsigned)(32 * F::kNacc)) add_piece(a, t, P, neg);
+    else rare_add(dig, P, t + 32 * F::kDig, neg);
+  }
+}
+
+// Carry the lane's accumulators into N+1 digits, sum them over the warp and
+// add them to the CTA's shared digits of one sum.  All 32 lanes call this.
+template <int N>
+__device__ __forceinline__ void warp_flush(long long (&a)[N], long long *sdig) {
+  long long d[N + 1];
+  long long carry = 0;
+#pragma unroll
+  for (int k = 0; k < N; ++k) {
+    const long long x = a[k] + carry;          // |a| < 2^62, |carry| < 2^31
+    d[k] = x & 0xFFFFFFFFll;
+    carry = x >> 32;
+    a[k] = 0;
+  }
+  d[N] = carry;
+#pragma unroll
+  for (int k = 0; k <= N; ++k) {
+    long long v = d[k];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    if ((threadIdx.x & 31) == 0 && v != 0)
+      atomicAdd(reinterpret_cast<unsigned long long *>(sdig + k), (unsigned long long)v);
+  }
+}
+
+__device__ __forceinline__ long long *global_digits(const EqParams &p, uint32_t region, uint32_t slot) {
+  return p.digits + ((size_t)region * p.nslots + slot) * kEqDigits;
+}
+
+// Global slot of local slot `ls` (0 = S_rr, 1 + 2j = S_rc of candidate j,
+// 2 + 2j = S_cc of candidate j).
+__device__ __forceinline__ uint32_t global_slot(const EqParams &p, uint32_t ls) {
+  return ls == 0 ? 0u : ls + 2u * p.j0;
+}
+
+__device__ __forceinline__ uint4 load_chunk(uint64_t addr, uint32_t bytes, bool vec, bool cached) {
+  if (!vec || bytes != 16u) return load_bytes(addr, bytes);
+  return cached ? __ldg(reinterpret_cast<const uint4 *>(addr)) : ldg16(addr);
+}
+
+template <int DT>
+__device__ __noinline__ void eq_tile(const EqParams &p, const CmpRegion &R, uint32_t region,
+                                     uint64_t a, uint32_t nb, long long *sdig) {
+  using F = Fmt<DT>;
+  constexpr int kPer = 16 / F::kBytes;
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t nchunks = (nb + 15u) >> 4;
+  const uint32_t per_warp = (nchunks + kWarps - 1) / kWarps;
+  const uint32_t c0 = warp * per_warp;
+  const uint32_t c1 = min(c0 + per_warp, nchunks);
+  const uint32_t rounds = (per_warp + 31u) >> 5;     // the same for every warp
+  if (p.do_rr) {
+    long long acc[F::kNacc];
+#pragma unroll
+    for (int k = 0; k < F::kNacc; ++k) acc[k] = 0;
+    long long *dig = global_digits(p, region, 0);
+#pragma unroll 1
+    for (uint32_t r = 0; r < rounds; ++r) {
+      const uint32_t c = c0 + 32u * r + lane;
+      uint4 rv = make_uint4(0u, 0u, 0u, 0u);
+      if (c < c1) rv = load_chunk(R.ref + a + 16ull * c, min(16u, nb - 16u * c), R.vec, true);
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        const Elem x = decode<DT>(rv, k);
+        if (x.fin) add_product<DT>(acc, x, x, dig);
+      }
+    }
+    warp_flush(acc, sdig);
+  }
+  for (uint32_t j = 0; j < p.K; ++j) {
+    const uint64_t cbase = p.cands[(size_t)j * p.nregions + region] + a;
+    long long rc[F::kNacc], cc[F::kNacc];
+#pragma unroll
+    for (int k = 0; k < F::kNacc; ++k) { rc[k] = 0; cc[k] = 0; }
+    long long *dig_rc = global_digits(p, region, global_slot(p, 1 + 2 * j));
+    long long *dig_cc = global_digits(p, region, global_slot(p, 2 + 2 * j));
+#pragma unroll 1
+    for (uint32_t r = 0; r < rounds; ++r) {
+      const uint32_t c = c0 + 32u * r + lane;
+      uint4 rv = make_uint4(0u, 0u, 0u, 0u), cv = rv;
+      if (c < c1) {
+        const uint32_t bytes = min(16u, nb - 16u * c);
+        rv = load_chunk(R.ref + a + 16ull * c, bytes, R.vec, true);   // L1 hit after j = 0
+        cv = load_chunk(cbase + 16ull * c, bytes, R.vec, false);
+      }
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        const Elem x = decode<DT>(rv, k);
+        const Elem y = decode<DT>(cv, k);
+        if (y.fin) {
+          add_product<DT>(cc, y, y, dig_cc);
+          if (x.fin) add_product<DT>(rc, x, y, dig_rc);
+        }
+      }
+    }
+    warp_flush(rc, sdig + (1 + 2 * j) * kWin);
+    warp_flush(cc, sdig + (2 + 2 * j) * kWin);
+  }
+}
+
+// Add the CTA's shared digits of `region` to its global digits; zero them.
+__device__ void cta_flush(const EqParams &p, uint32_t region, uint32_t dtype, long long *sdig) {
+  __syncthreads();
+  const int dig0 = dtype == kF32 ? Fmt<kF32>::kDig : dtype == kBF16 ? Fmt<kBF16>::kDig
+                 : dtype == kF16 ? Fmt<kF16>::kDig : Fmt<kF8>::kDig;
+  const uint32_t nloc = 1u + 2u * p.K;
+  for (uint32_t x = threadIdx.x; x < nloc * kWin; x += blockDim.x) {
+    const long long v = sdig[x];
+    if (v != 0) {
+      const uint32_t ls = x / kWin, k = x % kWin;
+      atomicAdd(reinterpret_cast<unsigned long long *>(global_digits(p, region, global_slot(p, ls)) +
+                                                       dig0 + k),
+                (unsigned long long)v);
+      sdig[x] = 0;
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kThreads) eq_kernel(EqParams p) {
+  __shared__ long long sdig[(1 + 2 * kMaxCands) * kWin];
+  for (uint32_t x = threadIdx.x; x < (1 + 2 * kMaxCands) * kWin; x += blockDim.x) sdig[x] = 0;
+  __syncthreads();
+  const uint64_t t0 = p.ntiles * blockIdx.x / gridDim.x;
+  const uint64_t t1 = p.ntiles * (blockIdx.x + 1) / gridDim.x;
+  uint32_t cur = 0xFFFFFFFFu, cur_dtype = 0;
+  for (uint64_t t = t0; t < t1; ++t) {
+    const uint32_t i = find_region(p.regions, p.nregions, t);
+    const CmpRegion R = p.regions[i];
+    if (i != cur) {
+      if (cur != 0xFFFFFFFFu) cta_flush(p, cur, cur_dtype, sdig);
+      cur = i;
+      cur_dtype = R.dtype;
+    }
+    const uint64_t a = (t - R.tile0) * kTileBytes;
+    const uint32_t nb = (uint32_t)umin64(kTileBytes, R.bytes - a);
+    switch (R.dtype) {
+      case kF32: eq_tile<kF32>(p, R, i, a, nb, sdig); break;
+      case kBF16: eq_tile<kBF16>(p, R, i, a, nb, sdig); break;
+      case kF16: eq_tile<kF16>(p, R, i, a, nb, sdig); break;
+      default: eq_tile<kF8>(p, R, i, a, nb, sdig); break;
+    }
+  }
+  if (cur != 0xFFFFFFFFu) cta_flush(p, cur, cur_dtype, sdig);
+}
+
+}  // namespace
+
+int eq_max_ctas_per_sm() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, eq_kernel, kThreads, 0) != cudaSuccess) {
+    cudaGetLastError();
+    return 1;
+  }
+  return n > 0 ? n : 1;
+}
+
+int launch_eq(const EqParams &p, int grid, void *stream) {
+  eq_kernel<<<grid, kThreads, 0, (cudaStream_t)stream>>>(p);
+  return (int)cudaGetLastError();
+}
+
+}  // namespace asmv

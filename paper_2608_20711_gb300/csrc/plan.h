@@ -110,11 +110,34 @@ struct CmpParams {
   TolF tol[7];
 };
 
-// Launchers (defined in fill.cu / compare.cu).  Return a cudaError_t.
+// The Eq. 1 sums (eqsum.cu).  Each sum of a region is kept as kEqDigits
+// signed 64-bit digits, digit k weighing 2^(32k + eq_digit_base(dtype)); the
+// digits of one region are [slot][kEqDigits] with slot 0 = S_rr and slots
+// 1 + 2j, 2 + 2j = S_rc, S_cc of candidate j.
+constexpr int kEqDigits = 20;
+constexpr int eq_digit_base(uint32_t dtype) {
+  return dtype == kF32 ? -318 : dtype == kBF16 ? -286 : dtype == kF16 ? -112 : -82;
+}
+
+struct EqParams {
+  const CmpRegion *regions;    // nregions + 1 entries (sentinel); bytes = 0 for non-float
+  const uint64_t *cands;       // [K][nregions] candidate payload addresses (this launch)
+  long long *digits;           // [nregions][nslots][kEqDigits]
+  uint64_t ntiles;             // tiles of kTileBytes
+  uint32_t nregions;
+  uint32_t K;                  // candidates in this launch (<= kMaxCands)
+  uint32_t j0;                 // index of this launch's first candidate
+  uint32_t nslots;             // 1 + 2 * (all candidates)
+  uint32_t do_rr;              // this launch also adds S_rr
+};
+
+// Launchers (defined in fill.cu / compare.cu / eqsum.cu).  Return a cudaError_t.
 int launch_fill(const FillParams &p, int grid, void *stream);
 int launch_compare(const CmpParams &p, int grid, void *stream);
 int fill_max_ctas_per_sm();
 uint32_t compare_tile_bytes(uint32_t K);
 size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes);
+int launch_eq(const EqParams &p, int grid, void *stream);
+int eq_max_ctas_per_sm();
 
 }  // namespace asmv

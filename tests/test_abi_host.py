@@ -1,0 +1,132 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads and
+exports every function include/asmv.h declares, the ctypes layouts match
+the header's, the host-only calls behave as documented (table validation,
+status strings, the exact-sum rounding of Eq. 1), and with no GPU a
+context cannot be created: nothing falls back to the CPU."""
+import ctypes
+import os
+import random
+import re
+from fractions import Fraction
+
+import pytest
+
+from paper_2608_20711_gb300 import asmv
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "asmv.h")
+
+
+def _lib():
+    if not os.path.exists(asmv.LIB_PATH):
+        from paper_2608_20711_gb300 import build
+        build.build()
+    return asmv.lib()
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return set(re.findall(r"\b(asmv_\w+)\s*\(", text)) - {"asmv_ctx"}
+
+
+def test_every_declared_function_is_exported():
+    L = _lib()
+    declared = _declared_functions()
+    assert declared == set(asmv.ABI_FUNCTIONS)
+    for name in declared:
+        assert hasattr(L, name), name
+
+
+def test_layouts_and_version():
+    text = open(HEADER).read()
+    assert ctypes.sizeof(asmv.Region) == 56
+    assert ctypes.sizeof(asmv.Stats) == 64
+    assert ctypes.sizeof(asmv.EqResult) == 40
+    ver = int(re.search(r"#define ASMV_ABI_VERSION (\d+)", text).group(1))
+    assert _lib().asmv_abi_version() == ver
+    for name, code in (("ASMV_EQ_COS", asmv.EQ_COS), ("ASMV_EQ_LINF", asmv.EQ_LINF),
+                       ("ASMV_EQ_INT", asmv.EQ_INT), ("ASMV_EQ_GUARD", asmv.EQ_GUARD)):
+        assert int(re.search(r"#define %s +(\d+)u" % name, text).group(1)) == code
+
+
+def test_status_strings():
+    _lib()
+    for st in (asmv.OK, asmv.EINVAL, asmv.ECUDA, asmv.ETIMEOUT, asmv.ENOMEM):
+        assert asmv.strerror(st)
+    assert asmv.strerror(asmv.OK) != asmv.strerror(asmv.EINVAL)
+
+
+def test_region_table_validation():
+    _lib()
+    ok = dict(alloc=1 << 20, n_elems=100, dtype="f32", dist="uniform", p0=-1.0, p1=1.0,
+              guard_lo=64, guard_hi=64)
+    assert asmv.check_regions([ok], for_fill=True) == asmv.OK
+    bad = [dict(ok, dtype=9), dict(ok, dist=7), dict(ok, dist="int_range", p0=0, p1=5),
+           dict(ok, p0=2.0, p1=1.0), dict(ok, n_elems=1 << 62), dict(ok, alloc=0)]
+    for b in bad:
+        assert asmv.check_regions([b], for_fill=True) == asmv.EINVAL, b
+    # overlap is a fill error, not a compare error
+    two = [ok, dict(ok, alloc=ok["alloc"] + 100)]
+    assert asmv.check_regions(two, for_fill=True) == asmv.EINVAL
+    assert asmv.check_regions(two, for_fill=False) == asmv.OK
+    assert asmv.check_regions([], for_fill=True) == asmv.OK
+
+
+def _exact(digits, base):
+    v = sum(int(d) << (32 * k) for k, d in enumerate(digits))
+    return float(Fraction(v) * Fraction(2) ** base) if base >= 0 else v / (1 << -base)
+
+
+def _digits_of(v, nd, rng):
+    """A (non-normalised) digit vector of the integer v."""
+    d = []
+    for k in range(nd - 1):
+        lo = v & 0xFFFFFFFF
+        if rng.random() < 0.5 and k < nd - 2:          # move a random multiple up a digit
+            extra = rng.randrange(-(1 << 20), 1 << 20)
+            lo += extra << 32
+        d.append(lo)
+        v = (v - lo) >> 32
+    d.append(v)
+    assert all(-(1 << 63) <= x < (1 << 63) for x in d)
+    return d
+
+
+def test_exact_to_double_random_and_ties():
+    _lib()
+    rng = random.Random(5)
+    nd, base = 20, -318
+    cases = [0, 1, -1, 1 << 300, -(1 << 300) + 1]
+    for _ in range(400):
+        bits = rng.randrange(1, 600)
+        cases.append(rng.choice([-1, 1]) * rng.getrandbits(bits))
+    # exact ties: (2^53 + odd/even) * 2^s + half, with and without sticky bits
+    for s in (0, 7, 100, 400):
+        for m in ((1 << 53) + 1, (1 << 53) + 2, (1 << 54) - 1):
+            half = 1 << s
+            for extra in (0, 1):
+                v = (m << (s + 1)) + half + (extra if s > 0 else 0)
+                cases += [v, -v]
+    for v in cases:
+        d = _digits_of(v, nd, rng)
+        assert asmv.exact_to_double(d, base) == _exact(d, base), v
+
+
+def test_exact_to_double_rejects_bad_arguments():
+    _lib()
+    with pytest.raises(asmv.AsmvError):
+        asmv.exact_to_double([], -318)
+    with pytest.raises(asmv.AsmvError):
+        asmv.exact_to_double([1] * 65, 0)
+    with pytest.raises(asmv.AsmvError):
+        asmv.exact_to_double([1], 1200)        # beyond the double range
+
+
+def test_no_gpu_means_no_context():
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    _lib()
+    with pytest.raises(asmv.AsmvError):
+        asmv.Context(0)
