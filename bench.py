@@ -8,7 +8,11 @@ GEMM input buffers, then one fp16 [32768, 32768] reference checked against
 8 candidates carrying 0..8 ULP of noise.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
-                       [--workload NAME] [--no-e2e] [--no-cpu]
+                       [--workload NAME] [--no-e2e] [--no-cpu] [--no-eq]
+
+Beside the step, the line carries `eq1`: Eq. 1 as a whole (the exact sums
+of the cosine term over the same reference and candidates), its kernel
+timed alone with CUDA events.
 For N > 1 launch under torchrun; every rank runs its own replica (weak
 scaling, no data-path collective) and rank 0 prints one JSON line.
 """
@@ -108,15 +112,21 @@ def kernel_traffic(kernel, workload):
     txt = open(path).read()
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
     h = re.search(r"source_sha256:\s*([0-9a-f]+)", txt)
-    if not m or not h or h.group(1) != source_hash():
+    if not m or not h or h.group(1) != source_hash(kernel):
         return None, path
     return float(m.group(1)), path
 
 
-def source_hash():
+# the source files each kernel is compiled from
+KERNEL_SOURCES = {"fill": ("fill.cu", "device.cuh", "ln_table.h", "plan.h"),
+                  "compare": ("compare.cu", "device.cuh", "plan.h"),
+                  "eqsum": ("eqsum.cu", "device.cuh", "plan.h")}
+
+
+def source_hash(kernel):
     d = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_20711_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(csrc, f), "rb") as fh:
             d.update(f.encode() + fh.read())
     return d.hexdigest()[:16]
@@ -415,6 +425,8 @@ def run_mine(args):
         "clocks": clk.summary(), "gpu_launches": launches, "roofline": roofline,
         "e2e": e2e,
     }
+    if args.eq:
+        line["eq1"] = run_eq1(setup, args, peak)
     if rank == 0 and world == 1 and args.cpu:
         line["cpu_baseline"] = cpu_oracle_sample(setup)
     if rank == 0:
@@ -424,6 +436,34 @@ def run_mine(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_eq1(setup, args, peak):
+    """Eq. 1 as a whole over the step's reference and candidates
+    (asmv_compare_eq); the kernel that adds the exact cosine sums is timed
+    alone, with CUDA events around its launches on the call's stream."""
+    ctx = setup.ctx
+    floats = ("f32", "bf16", "f16", "f8e4m3")
+    k = len(setup.cands)
+    ctx.compare_eq(setup.ref_regs, setup.cand_regs, setup.tol)
+    ctx.set_timing(True)
+    ms = []
+    for _ in range(max(3, args.steps)):
+        _, eqs = ctx.compare_eq(setup.ref_regs, setup.cand_regs, setup.tol)
+        ms.append(ctx.kernel_ms())
+    ctx.set_timing(False)
+    payload = sum(r.payload_bytes for r in setup.wl.regions if r.dtype in floats)
+    nbytes = payload * (1 + k)                 # the reference once, every candidate once
+    elems = sum(r.n_elems for r in setup.wl.regions if r.dtype in floats)
+    avg = float(np.mean(ms))
+    gbs = nbytes / (avg / 1e3) / 1e9
+    traffic, _ = kernel_traffic("eqsum", args.workload)
+    return {"kernel": "eq_kernel", "avg_launch_ms": round(avg, 4),
+            "algorithmic_bytes_per_launch": nbytes, "element_pairs_per_launch": elems * k,
+            "gbs": round(gbs, 1), "hbm_frac": round(gbs / peak, 4), "traffic": traffic,
+            "pairs_per_s": round(elems * k / (avg / 1e3), 1),
+            "theta": setup.asmv.THETA, "tau": setup.asmv.TAU,
+            "passing": int(sum(e["eq"] for cs in eqs for e in cs)), "checks": k * len(eqs[0])}
 
 
 def run_e2e(setup, args, device, world, barrier):
@@ -501,6 +541,7 @@ def main():
     ap.add_argument("--workload", default="batched_gemm_fp16")
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu", dest="cpu", action="store_false")
+    ap.add_argument("--no-eq", dest="eq", action="store_false")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     import __graft_entry__
