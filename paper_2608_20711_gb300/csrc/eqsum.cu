@@ -3,18 +3,22 @@
 //   S_rr = sum r*r over finite r,   S_cc = sum c*c over finite c,
 // for every float region of a reference and K candidates, added exactly.
 //
-// Exactness.  A decoded element is +-m 2^e with an integer significand m
-// (< 2^24 fp32, 2^8 bf16, 2^11 fp16, 2^4 fp8) and e the weight of its last
-// bit; a product is +-P 2^s with P = m_r m_c and s = e_r + e_c.  Each thread
-// adds its products at a fixed binary point 2^L into NACC signed 64-bit
-// accumulators 32 bits apart (accumulator q weighs 2^(L + 32q)):
-//   P 2^s = (P << (t & 31)) 2^(L + 32 (t >> 5)),  t = s - L,
-// (fp32 products are split into two 24-bit pieces first).  Integer additions
-// are exact and commute, so the sums do not depend on the order of the
-// elements or on the grid.  A product outside the window [L, L + 32 NACC)
-// goes straight to the region's global digits with 64-bit atomics: fp16 and
-// fp8 products always fit; bf16 and fp32 ones do for values between about
-// 2^-24 and 2^24.
+// Exactness.  Every sum is kept as integers at a fixed binary point and
+// integer additions are exact and commute, so the sums do not depend on the
+// order of the elements or on the grid.
+//   fp16 and fp8: a finite value is an integer multiple of one quantum, so
+//   each product is an integer at 2^-48 (fp16) or 2^-18 (fp8), formed with
+//   32x32+64-bit multiply-adds of signed limbs (eq_tile_fixed).
+//   bf16 and fp32: a decoded element is +-m 2^e with an integer significand
+//   m (< 2^8, 2^24) and e the weight of its last bit; a product is +-P 2^s,
+//   P = m_r m_c, s = e_r + e_c.  Each thread adds its products at a binary
+//   point 2^L into NACC signed 64-bit accumulators 32 bits apart
+//   (accumulator q weighs 2^(L + 32q)):
+//     P 2^s = (P << (t & 31)) 2^(L + 32 (t >> 5)),  t = s - L,
+//   (fp32 products are split into two 24-bit pieces first).  A product
+//   outside the window [L, L + 32 NACC) goes straight to the region's
+//   global digits with 64-bit atomics; values between about 2^-24 and 2^24
+//   stay in the window.
 //
 // Reduction.  Every tile, each warp carries its lanes' accumulators into
 // 32-bit digits, sums them over the warp with shuffles and adds them to the
@@ -42,8 +46,8 @@ template <int DT> struct Fmt;
 // kL: binary point of the window; kDig: index of the global digit at 2^kL
 template <> struct Fmt<kF32>  { static constexpr int kBytes = 4, kNacc = 4, kL = -94, kDig = 7; };
 template <> struct Fmt<kBF16> { static constexpr int kBytes = 2, kNacc = 3, kL = -62, kDig = 7; };
-template <> struct Fmt<kF16>  { static constexpr int kBytes = 2, kNacc = 2, kL = -48, kDig = 2; };
-template <> struct Fmt<kF8>   { static constexpr int kBytes = 1, kNacc = 1, kL = -18, kDig = 2; };
+template <> struct Fmt<kF16>  { static constexpr int kL = -48, kDig = 2; };   // fixed point, below
+template <> struct Fmt<kF8>   { static constexpr int kL = -18, kDig = 2; };
 
 static_assert(Fmt<kF32>::kL - 32 * Fmt<kF32>::kDig == eq_digit_base(kF32), "fp32 digits");
 static_assert(Fmt<kBF16>::kL - 32 * Fmt<kBF16>::kDig == eq_digit_base(kBF16), "bf16 digits");
@@ -236,6 +240,177 @@ __device__ __noinline__ void eq_tile(const EqParams &p, const CmpRegion &R, uint
   }
 }
 
+// ---------------------------------------------------------------------
+// fp16 and fp8: every finite value is an integer multiple of one quantum,
+// x = X 2^-24 with |X| < 2^40 (fp16) or x = X 2^-9 with |X| < 2^18 (fp8
+// e4m3), so the sums are sums of integer products at one binary point
+// (2^-48, 2^-18).  fp16: X = hi 2^20 + lo with signed limbs (|hi| <= 2^20,
+// |lo| <= 2^19), and
+//   x*y 2^48 = (hi hi') 2^40 + (hi lo' + lo hi') 2^20 + lo lo',
+// each partial product at most 2^40 and added with one 32x32+64
+// multiply-add; fp8: X X' < 2^36 with one multiply-add.  A non-finite value
+// gets X = 0 and drops out of every sum it would enter.
+// ---------------------------------------------------------------------
+struct Limbs { int hi, lo; };
+struct Acc3 { long long s2, s1, s0; };        // s2 2^40 + s1 2^20 + s0
+
+// round(v) for |v| < 2^22: adding 1.5 2^23 leaves the integer in the low
+// mantissa bits (one fp32 rounding, to nearest even).
+constexpr float kMagic = 12582912.0f;
+constexpr int kMagicBits = 0x4B400000;
+
+// fp16 bits -> X = x 2^24 as hi 2^20 + lo, exactly, on the fp32 pipe:
+// hi = round(16 x) (|hi| <= 2^20), lo = (x - hi/16) 2^24 (an integer, since
+// x is a multiple of 2^-24 and |x - hi/16| <= 2^-5, exact in fp32).
+__device__ __forceinline__ Limbs fix_f16(uint32_t b) {
+  b = ((b & 0x7C00u) == 0x7C00u) ? 0u : b;                      // NaN, Inf -> 0
+  const float x = __half2float(__ushort_as_half((unsigned short)b));
+  const float hf = __fmaf_rn(x, 16.0f, kMagic);
+  const float l = __fmaf_rn(__fsub_rn(hf, kMagic), -0.0625f, x);
+  return {__float_as_int(hf) - kMagicBits,
+          __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic)) - kMagicBits};
+}
+
+// fp8 e4m3 bits -> X = x 2^9 (|X| < 2^18), exactly.
+__device__ __forceinline__ int fix_f8(uint32_t b) {
+  b = ((b & 0x7Fu) == 0x7Fu) ? 0u : b;                          // NaN -> 0
+  const __half_raw h = __nv_cvt_fp8_to_halfraw((__nv_fp8_storage_t)b, __NV_E4M3);
+  const float x = __half2float(__half(h));
+  return __float_as_int(__fmaf_rn(x, 512.0f, kMagic)) - kMagicBits;
+}
+
+__device__ __forceinline__ long long mad_wide(int a, int b, long long c) {
+  return (long long)a * (long long)b + c;
+}
+
+__device__ __forceinline__ void mac(Acc3 &a, const Limbs &x, const Limbs &y) {
+  a.s2 = mad_wide(x.hi, y.hi, a.s2);
+  a.s1 = mad_wide(x.hi, y.lo, a.s1);
+  a.s1 = mad_wide(x.lo, y.hi, a.s1);
+  a.s0 = mad_wide(x.lo, y.lo, a.s0);
+}
+
+__device__ __forceinline__ void sq(Acc3 &a, const Limbs &x) {
+  a.s2 = mad_wide(x.hi, x.hi, a.s2);
+  a.s1 = mad_wide(x.hi, 2 * x.lo, a.s1);
+  a.s0 = mad_wide(x.lo, x.lo, a.s0);
+}
+
+// Warp-sum a digit vector and add it to the CTA's shared digits.
+template <int N>
+__device__ __forceinline__ void warp_add_digits(long long (&d)[N], long long *sdig) {
+#pragma unroll
+  for (int k = 0; k < N; ++k) {
+    long long v = d[k];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    if ((threadIdx.x & 31) == 0 && v != 0)
+      atomicAdd(reinterpret_cast<unsigned long long *>(sdig + k), (unsigned long long)v);
+  }
+}
+
+// sum = s2 2^40 + s1 2^20 + s0 (|s| < 2^63) as four digits of 32 bits.
+__device__ __forceinline__ void flush3(Acc3 &a, long long *sdig) {
+  const __int128 T = (__int128)a.s0 + (__int128)a.s1 * ((__int128)1 << 20) +
+                    (__int128)a.s2 * ((__int128)1 << 40);
+  long long d[4] = {(long long)(T & 0xFFFFFFFF), (long long)((T >> 32) & 0xFFFFFFFF),
+                    (long long)((T >> 64) & 0xFFFFFFFF), (long long)(T >> 96)};
+  warp_add_digits(d, sdig);
+  a.s2 = a.s1 = a.s0 = 0;
+}
+
+__device__ __forceinline__ void flush1(long long &s, long long *sdig) {
+  long long d[2] = {s & 0xFFFFFFFFll, s >> 32};
+  warp_add_digits(d, sdig);
+  s = 0;
+}
+
+__device__ __forceinline__ uint32_t half_of(const uint4 &v, int k) {
+  const uint32_t w = k < 2 ? v.x : k < 4 ? v.y : k < 6 ? v.z : v.w;
+  return (k & 1) ? (w >> 16) : (w & 0xFFFFu);
+}
+__device__ __forceinline__ uint32_t byte_of(const uint4 &v, int k) {
+  const uint32_t w = k < 4 ? v.x : k < 8 ? v.y : k < 12 ? v.z : v.w;
+  return (w >> (8 * (k & 3))) & 0xFFu;
+}
+
+// One tile of an fp16 or fp8 region: S_rr once, then the candidates two at
+// a time (the reference chunk is decoded once per pair).
+template <int DT>
+__device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R, uint32_t region,
+                                           uint64_t a, uint32_t nb, long long *sdig) {
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t nchunks = (nb + 15u) >> 4;
+  const uint32_t per_warp = (nchunks + kWarps - 1) / kWarps;
+  const uint32_t c0 = warp * per_warp;
+  const uint32_t c1 = min(c0 + per_warp, nchunks);
+  const uint32_t rounds = (per_warp + 31u) >> 5;     // the same for every warp
+  const uint64_t ref = R.ref + a;
+  if (p.do_rr) {
+    Acc3 rr = {0, 0, 0};
+    long long r8 = 0;
+#pragma unroll 1
+    for (uint32_t r = 0; r < rounds; ++r) {
+      const uint32_t c = c0 + 32u * r + lane;
+      uint4 rv = make_uint4(0u, 0u, 0u, 0u);
+      if (c < c1) rv = load_chunk(ref + 16ull * c, min(16u, nb - 16u * c), R.vec, true);
+      if (DT == kF16) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) sq(rr, fix_f16(half_of(rv, k)));
+      } else {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) { const int x = fix_f8(byte_of(rv, k)); r8 = mad_wide(x, x, r8); }
+      }
+    }
+    if (DT == kF16) flush3(rr, sdig); else flush1(r8, sdig);
+  }
+  for (uint32_t j = 0; j < p.K; j += 2) {
+    const bool two = j + 1 < p.K;                    // uniform
+    const uint64_t cb0 = p.cands[(size_t)j * p.nregions + region] + a;
+    const uint64_t cb1 = two ? p.cands[(size_t)(j + 1) * p.nregions + region] + a : cb0;
+    Acc3 rc0 = {0, 0, 0}, cc0 = {0, 0, 0}, rc1 = {0, 0, 0}, cc1 = {0, 0, 0};
+    long long rc8_0 = 0, cc8_0 = 0, rc8_1 = 0, cc8_1 = 0;
+#pragma unroll 1
+    for (uint32_t r = 0; r < rounds; ++r) {
+      const uint32_t c = c0 + 32u * r + lane;
+      uint4 rv = make_uint4(0u, 0u, 0u, 0u), v0 = rv, v1 = rv;
+      if (c < c1) {
+        const uint32_t bytes = min(16u, nb - 16u * c);
+        rv = load_chunk(ref + 16ull * c, bytes, R.vec, true);     // L1 hit after the first pair
+        v0 = load_chunk(cb0 + 16ull * c, bytes, R.vec, false);
+        if (two) v1 = load_chunk(cb1 + 16ull * c, bytes, R.vec, false);
+      }
+      if (DT == kF16) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const Limbs x = fix_f16(half_of(rv, k));
+          const Limbs y0 = fix_f16(half_of(v0, k));
+          const Limbs y1 = fix_f16(half_of(v1, k));
+          mac(rc0, x, y0); sq(cc0, y0);
+          mac(rc1, x, y1); sq(cc1, y1);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int x = fix_f8(byte_of(rv, k));
+          const int y0 = fix_f8(byte_of(v0, k)), y1 = fix_f8(byte_of(v1, k));
+          rc8_0 = mad_wide(x, y0, rc8_0); cc8_0 = mad_wide(y0, y0, cc8_0);
+          rc8_1 = mad_wide(x, y1, rc8_1); cc8_1 = mad_wide(y1, y1, cc8_1);
+        }
+      }
+    }
+    if (DT == kF16) {
+      flush3(rc0, sdig + (1 + 2 * j) * kWin);
+      flush3(cc0, sdig + (2 + 2 * j) * kWin);
+      if (two) { flush3(rc1, sdig + (3 + 2 * j) * kWin); flush3(cc1, sdig + (4 + 2 * j) * kWin); }
+    } else {
+      flush1(rc8_0, sdig + (1 + 2 * j) * kWin);
+      flush1(cc8_0, sdig + (2 + 2 * j) * kWin);
+      if (two) { flush1(rc8_1, sdig + (3 + 2 * j) * kWin); flush1(cc8_1, sdig + (4 + 2 * j) * kWin); }
+    }
+  }
+}
+
 // Add the CTA's shared digits of `region` to its global digits; zero them.
 __device__ void cta_flush(const EqParams &p, uint32_t region, uint32_t dtype, long long *sdig) {
   __syncthreads();
@@ -275,8 +450,8 @@ __global__ void __launch_bounds__(kThreads) eq_kernel(EqParams p) {
     switch (R.dtype) {
       case kF32: eq_tile<kF32>(p, R, i, a, nb, sdig); break;
       case kBF16: eq_tile<kBF16>(p, R, i, a, nb, sdig); break;
-      case kF16: eq_tile<kF16>(p, R, i, a, nb, sdig); break;
-      default: eq_tile<kF8>(p, R, i, a, nb, sdig); break;
+      case kF16: eq_tile_fixed<kF16>(p, R, i, a, nb, sdig); break;
+      default: eq_tile_fixed<kF8>(p, R, i, a, nb, sdig); break;
     }
   }
   if (cur != 0xFFFFFFFFu) cta_flush(p, cur, cur_dtype, sdig);
