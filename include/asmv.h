@@ -238,6 +238,57 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
  * asmv_compare_eq never reach). */
 int asmv_exact_to_double(const int64_t *digits, int ndigits, int base_exp, double *out);
 
+/* ---------------------------------------------------------------------
+ * GatedEval timing and the commit gate (Sec. 3.4, Algorithm 1; Eq. 2).
+ * Correctness first (asmv_compare_eq over every evaluated input), then
+ * timing: warm-up launches, then R launches each timed with its own pair of
+ * CUDA events; the latency is their median.  The speedup of a candidate c
+ * is s(c) = T(K0) / T(c).  Eq. 2 commits c only if it is equivalent on
+ * every input and
+ *   s(c) >= max(m*, s_floor),   m* = (1 + max(eps, k * cv)) * s(K*),
+ * with K* the current verified best (s(K0) = 1) and cv the coefficient of
+ * variation of the timings.  The paper uses eps = 0.002, k = 0.85,
+ * s_floor = 1.0 (Sec. 5).
+ * ------------------------------------------------------------------- */
+#define ASMV_GATE_EPS     0.002
+#define ASMV_GATE_K       0.85
+#define ASMV_GATE_S_FLOOR 1.0
+
+typedef struct {
+  double median_ms;   /* median (mean of the two middle samples when R is even) */
+  double mean_ms;     /* sum in sample order, divided by R */
+  double cv;          /* sqrt(sum (x - mean)^2 / (R - 1)) / mean; 0 when R == 1 */
+  uint64_t r;         /* number of samples */
+} asmv_timing;        /* 32 bytes */
+
+typedef struct { double eps, k, s_floor; } asmv_gate_params;
+
+/* Median, mean and coefficient of variation of r timing samples, each
+ * operation in double in the order stated above.  EINVAL for a null
+ * pointer, r == 0, or a sample that is not finite and positive. */
+int asmv_timing_summary(const double *samples_ms, size_t r, asmv_timing *out);
+
+/* Eq. 2: *m_star = (1 + max(eps, k * cv)) * s_best (multiply k*cv, take the
+ * max, add 1, multiply by s_best), *commit = all_eq && s_cand >=
+ * max(*m_star, s_floor).  EINVAL for null pointers, non-finite or negative
+ * arguments, or s_best == 0. */
+int asmv_commit_gate(int all_eq, double s_cand, double s_best, double cv,
+                     const asmv_gate_params *params, double *m_star, int *commit);
+
+/* Launch callback: enqueue the kernel(s) to time on `stream`. */
+typedef void (*asmv_launch_fn)(void *user, asmv_stream_t stream);
+
+/* Event-timed launches: `warmup` untimed calls of fn, then r calls, each
+ * bracketed by its own pair of CUDA events recorded on `stream`;
+ * samples_ms[i] is the device time of call i.  Synchronises the stream
+ * once at the end.  Runs on the current CUDA device; the events are
+ * created and destroyed inside the call.  EINVAL for a null fn or
+ * samples_ms or r == 0; ECUDA if event creation, recording or timing
+ * fails (the CUDA error is returned through *cuda_error when it is not
+ * null). */
+int asmv_time_launches(asmv_launch_fn fn, void *user, int warmup, size_t r,
+                       double *samples_ms, asmv_stream_t stream, int *cuda_error);
+
 /* Host-only validation of a region table, the checks every call above
  * makes before touching the device, except the device-memory checks.
  * for_fill != 0 adds the distribution and overlap rules of asmv_fill.

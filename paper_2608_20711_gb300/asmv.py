@@ -57,6 +57,19 @@ class EqResult(ctypes.Structure):
                 ("flags", ctypes.c_uint32), ("eq", ctypes.c_uint32)]
 
 
+class Timing(ctypes.Structure):
+    """asmv_timing (32 bytes)."""
+    _fields_ = [("median_ms", ctypes.c_double), ("mean_ms", ctypes.c_double),
+                ("cv", ctypes.c_double), ("r", ctypes.c_uint64)]
+
+
+class GateParams(ctypes.Structure):
+    _fields_ = [("eps", ctypes.c_double), ("k", ctypes.c_double), ("s_floor", ctypes.c_double)]
+
+
+GATE_EPS, GATE_K, GATE_S_FLOOR = 0.002, 0.85, 1.0     # Eq. 2 constants used in the paper (Sec. 5)
+LAUNCH_FN = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_void_p)
+
 STATS_FIELDS = [f for f, _ in Stats._fields_]
 EQ_FIELDS = [f for f, _ in EqResult._fields_]
 EQ_COS, EQ_LINF, EQ_INT, EQ_GUARD = 1, 2, 4, 8
@@ -68,7 +81,8 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_compare", "asmv_compare_batched", "asmv_check_regions",
                  "asmv_ctx_set_timing", "asmv_ctx_kernel_ms", "asmv_ctx_cuda_error",
                  "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version",
-                 "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double")
+                 "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double",
+                 "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches")
 NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -113,6 +127,13 @@ def lib():
                                       ctypes.c_double, SP, ctypes.POINTER(EqResult), vp]
         L.asmv_exact_to_double.argtypes = [ctypes.POINTER(ctypes.c_int64), ctypes.c_int,
                                            ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
+        dp = ctypes.POINTER(ctypes.c_double)
+        L.asmv_timing_summary.argtypes = [dp, sz, ctypes.POINTER(Timing)]
+        L.asmv_commit_gate.argtypes = [ctypes.c_int, ctypes.c_double, ctypes.c_double,
+                                       ctypes.c_double, ctypes.POINTER(GateParams), dp,
+                                       ctypes.POINTER(ctypes.c_int)]
+        L.asmv_time_launches.argtypes = [LAUNCH_FN, vp, ctypes.c_int, sz, dp, vp,
+                                         ctypes.POINTER(ctypes.c_int)]
         _lib = L
     return _lib
 
@@ -300,6 +321,54 @@ def exact_to_double(digits: Sequence[int], base_exp: int) -> float:
     if rc != OK:
         raise AsmvError(rc, strerror(rc))
     return out.value
+
+
+def timing_summary(samples_ms: Sequence[float]) -> dict:
+    """asmv_timing_summary: median, mean and cv of timing samples."""
+    arr = (ctypes.c_double * max(1, len(samples_ms)))(*[float(x) for x in samples_ms])
+    out = Timing()
+    rc = lib().asmv_timing_summary(arr, len(samples_ms), ctypes.byref(out))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return {"median_ms": out.median_ms, "mean_ms": out.mean_ms, "cv": out.cv, "r": int(out.r)}
+
+
+def commit_gate(all_eq: bool, s_cand: float, s_best: float, cv: float, eps: float = GATE_EPS,
+                k: float = GATE_K, s_floor: float = GATE_S_FLOOR):
+    """asmv_commit_gate (Eq. 2): returns (m_star, commit)."""
+    m = ctypes.c_double()
+    c = ctypes.c_int()
+    rc = lib().asmv_commit_gate(1 if all_eq else 0, float(s_cand), float(s_best), float(cv),
+                                ctypes.byref(GateParams(eps, k, s_floor)), ctypes.byref(m),
+                                ctypes.byref(c))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return m.value, bool(c.value)
+
+
+def time_launches(fn, r: int, warmup: int = 3, stream=None) -> List[float]:
+    """asmv_time_launches: fn(stream_handle) enqueues the work to time; returns
+    the device time of each of r calls (ms), after `warmup` untimed calls."""
+    handle = _stream_handle(stream)
+    err: List[BaseException] = []
+
+    def cb(_user, st):
+        if err:
+            return
+        try:
+            fn(st or 0)                  # a null stream handle arrives as None
+        except BaseException as e:       # re-raised below, after the C call returns
+            err.append(e)
+    cfn = LAUNCH_FN(cb)
+    out = (ctypes.c_double * max(1, r))()
+    cuda_err = ctypes.c_int()
+    rc = lib().asmv_time_launches(cfn, None, int(warmup), int(r), out, handle,
+                                  ctypes.byref(cuda_err))
+    if err:
+        raise err[0]
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc), cuda_err.value)
+    return [out[i] for i in range(r)]
 
 
 def compare_noalloc(ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:
