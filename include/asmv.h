@@ -289,6 +289,46 @@ typedef void (*asmv_launch_fn)(void *user, asmv_stream_t stream);
 int asmv_time_launches(asmv_launch_fn fn, void *user, int warmup, size_t r,
                        double *samples_ms, asmv_stream_t stream, int *cuda_error);
 
+/* ---------------------------------------------------------------------
+ * Tier 2 replay (Sec. 3.4): a captured dispatch is replayed against memory
+ * restored to its captured pre-dispatch state, at the original virtual
+ * addresses when the kernel arguments hold absolute pointers.
+ * ------------------------------------------------------------------- */
+
+/* Restore: for each region i, copy payload_bytes(i) bytes from the device
+ * address src[i] (the captured pre-dispatch payload, any alignment) into
+ * the region's payload, and write the region's canary over both guard
+ * bands.  One kernel for the whole table; asynchronous on `stream`.
+ * EINVAL: as asmv_fill's table rules without the distribution rules
+ * (allocations must not overlap), a null src with n > 0, a null src[i]
+ * for a non-empty payload, a source that is not device memory of ctx's
+ * device or that overlaps a region's allocation. */
+int asmv_restore(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *src, size_t n,
+                 asmv_stream_t stream);
+
+/* Capture: for each region i, copy its payload into the device address
+ * dst[i] (payload_bytes(i) bytes, any alignment); guard bands are neither
+ * read nor written.  Asynchronous on `stream`.  EINVAL as asmv_restore,
+ * with destinations that must not overlap one another or any region. */
+int asmv_capture(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *dst, size_t n,
+                 asmv_stream_t stream);
+
+/* Device memory at a chosen virtual address.  asmv_va_map reserves `bytes`
+ * (rounded up to the allocation granularity) of virtual address space at
+ * `addr` (0: the driver chooses), backs it with physical memory of
+ * `device`, maps it and grants the device read/write access.  addr must be
+ * a multiple of asmv_va_granularity(device).  EINVAL for a null out, zero
+ * bytes, a misaligned addr, or an addr whose range the driver cannot give
+ * (in use); ENOMEM when memory is short; ECUDA otherwise.  Memory from
+ * asmv_va_map is valid in every call above.  asmv_va_unmap waits for the
+ * device to go idle, then unmaps and frees. */
+typedef struct asmv_va asmv_va;
+int asmv_va_granularity(int device, size_t *out);
+int asmv_va_map(int device, uint64_t addr, size_t bytes, asmv_va **out);
+uint64_t asmv_va_address(const asmv_va *va);
+size_t asmv_va_size(const asmv_va *va);
+int asmv_va_unmap(asmv_va *va);
+
 /* Host-only validation of a region table, the checks every call above
  * makes before touching the device, except the device-memory checks.
  * for_fill != 0 adds the distribution and overlap rules of asmv_fill.

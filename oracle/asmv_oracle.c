@@ -538,6 +538,17 @@ void oracle_compare_region(const uint8_t *ref_alloc, uint32_t ref_glo,
 }
 
 /* ======================================================================
+ * Tier 2 replay restore (Sec. 3.4, Tier 2): a region is put back into its
+ * captured pre-dispatch state -- the captured payload bytes, and the canary
+ * in both guard bands -- before each replay.
+ * ====================================================================== */
+void oracle_restore_region(uint8_t *alloc, uint64_t payload_bytes, uint32_t glo, uint32_t ghi,
+                           uint8_t canary, const uint8_t *captured) {
+  oracle_fill_guards(alloc, payload_bytes, glo, ghi, canary);
+  memcpy(alloc + glo, captured, payload_bytes);
+}
+
+/* ======================================================================
  * Eq. 1 aggregate terms.  The cosine c_x = cos(K'(x), O(x)) of a float
  * region is built from three sums over its elements:
  *   S_rc = sum r*c,   S_rr = sum r*r,   S_cc = sum c*c.

@@ -116,6 +116,8 @@ def _load(path):
                 c.POINTER(_RegionStats)]
             L.oracle_eq_sums_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
                                                c.c_uint64, _i64p]
+            L.oracle_restore_region.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
+                                                c.c_uint8, _u8p]
     return L
 
 
@@ -376,3 +378,13 @@ def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
     out["flags"] = flags
     out["eq"] = int(flags == EQ_COS | EQ_LINF | EQ_INT | EQ_GUARD)
     return out
+
+
+# ------------------------------------------------------- Tier 2 restore
+def restore_region(alloc, payload_bytes, guard_lo, guard_hi, canary, captured):
+    """Write the canary over both guard bands of `alloc` (a uint8 array of
+    guard_lo + payload_bytes + guard_hi bytes) and the captured bytes over
+    its payload."""
+    assert alloc.size >= guard_lo + payload_bytes + guard_hi and captured.size >= payload_bytes
+    lib().oracle_restore_region(_ptr(alloc, _u8p), payload_bytes, guard_lo, guard_hi, canary,
+                                _ptr(np.ascontiguousarray(captured), _u8p))

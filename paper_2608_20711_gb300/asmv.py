@@ -82,7 +82,9 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_ctx_set_timing", "asmv_ctx_kernel_ms", "asmv_ctx_cuda_error",
                  "asmv_ctx_launches", "asmv_strerror", "asmv_abi_version",
                  "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double",
-                 "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches")
+                 "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches",
+                 "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
+                 "asmv_va_address", "asmv_va_size", "asmv_va_unmap")
 NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -134,6 +136,16 @@ def lib():
                                        ctypes.POINTER(ctypes.c_int)]
         L.asmv_time_launches.argtypes = [LAUNCH_FN, vp, ctypes.c_int, sz, dp, vp,
                                          ctypes.POINTER(ctypes.c_int)]
+        u64p = ctypes.POINTER(ctypes.c_uint64)
+        L.asmv_restore.argtypes = [vp, RP, u64p, sz, vp]
+        L.asmv_capture.argtypes = [vp, RP, u64p, sz, vp]
+        L.asmv_va_granularity.argtypes = [ctypes.c_int, ctypes.POINTER(sz)]
+        L.asmv_va_map.argtypes = [ctypes.c_int, ctypes.c_uint64, sz, ctypes.POINTER(vp)]
+        L.asmv_va_address.argtypes = [vp]
+        L.asmv_va_address.restype = ctypes.c_uint64
+        L.asmv_va_size.argtypes = [vp]
+        L.asmv_va_size.restype = sz
+        L.asmv_va_unmap.argtypes = [vp]
         _lib = L
     return _lib
 
@@ -291,6 +303,19 @@ class Context:
         flat = stats_dicts(out, k * n)
         return [flat[j * n:(j + 1) * n] for j in range(k)]
 
+    def restore(self, regions: Sequence, src: Sequence[int], stream=None):
+        """asmv_restore (Tier 2): payload i <- device buffer src[i]; guard
+        bands <- canary.  Asynchronous on the stream."""
+        arr = region_array(regions)
+        a = (ctypes.c_uint64 * max(1, len(regions)))(*[int(x) for x in src])
+        self._check(self._lib.asmv_restore(self._h, arr, a, len(regions), _stream_handle(stream)))
+
+    def capture(self, regions: Sequence, dst: Sequence[int], stream=None):
+        """asmv_capture: device buffer dst[i] <- payload i.  Asynchronous."""
+        arr = region_array(regions)
+        a = (ctypes.c_uint64 * max(1, len(regions)))(*[int(x) for x in dst])
+        self._check(self._lib.asmv_capture(self._h, arr, a, len(regions), _stream_handle(stream)))
+
     def compare_eq(self, ref: Sequence, cands: Sequence[Sequence], tol, theta: float = THETA,
                    tau: float = TAU, stream=None):
         """asmv_compare_eq: (stats, eq) with stats[j][i] as compare_batched
@@ -369,6 +394,41 @@ def time_launches(fn, r: int, warmup: int = 3, stream=None) -> List[float]:
     if rc != OK:
         raise AsmvError(rc, strerror(rc), cuda_err.value)
     return [out[i] for i in range(r)]
+
+
+def va_granularity(device: int = 0) -> int:
+    g = ctypes.c_size_t()
+    rc = lib().asmv_va_granularity(int(device), ctypes.byref(g))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return int(g.value)
+
+
+class VaMapping:
+    """asmv_va_map: device memory at a chosen virtual address (0: any)."""
+
+    def __init__(self, nbytes: int, addr: int = 0, device: int = 0):
+        self._lib = lib()
+        h = ctypes.c_void_p()
+        rc = self._lib.asmv_va_map(int(device), int(addr), int(nbytes), ctypes.byref(h))
+        if rc != OK:
+            raise AsmvError(rc, strerror(rc))
+        self._h = h
+        self.address = int(self._lib.asmv_va_address(h))
+        self.size = int(self._lib.asmv_va_size(h))
+
+    def unmap(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            rc = self._lib.asmv_va_unmap(self._h)
+            if rc != OK:
+                raise AsmvError(rc, strerror(rc))
+            self._h = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.unmap()
 
 
 def compare_noalloc(ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:

@@ -26,6 +26,7 @@ static_assert(sizeof(asmv_region) == 56, "asmv_region layout");
 static_assert(sizeof(asmv_stats) == 64, "asmv_stats layout");
 static_assert(sizeof(asmv_eq) == 40, "asmv_eq layout");
 static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
+static_assert(sizeof(CopyRegion) == 48, "copy region layout");
 static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
               "plan layouts");
 
@@ -199,6 +200,7 @@ struct asmv_ctx {
   int sms = 0;
   int fill_ctas = 1;
   int eq_ctas = 1;
+  int copy_ctas = 1;
   void *dws = nullptr;
   size_t dws_cap = 0;
   unsigned char *hst = nullptr;
@@ -448,6 +450,7 @@ int asmv_ctx_create(asmv_ctx **out, int device) {
   }
   ctx->fill_ctas = fill_max_ctas_per_sm();
   ctx->eq_ctas = eq_max_ctas_per_sm();
+  ctx->copy_ctas = copy_max_ctas_per_sm();
   void *fn = nullptr;
   cudaDriverEntryPointQueryResult q;
   if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &fn, 12000, cudaEnableDefault, &q) ==
@@ -836,6 +839,97 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
   std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
   std::memcpy(eq_host, res.data(), res.size() * sizeof(asmv_eq));
   return ASMV_OK;
+}
+
+// Shared body of asmv_restore / asmv_capture: move every region's payload
+// between the region and the caller's buffer addrs[i] (restore: buffer ->
+// region, and guard bands rewritten; capture: region -> buffer).
+static int run_copy(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *addrs, size_t n,
+                    asmv_stream_t stream, bool restore) {
+  if (ctx == nullptr || (n > 0 && addrs == nullptr)) return ASMV_EINVAL;
+  int rc = check_table(regions, n, false);
+  if (rc != ASMV_OK) return rc;
+  // allocations pairwise disjoint; buffers disjoint from every allocation
+  // (and, for capture, from one another)
+  std::vector<std::pair<std::pair<uint64_t, uint64_t>, int>> spans;   // (range, 0 alloc / 1 buffer)
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    region_extent(regions[i], &pb, &tot);
+    if (tot > 0) spans.push_back({{regions[i].alloc, regions[i].alloc + tot}, 0});
+    if (pb > 0) {
+      if (addrs[i] == 0 || addrs[i] + pb < addrs[i]) return ASMV_EINVAL;
+      spans.push_back({{addrs[i], addrs[i] + pb}, 1});
+    }
+  }
+  std::sort(spans.begin(), spans.end());
+  for (size_t i = 0; i < spans.size(); ++i)
+    for (size_t j = i + 1; j < spans.size() && spans[j].first.first < spans[i].first.second; ++j)
+      if (spans[i].second == 0 || spans[j].second == 0 || !restore) return ASMV_EINVAL;
+  if (n == 0) return ASMV_OK;
+  DeviceScope ds(ctx->device);
+  if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
+  std::pair<uint64_t, uint64_t> last(0, 0);
+  if ((rc = check_device_table(ctx, regions, n, last)) != ASMV_OK) return rc;
+  for (size_t i = 0; i < n; ++i) {
+    uint64_t pb, tot;
+    region_extent(regions[i], &pb, &tot);
+    if ((rc = check_device_span(ctx, addrs[i], pb, last)) != ASMV_OK) return rc;
+  }
+  std::vector<CopyRegion> cr(n + 1);
+  std::vector<GuardSeg> segs;
+  uint64_t tile = 0;
+  for (size_t i = 0; i < n; ++i) {
+    const asmv_region &r = regions[i];
+    uint64_t pb, tot;
+    region_extent(r, &pb, &tot);
+    CopyRegion &c = cr[i];
+    std::memset(&c, 0, sizeof c);
+    const uint64_t payload = r.alloc + r.guard_lo;
+    c.dst = restore ? payload : addrs[i];
+    c.src = restore ? addrs[i] : payload;
+    c.bytes = pb;
+    c.tile0 = tile;
+    c.vec = (c.dst % 16 == 0) && (c.src % 16 == 0);
+    tile += tiles_of(pb);
+    if (restore) add_region_guards(segs, r, kSegFill, (uint32_t)i);
+  }
+  std::memset(&cr[n], 0, sizeof(CopyRegion));
+  cr[n].tile0 = tile;
+  if (tile == 0 && segs.empty()) return ASMV_OK;
+  Image img;
+  const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CopyRegion));
+  const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
+  unsigned char *dev = nullptr;
+  const cudaStream_t s = (cudaStream_t)stream;
+  if ((rc = stage(ctx, img, 0, s, &dev)) != ASMV_OK) return rc;
+  CopyParams p;
+  std::memset(&p, 0, sizeof p);
+  p.regions = (const CopyRegion *)(dev + o_regs);
+  p.segs = (const GuardSeg *)(dev + o_segs);
+  p.ntiles = tile;
+  p.nregions = (uint32_t)n;
+  p.nsegs = (uint32_t)segs.size();
+  cudaError_t e;
+  if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  if ((e = (cudaError_t)launch_copy(p, grid_for(ctx, tile, segs.size(), ctx->copy_ctas), s)) !=
+      cudaSuccess)
+    return fail_cuda(ctx, e);
+  ctx->launches += 1;
+  if (ctx->timing) {
+    if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
+    ctx->timed = true;
+  }
+  return after_launch(ctx, s);
+}
+
+int asmv_restore(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *src, size_t n,
+                 asmv_stream_t stream) {
+  return run_copy(ctx, regions, src, n, stream, true);
+}
+
+int asmv_capture(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *dst, size_t n,
+                 asmv_stream_t stream) {
+  return run_copy(ctx, regions, dst, n, stream, false);
 }
 
 int asmv_exact_to_double(const int64_t *digits, int ndigits, int base_exp, double *out) {

@@ -131,7 +131,23 @@ struct EqParams {
   uint32_t do_rr;              // this launch also adds S_rr
 };
 
-// Launchers (defined in fill.cu / compare.cu / eqsum.cu).  Return a cudaError_t.
+// One region of a restore or capture launch (48 B): move `bytes` from src to
+// dst; the table has a sentinel entry after the last region.
+struct CopyRegion {
+  uint64_t dst, src, bytes, tile0;
+  uint32_t vec;         // src and dst both 16-byte aligned
+  uint32_t pad_[3];
+};
+
+struct CopyParams {
+  const CopyRegion *regions;   // nregions + 1 entries
+  const GuardSeg *segs;        // guard bands to rewrite with the canary (restore only)
+  uint64_t ntiles;             // tiles of kTileBytes
+  uint32_t nregions;
+  uint32_t nsegs;
+};
+
+// Launchers (defined in fill.cu / compare.cu / eqsum.cu / copy.cu).  Return a cudaError_t.
 int launch_fill(const FillParams &p, int grid, void *stream);
 int launch_compare(const CmpParams &p, int grid, void *stream);
 int fill_max_ctas_per_sm();
@@ -139,5 +155,7 @@ uint32_t compare_tile_bytes(uint32_t K);
 size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes);
 int launch_eq(const EqParams &p, int grid, void *stream);
 int eq_max_ctas_per_sm();
+int launch_copy(const CopyParams &p, int grid, void *stream);
+int copy_max_ctas_per_sm();
 
 }  // namespace asmv
