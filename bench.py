@@ -12,7 +12,8 @@ Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|referenc
 
 Beside the step, the line carries `eq1`: Eq. 1 as a whole (the exact sums
 of the cosine term over the same reference and candidates), its kernel
-timed alone with CUDA events.
+timed alone with CUDA events; and `restore`: the Tier 2 restore of the
+step's input regions from a captured snapshot, timed the same way.
 For N > 1 launch under torchrun; every rank runs its own replica (weak
 scaling, no data-path collective) and rank 0 prints one JSON line.
 """
@@ -120,7 +121,8 @@ def kernel_traffic(kernel, workload):
 # the source files each kernel is compiled from
 KERNEL_SOURCES = {"fill": ("fill.cu", "device.cuh", "ln_table.h", "plan.h"),
                   "compare": ("compare.cu", "device.cuh", "plan.h"),
-                  "eqsum": ("eqsum.cu", "device.cuh", "plan.h")}
+                  "eqsum": ("eqsum.cu", "device.cuh", "plan.h"),
+                  "copy": ("copy.cu", "device.cuh", "plan.h")}
 
 
 def source_hash(kernel):
@@ -427,6 +429,8 @@ def run_mine(args):
     }
     if args.eq:
         line["eq1"] = run_eq1(setup, args, peak)
+    if args.restore:
+        line["restore"] = run_restore(setup, args, peak)
     if rank == 0 and world == 1 and args.cpu:
         line["cpu_baseline"] = cpu_oracle_sample(setup)
     if rank == 0:
@@ -464,6 +468,42 @@ def run_eq1(setup, args, peak):
             "pairs_per_s": round(elems * k / (avg / 1e3), 1),
             "theta": setup.asmv.THETA, "tau": setup.asmv.TAU,
             "passing": int(sum(e["eq"] for cs in eqs for e in cs)), "checks": k * len(eqs[0])}
+
+
+def run_restore(setup, args, peak):
+    """Tier 2 restore of the step's input regions (asmv_restore) from a
+    snapshot taken with asmv_capture; the copy kernel timed alone with CUDA
+    events around its launch."""
+    torch = setup.torch
+    ctx = setup.ctx
+    specs = setup.fill_specs
+    offs, total = [], 0
+    for r in specs:
+        total = (total + 255) // 256 * 256
+        offs.append(total)
+        total += r.payload_bytes
+    snap = torch.empty(max(total, 1), dtype=torch.uint8, device=setup.device)
+    src = [snap.data_ptr() + o for o in offs]
+    ctx.capture(setup.fill_regs, src)
+    ctx.restore(setup.fill_regs, src)
+    ctx.set_timing(True)
+    ms = []
+    for _ in range(max(3, args.steps)):
+        ctx.restore(setup.fill_regs, src)
+        ms.append(ctx.kernel_ms())
+    ctx.set_timing(False)
+    torch.cuda.synchronize(setup.device)
+    payload = sum(r.payload_bytes for r in specs)
+    guards = sum(r.guard_lo + r.guard_hi for r in specs)
+    nbytes = 2 * payload + guards                # source read, payload written, guards written
+    avg = float(np.mean(ms))
+    gbs = nbytes / (avg / 1e3) / 1e9
+    traffic, _ = kernel_traffic("copy", args.workload)
+    del snap
+    return {"kernel": "copy_kernel", "regions": len(specs), "avg_launch_ms": round(avg, 4),
+            "algorithmic_bytes_per_launch": nbytes, "gbs": round(gbs, 1),
+            "hbm_frac": round(gbs / peak, 4), "traffic": traffic,
+            "peak_kind": "measured copy bandwidth (read + write bytes)"}
 
 
 def run_e2e(setup, args, device, world, barrier):
@@ -542,6 +582,7 @@ def main():
     ap.add_argument("--no-e2e", dest="e2e", action="store_false")
     ap.add_argument("--no-cpu", dest="cpu", action="store_false")
     ap.add_argument("--no-eq", dest="eq", action="store_false")
+    ap.add_argument("--no-restore", dest="restore", action="store_false")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     import __graft_entry__
