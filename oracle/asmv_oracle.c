@@ -39,6 +39,16 @@
  *      |int(c) - int(r)| and rel error abs/|r| (same r == 0 rule).
  *   R7 first_mismatch is the lowest element index; first_guard_bad the lowest
  *      byte offset from the allocation start (low guard before high guard).
+ *   R10 Further stored formats (for captured state of other producers):
+ *      OCP FP8 E5M2 (bias 15, Inf and NaN at exponent 31); the "fnuz" FP8
+ *      formats E4M3FNUZ (bias 8) and E5M2FNUZ (bias 16), finite only, no
+ *      negative zero, 0x80 the only NaN; IEEE binary64; int16 and int64.
+ *      Encoding from fp32 rounds to nearest even and saturates finite
+ *      overflow and infinities at the largest finite value (fnuz results of
+ *      magnitude zero are +0); binary64 values are the exact widening of
+ *      the fp32 value.  For binary64, d = RN64(|c - r|) is one rounded
+ *      subtraction.  For int64, |c - r| is formed exactly and rounded once
+ *      to fp64, and rel = RN64(that / RN64(|r|)).
  *
  * Parity pins live in tests/test_oracle_*.py.  The stats of the large
  * perturbed workloads (attention outputs, the 4096-region snapshot, the
@@ -52,20 +62,26 @@
 
 /* ---- dtype and distribution codes (the numbering of the public ABI) ---- */
 enum { OD_F32 = 0, OD_BF16 = 1, OD_F16 = 2, OD_F8E4M3 = 3, OD_I32 = 4,
-       OD_I8 = 5, OD_U8 = 6, OD_NDTYPES = 7 };
+       OD_I8 = 5, OD_U8 = 6, OD_F8E5M2 = 7, OD_F8E4M3FNUZ = 8,
+       OD_F8E5M2FNUZ = 9, OD_F64 = 10, OD_I16 = 11, OD_I64 = 12,
+       OD_NDTYPES = 13 };
 enum { OX_RAW = 0, OX_UNIFORM = 1, OX_NORMAL = 2, OX_INT_RANGE = 3,
        OX_NONE = 4 };
 
 int oracle_dtype_size(int dt) {
   switch (dt) {
     case OD_F32: case OD_I32: return 4;
-    case OD_BF16: case OD_F16: return 2;
-    case OD_F8E4M3: case OD_I8: case OD_U8: return 1;
+    case OD_BF16: case OD_F16: case OD_I16: return 2;
+    case OD_F8E4M3: case OD_I8: case OD_U8: case OD_F8E5M2: case OD_F8E4M3FNUZ:
+    case OD_F8E5M2FNUZ: return 1;
+    case OD_F64: case OD_I64: return 8;
     default: return 0;
   }
 }
 
-static int is_float_dtype(int dt) { return dt <= OD_F8E4M3; }
+static int is_float_dtype(int dt) {
+  return dt <= OD_F8E4M3 || (dt >= OD_F8E5M2 && dt <= OD_F64);
+}
 
 /* ======================================================================
  * Philox4x32-10, written from Salmon et al. (SC'11), Sec. 3 / Table 2:
@@ -137,6 +153,34 @@ double oracle_decode_f8e4m3(uint8_t b) {
   return sign ? -v : v;
 }
 
+/* OCP FP8 E5M2: bias 15, the top byte of an IEEE binary16; exponent field
+ * 31 holds Inf (mantissa 0) and NaN. */
+double oracle_decode_f8e5m2(uint8_t b) {
+  int sign = (b >> 7) & 1, ex = (b >> 2) & 31, man = b & 3;
+  double v;
+  if (ex == 31) v = man ? NAN : INFINITY;
+  else if (ex == 0) v = ldexp((double)man, -16);
+  else v = ldexp((double)(4 + man), ex - 17);
+  return sign ? -v : v;
+}
+
+/* The "fnuz" FP8 formats (finite, no negative zero): every exponent field
+ * is finite, and the bit pattern 0x80 (negative zero elsewhere) is the one
+ * NaN.  E4M3FNUZ: bias 8, max 240; E5M2FNUZ: bias 16, max 57344. */
+double oracle_decode_f8e4m3fnuz(uint8_t b) {
+  if (b == 0x80u) return NAN;
+  int sign = (b >> 7) & 1, ex = (b >> 3) & 15, man = b & 7;
+  double v = (ex == 0) ? ldexp((double)man, -10) : ldexp((double)(8 + man), ex - 11);
+  return sign ? -v : v;
+}
+
+double oracle_decode_f8e5m2fnuz(uint8_t b) {
+  if (b == 0x80u) return NAN;
+  int sign = (b >> 7) & 1, ex = (b >> 2) & 31, man = b & 3;
+  double v = (ex == 0) ? ldexp((double)man, -17) : ldexp((double)(4 + man), ex - 18);
+  return sign ? -v : v;
+}
+
 /* Decode element i of a payload of dtype dt to fp64.  Integer types give
  * their (signed or unsigned) integer value. */
 static double decode_elem(const uint8_t *p, int dt, uint64_t i) {
@@ -148,6 +192,12 @@ static double decode_elem(const uint8_t *p, int dt, uint64_t i) {
     case OD_I32: { int32_t v; memcpy(&v, p + 4 * i, 4); return (double)v; }
     case OD_I8: return (double)(int8_t)p[i];
     case OD_U8: return (double)p[i];
+    case OD_F8E5M2: return oracle_decode_f8e5m2(p[i]);
+    case OD_F8E4M3FNUZ: return oracle_decode_f8e4m3fnuz(p[i]);
+    case OD_F8E5M2FNUZ: return oracle_decode_f8e5m2fnuz(p[i]);
+    case OD_F64: { double d; memcpy(&d, p + 8 * i, 8); return d; }
+    case OD_I16: { int16_t v; memcpy(&v, p + 2 * i, 2); return (double)v; }
+    case OD_I64: { int64_t v; memcpy(&v, p + 8 * i, 8); return (double)v; }   /* rounded above 2^53 */
     default: return NAN;
   }
 }
@@ -196,6 +246,49 @@ uint16_t oracle_f32_to_f16(float f) {
   if (e + 15 >= 31) return (uint16_t)(sign | 0x7C00u);
   return (uint16_t)(sign | ((uint32_t)(e + 15) << 10) | (q - 1024));
 }
+
+/* fp32 -> an 8-bit float with `eb` exponent bits, `mb` mantissa bits and
+ * bias `bias`, round to nearest even.  Finite overflow and infinities
+ * saturate to the largest finite value `maxmag` (its bit pattern without
+ * sign).  fnuz formats have no negative zero (a result of magnitude zero is
+ * +0) and encode NaN as 0x80; the others keep the sign of zero and encode
+ * NaN as S.1..1 with every mantissa bit set. */
+static uint8_t encode_fp8(float f, int eb, int mb, int bias, uint8_t maxmag, int fnuz) {
+  uint32_t u = f32_bits(f);
+  uint8_t sign = (uint8_t)((u >> 24) & 0x80u);
+  uint32_t a = u & 0x7FFFFFFFu;
+  if (a > 0x7F800000u) return fnuz ? 0x80u : (uint8_t)(sign | 0x7Fu);
+  uint8_t mag;
+  if (a == 0x7F800000u) {
+    mag = maxmag;
+  } else {
+    uint32_t bexp = a >> 23, frac = a & 0x7FFFFFu;
+    int e = (bexp == 0) ? -126 : (int)bexp - 127;
+    int emin = 1 - bias;                             /* exponent of the least normal */
+    int qmin = emin - mb;                            /* quantum of the subnormals */
+    if (e < qmin - 1) {
+      mag = 0;                                       /* below half the least subnormal */
+    } else {
+      int qe = (e - mb > qmin) ? e - mb : qmin;
+      uint32_t q = rne_to_quantum(bexp, frac, qe);
+      uint32_t field;
+      if (qe == qmin) {
+        field = q;                                   /* subnormal, or rounds up to the least normal */
+      } else {
+        if (q == (2u << mb)) { q = 1u << mb; e += 1; }
+        int ef = e + bias;
+        field = (ef > (1 << eb) - 1) ? 0xFFu : (((uint32_t)ef << mb) | (q - (1u << mb)));
+      }
+      mag = (field > maxmag) ? maxmag : (uint8_t)field;
+    }
+  }
+  if (fnuz && mag == 0) return 0;
+  return (uint8_t)(sign | mag);
+}
+
+uint8_t oracle_f32_to_f8e5m2(float f) { return encode_fp8(f, 5, 2, 15, 0x7Bu, 0); }
+uint8_t oracle_f32_to_f8e4m3fnuz(float f) { return encode_fp8(f, 4, 3, 8, 0x7Fu, 1); }
+uint8_t oracle_f32_to_f8e5m2fnuz(float f) { return encode_fp8(f, 5, 2, 16, 0x7Fu, 1); }
 
 /* fp32 -> OCP E4M3: RNE, finite overflow and infinities saturate to +-448,
  * NaN maps to S.1111.111. */
@@ -352,6 +445,10 @@ static void store_float(uint8_t *p, int dt, uint64_t i, float v) {
     case OD_BF16: { uint16_t h = oracle_f32_to_bf16(v); memcpy(p + 2 * i, &h, 2); break; }
     case OD_F16: { uint16_t h = oracle_f32_to_f16(v); memcpy(p + 2 * i, &h, 2); break; }
     case OD_F8E4M3: p[i] = oracle_f32_to_f8e4m3(v); break;
+    case OD_F8E5M2: p[i] = oracle_f32_to_f8e5m2(v); break;
+    case OD_F8E4M3FNUZ: p[i] = oracle_f32_to_f8e4m3fnuz(v); break;
+    case OD_F8E5M2FNUZ: p[i] = oracle_f32_to_f8e5m2fnuz(v); break;
+    case OD_F64: { double d = (double)v; memcpy(p + 8 * i, &d, 8); break; }   /* exact */
   }
 }
 
@@ -359,6 +456,8 @@ static void store_int(uint8_t *p, int dt, uint64_t i, int64_t v) {
   switch (dt) {
     case OD_I32: { int32_t x = (int32_t)v; memcpy(p + 4 * i, &x, 4); break; }
     case OD_I8: case OD_U8: p[i] = (uint8_t)v; break;
+    case OD_I16: { int16_t x = (int16_t)v; memcpy(p + 2 * i, &x, 2); break; }
+    case OD_I64: memcpy(p + 8 * i, &v, 8); break;
   }
 }
 
@@ -466,7 +565,18 @@ void oracle_compare_range(const uint8_t *ref, const uint8_t *cand, int dt,
     int mismatch;
     double abs_err = 0.0, rel_err = 0.0;
     int finite_pair = 1;
-    if (!is_float_dtype(dt)) {
+    if (!is_float_dtype(dt) && dt == OD_I64) {
+      /* |c - r| formed exactly in 128 bits, then rounded once; |r| rounded once */
+      int64_t r, c;
+      memcpy(&r, ref + 8 * i, 8);
+      memcpy(&c, cand + 8 * i, 8);
+      mismatch = r != c;
+      __int128 dd = (__int128)c - (__int128)r;
+      if (dd < 0) dd = -dd;
+      abs_err = (double)(unsigned __int128)dd;
+      if (r != 0) rel_err = abs_err / fabs((double)r);
+      else rel_err = (abs_err == 0.0) ? 0.0 : INFINITY;
+    } else if (!is_float_dtype(dt)) {
       mismatch = memcmp(ref + (uint64_t)sz * i, cand + (uint64_t)sz * i, (size_t)sz) != 0;
       double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);
       abs_err = fabs(c - r);                         /* exact: |c - r| < 2^33 */
@@ -564,7 +674,8 @@ void oracle_restore_region(uint8_t *alloc, uint64_t payload_bytes, uint32_t glo,
  *      digits, digit k weighing 2^(32 k + OEQ_BASE).  The final rounding is
  *      done by the caller from the digits.
  * The range covers every product of two fp32 values (2^-298 .. 2^256) with
- * 2^64 of headroom for the sum.
+ * 2^64 of headroom for the sum.  Binary64 regions have no exact sums here
+ * (their products need 106 bits): they return zeros.
  * ====================================================================== */
 #define OEQ_DIGITS 20
 #define OEQ_BASE (-320)
@@ -606,7 +717,7 @@ void oracle_eq_sums_range(const uint8_t *ref, const uint8_t *cand, int dt,
                           uint64_t i0, uint64_t i1, int64_t *out) {
   int64_t *rc = out, *rr = out + OEQ_DIGITS, *cc = out + 2 * OEQ_DIGITS;
   for (int k = 0; k < 3 * OEQ_DIGITS; ++k) out[k] = 0;
-  if (!is_float_dtype(dt)) return;
+  if (!is_float_dtype(dt) || dt == OD_F64) return;   /* fp64 products are not exact in fp64 */
   uint64_t since = 0;
   for (uint64_t i = i0; i < i1; ++i) {
     double r = decode_elem(ref, dt, i), c = decode_elem(cand, dt, i);

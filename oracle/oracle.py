@@ -18,13 +18,17 @@ import numpy as np
 from . import build as _build
 
 F32, BF16, F16, F8E4M3, I32, I8, U8 = range(7)
+F8E5M2, F8E4M3FNUZ, F8E5M2FNUZ, F64, I16, I64 = range(7, 13)
+NDTYPES = 13
 RAW, UNIFORM, NORMAL, INT_RANGE, NONE = range(5)
-DTYPE_SIZE = {F32: 4, BF16: 2, F16: 2, F8E4M3: 1, I32: 4, I8: 1, U8: 1}
-FLOAT_DTYPES = (F32, BF16, F16, F8E4M3)
+DTYPE_SIZE = {F32: 4, BF16: 2, F16: 2, F8E4M3: 1, I32: 4, I8: 1, U8: 1, F8E5M2: 1,
+              F8E4M3FNUZ: 1, F8E5M2FNUZ: 1, F64: 8, I16: 2, I64: 8}
+FLOAT_DTYPES = (F32, BF16, F16, F8E4M3, F8E5M2, F8E4M3FNUZ, F8E5M2FNUZ, F64)
 U64_NONE = (1 << 64) - 1
 # codes by the names the workload descriptions use
 CODE_OF_DTYPE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32,
-                 "i8": I8, "u8": U8}
+                 "i8": I8, "u8": U8, "f8e5m2": F8E5M2, "f8e4m3fnuz": F8E4M3FNUZ,
+                 "f8e5m2fnuz": F8E5M2FNUZ, "f64": F64, "i16": I16, "i64": I64}
 CODE_OF_DIST = {"raw": RAW, "uniform": UNIFORM, "normal": NORMAL, "int_range": INT_RANGE,
                 "none": NONE}
 
@@ -344,7 +348,10 @@ def eq_cos(s_rc, s_rr, s_cc):
 
 
 def eq_sums(ref_payload, cand_payload, dtype, n_elems, threads=1):
-    """The three sums of one float region, each exact then rounded to fp64."""
+    """The three sums of one float region, each exact then rounded to fp64
+    (not defined for binary64 regions)."""
+    if dtype == F64:
+        raise ValueError("Eq. 1 sums are not defined here for binary64 regions")
     spans = _split(n_elems, threads)
     parts = [None] * len(spans)
 
@@ -363,7 +370,7 @@ def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
     pairs and fails on any NaN/Inf-position mismatch.  S_rc sums over pairs
     with both values finite, S_rr over finite r, S_cc over finite c.  Integer and opaque
     regions have no cosine (NaN) and pass the two float terms."""
-    flt = dtype in (F32, BF16, F16, F8E4M3)
+    flt = dtype in FLOAT_DTYPES
     out = dict(sums) if flt else {"sum_rc": 0.0, "sum_rr": 0.0, "sum_cc": 0.0}
     out["cos"] = eq_cos(out["sum_rc"], out["sum_rr"], out["sum_cc"]) if flt else float("nan")
     flags = 0

@@ -20,7 +20,8 @@ from oracle import oracle as O
 
 PIN_MODULES = ("tests.test_oracle_codecs", "tests.test_oracle_philox",
                "tests.test_oracle_fill", "tests.test_oracle_compare",
-               "tests.test_oracle_eq", "tests.test_oracle_boxmuller")
+               "tests.test_oracle_eq", "tests.test_oracle_dtypes", "tests.test_oracle_restore",
+               "tests.test_oracle_boxmuller")
 # pins that take seconds run last, in this order
 EXPENSIVE = ("test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
              "test_ln_u24_all_inputs")
@@ -104,6 +105,17 @@ MUTANTS = [
     ("eq_sign_dropped", "int64_t sg = (p < 0.0) ? -1 : 1;", "int64_t sg = 1;"),
     ("eq_lsb_off_by_one", "int lsb = e - 53;", "int lsb = e - 52;"),
     ("eq_mid_digit_shift", "((m >> (32 - b)) & 0xFFFFFFFFu)", "((m >> (31 - b)) & 0xFFFFFFFFu)"),
+    # further stored formats
+    ("fnuz_negative_zero_kept", "if (fnuz && mag == 0) return 0;", ""),
+    ("e5m2_saturates_to_inf", "encode_fp8(f, 5, 2, 15, 0x7Bu, 0)", "encode_fp8(f, 5, 2, 15, 0x7Cu, 0)"),
+    ("e4m3fnuz_encoder_bias", "encode_fp8(f, 4, 3, 8, 0x7Fu, 1)", "encode_fp8(f, 4, 3, 7, 0x7Fu, 1)"),
+    ("e5m2fnuz_decoder_bias", "ldexp((double)(4 + man), ex - 18)", "ldexp((double)(4 + man), ex - 17)"),
+    ("e4m3fnuz_nan_pattern", "double oracle_decode_f8e4m3fnuz(uint8_t b) {\n  if (b == 0x80u) return NAN;",
+     "double oracle_decode_f8e4m3fnuz(uint8_t b) {\n  if (b == 0xFFu) return NAN;"),
+    ("i64_difference_rounded_late", "abs_err = (double)(unsigned __int128)dd;",
+     "abs_err = fabs((double)c - (double)r);"),
+    ("restore_guards_skipped", "oracle_fill_guards(alloc, payload_bytes, glo, ghi, canary);\n  memcpy",
+     "memcpy"),
 ]
 
 
