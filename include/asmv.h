@@ -41,7 +41,7 @@
 extern "C" {
 #endif
 
-#define ASMV_ABI_VERSION 2
+#define ASMV_ABI_VERSION 3
 
 /* A CUDA stream (the same type as cudaStream_t); NULL is the legacy
  * default stream. */
@@ -57,7 +57,13 @@ typedef enum {
   ASMV_I32 = 4,        /* two's complement int32 */
   ASMV_I8 = 5,         /* two's complement int8 */
   ASMV_U8_OPAQUE = 6,  /* opaque bytes (compared as unsigned 8-bit values) */
-  ASMV_NDTYPES = 7
+  ASMV_F8E5M2 = 7,     /* OCP FP8 E5M2 (bias 15; Inf and NaN at exponent 31; max 57344) */
+  ASMV_F8E4M3FNUZ = 8, /* FP8 E4M3 "fnuz": bias 8, finite, no -0, 0x80 is NaN; max 240 */
+  ASMV_F8E5M2FNUZ = 9, /* FP8 E5M2 "fnuz": bias 16, finite, no -0, 0x80 is NaN; max 57344 */
+  ASMV_F64 = 10,       /* IEEE binary64 */
+  ASMV_I16 = 11,       /* two's complement int16 */
+  ASMV_I64 = 12,       /* two's complement int64 */
+  ASMV_NDTYPES = 13
 } asmv_dtype;
 
 /* Payload distributions of asmv_fill (Sec. 3.4, Tier 1: deterministic
@@ -69,7 +75,9 @@ typedef enum {
  *   UNIFORM   float dtypes: word w = word (i mod 4) of block (i div 4),
  *             f = (w >> 8) * 2^-24, v = p0 + f*(p1 - p0) in fp32 (p0, p1 and
  *             p1 - p0 rounded to fp32 first; multiply then add), then
- *             round-to-nearest-even to the dtype (fp8 saturates to +-448).
+ *             round-to-nearest-even to the dtype (every fp8 format saturates
+ *             at its largest finite value; fnuz formats give +0 for a zero
+ *             result; binary64 is the exact widening of the fp32 value).
  *   NORMAL    float dtypes: Box-Muller on words (0,1) and (2,3) of block
  *             (i div 4): u1 = ((w0 >> 8) + 1) 2^-24, u2 = (w1 >> 8) 2^-24,
  *             z0 = sqrt(-2 ln u1) cos(2 pi u2), z1 = ... sin(2 pi u2);
@@ -78,7 +86,7 @@ typedef enum {
  *             evaluations, so results are bit-reproducible.
  *   INT_RANGE integer dtypes: w as for UNIFORM, v = lo + ((w*(hi-lo)) >> 32)
  *             with lo = p0, hi = p1 (integers; 1 <= hi - lo <= 2^32 and
- *             [lo, hi) inside the dtype's range).
+ *             [lo, hi) inside the dtype's range; for int64 |p0|, |p1| <= 2^53).
  *   NONE      the payload is left untouched; only guard bands are written. */
 typedef enum {
   ASMV_DIST_RAW = 0,
@@ -118,7 +126,9 @@ typedef struct {
 typedef struct {
   uint64_t mismatches;           /* elements failing the check (incl. non-finite) */
   uint64_t first_mismatch;       /* lowest failing element index; UINT64_MAX if none */
-  double max_abs_err;            /* max over finite pairs of |c - r| (exact fp64); 0 if none */
+  double max_abs_err;            /* max over finite pairs of |c - r| (exact fp64; binary64
+                                    pairs: the rounded difference; int64: the exact
+                                    difference rounded once); 0 if none */
   double max_rel_err;            /* max over finite pairs of |c - r| / |r|; r == 0 gives
                                     0 when c == r, else +Inf */
   uint64_t nonfinite_mismatches; /* failing pairs with a NaN or Inf on either side */
@@ -223,9 +233,10 @@ typedef struct {
  * eq_host[j*n + i] the Eq. 1 result of candidate j on region i (k*n entries
  * each, caller-owned).  theta is any finite double; tau a finite double
  * >= 0.  Float regions of more than 2^31 elements are rejected (the exact
- * sums keep per-digit counts below 2^31).  Synchronous.  Errors as
- * asmv_compare_batched, plus EINVAL for a null eq_host, a non-finite theta
- * or tau, a negative tau, or a float region over that size. */
+ * sums keep per-digit counts below 2^31), and so are binary64 regions (the
+ * exact sums here cover formats whose products are exact in fp64).
+ * Synchronous.  Errors as asmv_compare_batched, plus EINVAL for a null
+ * eq_host, a non-finite theta or tau, a negative tau, or such a region. */
 int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
                     size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
                     asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream);

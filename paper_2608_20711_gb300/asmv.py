@@ -19,10 +19,12 @@ LIB_PATH = os.path.join(HERE, "libasmv.so")
 
 # asmv_dtype / asmv_dist codes
 F32, BF16, F16, F8E4M3, I32, I8, U8_OPAQUE = range(7)
-NDTYPES = 7
+F8E5M2, F8E4M3FNUZ, F8E5M2FNUZ, F64, I16, I64 = range(7, 13)
+NDTYPES = 13
 DIST_RAW, DIST_UNIFORM, DIST_NORMAL, DIST_INT_RANGE, DIST_NONE = range(5)
 DTYPE_CODE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32,
-              "i8": I8, "u8": U8_OPAQUE}
+              "i8": I8, "u8": U8_OPAQUE, "f8e5m2": F8E5M2, "f8e4m3fnuz": F8E4M3FNUZ,
+              "f8e5m2fnuz": F8E5M2FNUZ, "f64": F64, "i16": I16, "i64": I64}
 DIST_CODE = {"raw": DIST_RAW, "uniform": DIST_UNIFORM, "normal": DIST_NORMAL,
              "int_range": DIST_INT_RANGE, "none": DIST_NONE}
 OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM = 0, -1, -2, -3, -4

@@ -34,9 +34,10 @@ namespace {
 
 typedef int (*AddrRangeFn)(unsigned long long *base, size_t *size, unsigned long long ptr);
 
-const int kDtypeSize[ASMV_NDTYPES] = {4, 2, 2, 1, 4, 1, 1};
+const int kDtypeSize[ASMV_NDTYPES] = {4, 2, 2, 1, 4, 1, 1, 1, 1, 1, 8, 2, 8};
+static_assert(ASMV_NDTYPES == kNDtypes && ASMV_F64 == kF64 && ASMV_I64 == kI64, "dtype codes");
 
-bool is_float(uint32_t dt) { return dt <= ASMV_F8E4M3; }
+bool is_float(uint32_t dt) { return dt < ASMV_NDTYPES && is_float_dt(dt); }
 
 // ------------------------------------------------------------ validation
 bool region_extent(const asmv_region &r, uint64_t *payload_bytes, uint64_t *total) {
@@ -78,6 +79,8 @@ bool dist_ok(const asmv_region &r) {
       double lo_lim, hi_lim;
       if (r.dtype == ASMV_I32) { lo_lim = -2147483648.0; hi_lim = 2147483648.0; }
       else if (r.dtype == ASMV_I8) { lo_lim = -128.0; hi_lim = 128.0; }
+      else if (r.dtype == ASMV_I16) { lo_lim = -32768.0; hi_lim = 32768.0; }
+      else if (r.dtype == ASMV_I64) { lo_lim = -9007199254740992.0; hi_lim = 9007199254740992.0; }
       else { lo_lim = 0.0; hi_lim = 256.0; }
       return r.p0 >= lo_lim && r.p1 <= hi_lim && (r.p1 - r.p0) <= 4294967296.0;
     }
@@ -108,7 +111,8 @@ int check_table(const asmv_region *regs, size_t n, bool for_fill) {
 
 bool tol_ok(const asmv_tol *tol) {
   if (tol == nullptr) return false;
-  for (int d = 0; d <= ASMV_F8E4M3; ++d) {
+  for (int d = 0; d < ASMV_NDTYPES; ++d) {
+    if (!is_float((uint32_t)d)) continue;
     if (std::isnan(tol[d].atol) || std::isnan(tol[d].rtol)) return false;
     if (tol[d].atol < 0.0 || tol[d].rtol < 0.0) return false;
   }
@@ -633,7 +637,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   p.ntiles = tile;
   p.nregions = (uint32_t)n;
   p.tile_bytes = tile_bytes;
-  for (int d = 0; d < 7; ++d) {
+  for (int d = 0; d < ASMV_NDTYPES; ++d) {
     if (is_float((uint32_t)d) && tol) p.tol[d] = make_tolf(tol[d]);
   }
   cudaError_t e;
@@ -727,7 +731,7 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
     CmpRegion &c = cr[i];
     std::memset(&c, 0, sizeof c);
     c.ref = r.alloc + r.guard_lo;
-    c.bytes = is_float(r.dtype) ? pb : 0;
+    c.bytes = (is_float(r.dtype) && r.dtype != ASMV_F64) ? pb : 0;
     c.tile0 = tile;
     c.dtype = r.dtype;
     bool vec = (c.ref % 16) == 0;
@@ -797,7 +801,9 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
   int rc = check_pairs(ref, cands, k, n);
   if (rc != ASMV_OK) return rc;
   for (size_t i = 0; i < n; ++i)
-    if (is_float(ref[i].dtype) && ref[i].n_elems > ((uint64_t)1 << 31)) return ASMV_EINVAL;
+    if (is_float(ref[i].dtype) &&
+        (ref[i].dtype == ASMV_F64 || ref[i].n_elems > ((uint64_t)1 << 31)))
+      return ASMV_EINVAL;
   if (n == 0) return ASMV_OK;
   DeviceScope ds(ctx->device);
   if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);

@@ -97,6 +97,31 @@ __device__ __forceinline__ uint32_t exact_float(float r, float c, Hot &h, const 
   return d > bound ? 1u : 0u;
 }
 
+// Exact fp64 evaluation of one binary64 pair; returns the mismatch bit.
+__device__ __forceinline__ uint32_t exact_double(double r64, double c64, Hot &h, const TolF &t) {
+  const bool rn = isnan(r64), cn = isnan(c64), ri = isinf(r64), ci = isinf(c64);
+  if (rn | cn | ri | ci) {
+    const bool match = (rn && cn) || (ri && ci && (signbit(r64) == signbit(c64)));
+    if (!match) h.nonfin++;
+    return match ? 0u : 1u;
+  }
+  const double d = fabs(__dsub_rn(c64, r64));
+  const double bound = __dadd_rn(t.atol, __dmul_rn(t.rtol, fabs(r64)));
+  h.dabs = umax64(h.dabs, dbits(d));
+  rel_update(h, d, r64);
+  return d > bound ? 1u : 0u;
+}
+
+// Exact evaluation of one differing int64 pair: |c - r| formed in 128 bits
+// (it can reach 2^64 - 1) and rounded once; |r| rounded once.
+__device__ __forceinline__ void exact_int64(long long r, long long c, Hot &h) {
+  const unsigned long long dlo = (c >= r) ? (unsigned long long)c - (unsigned long long)r
+                                          : (unsigned long long)r - (unsigned long long)c;
+  const double d = __ull2double_rn(dlo);               // |c - r| < 2^64 fits the unsigned difference
+  h.dabs = umax64(h.dabs, dbits(d));
+  rel_update(h, d, __ll2double_rn(r));
+}
+
 // Exact evaluation of one differing integer pair (always a mismatch).
 __device__ __forceinline__ void exact_int(int64_t r, int64_t c, Hot &h) {
   const int64_t dd = c - r;
@@ -117,6 +142,13 @@ template <> struct Fmt<kF8> { static constexpr int E = 16; };
 template <> struct Fmt<kI32> { static constexpr int E = 4; };
 template <> struct Fmt<kI8> { static constexpr int E = 16; };
 template <> struct Fmt<kU8> { static constexpr int E = 16; };
+template <> struct Fmt<kF8E5M2> { static constexpr int E = 16; };
+template <> struct Fmt<kF8E4FNUZ> { static constexpr int E = 16; };
+template <> struct Fmt<kF8E5FNUZ> { static constexpr int E = 16; };
+template <> struct Fmt<kF64> { static constexpr int E = 2; };
+template <> struct Fmt<kI16> { static constexpr int E = 8; };
+template <> struct Fmt<kI64> { static constexpr int E = 2; };
+
 
 // Element j of a chunk decoded to fp32 (float dtypes; runtime j).
 template <uint32_t DT>
@@ -125,11 +157,13 @@ __device__ __forceinline__ float elem_f32(const uint4 &v, int j) {
   if (DT == kBF16) return __uint_as_float(((word_of(v, j >> 1) >> (16 * (j & 1))) & 0xFFFFu) << 16);
   if (DT == kF16) return __half2float(__ushort_as_half((unsigned short)(word_of(v, j >> 1) >> (16 * (j & 1)))));
   const uint32_t b = (word_of(v, j >> 2) >> (8 * (j & 3))) & 0xFFu;
-  return f8x2_to_f32(b).x;
+  return f16x2_to_f32(fp8x2_to_half2_bits<DT>(b)).x;
 }
 
 template <uint32_t DT>
 __device__ __forceinline__ int64_t elem_int(const uint4 &v, int j) {
+  if (DT == kI64) return (int64_t)(((unsigned long long)word_of(v, 2 * j + 1) << 32) | word_of(v, 2 * j));
+  if (DT == kI16) return (int64_t)(int16_t)(word_of(v, j >> 1) >> (16 * (j & 1)));
   if (DT == kI32) return (int64_t)(int32_t)word_of(v, j);
   const uint32_t b = (word_of(v, j >> 2) >> (8 * (j & 3))) & 0xFFu;
   if (DT == kI8) return (int64_t)(int8_t)b;
@@ -138,8 +172,11 @@ __device__ __forceinline__ int64_t elem_int(const uint4 &v, int j) {
 
 template <uint32_t DT>
 __device__ __forceinline__ uint32_t elem_bits(const uint4 &v, int j) {
-  if (DT == kI32 || DT == kI8 || DT == kU8) return (uint32_t)(int32_t)elem_int<DT>(v, j);
   return __float_as_uint(elem_f32<DT>(v, j));
+}
+
+template <uint32_t DT> __device__ __forceinline__ constexpr bool is_int_dt() {
+  return DT == kI32 || DT == kI8 || DT == kU8 || DT == kI16 || DT == kI64;
 }
 
 // Chunks the screen cannot settle are queued per warp in shared memory and
@@ -183,9 +220,18 @@ __device__ __forceinline__ void settle_chunk(const QEntry &e, Hot &h, const TolF
   uint32_t bad = 0;
 #pragma unroll 1
   for (int j = 0; j < E; ++j) {
-    if (DT == kI32 || DT == kI8 || DT == kU8) {
+    if (DT == kI64) {
+      const int64_t r = elem_int<DT>(e.R, j), c = elem_int<DT>(e.C, j);
+      if (r != c) { exact_int64(r, c, h); bad |= 1u << j; }
+    } else if (is_int_dt<DT>()) {
       const int64_t r = elem_int<DT>(e.R, j), c = elem_int<DT>(e.C, j);
       if (r != c) { exact_int(r, c, h); bad |= 1u << j; }
+    } else if (DT == kF64) {
+      const unsigned long long rb = ((unsigned long long)word_of(e.R, 2 * j + 1) << 32) | word_of(e.R, 2 * j);
+      const unsigned long long cb = ((unsigned long long)word_of(e.C, 2 * j + 1) << 32) | word_of(e.C, 2 * j);
+      if (rb != cb)
+        bad |= exact_double(__longlong_as_double((long long)rb), __longlong_as_double((long long)cb), h,
+                            t) << j;
     } else {
       const uint32_t rb = elem_bits<DT>(e.R, j), cb = elem_bits<DT>(e.C, j);
       if (rb != cb) bad |= settle_float(__uint_as_float(rb), __uint_as_float(cb), h, t) << j;
@@ -260,8 +306,8 @@ template <uint32_t DT>
 __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e0, Hot &h,
                                       const TolF &t, Queue *q) {
   if (R.x == C.x && R.y == C.y && R.z == C.z && R.w == C.w) return;
-  if (DT == kI32 || DT == kI8 || DT == kU8) {
-    push_chunk<DT>(R, C, e0, q, h, t);          // integer differences are evaluated exactly
+  if (is_int_dt<DT>() || DT == kF64) {
+    push_chunk<DT>(R, C, e0, q, h, t);          // integer and binary64 differences are evaluated exactly
     return;
   }
   const float Tp = fminf(h.T, ASMV_HALF_LESS);
@@ -304,12 +350,8 @@ __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e
       uint32_t rw, cw;
       if (DT == kF16) { rw = word_of(R, w); cw = word_of(C, w); }
       else {
-        const __half2_raw rh = __nv_cvt_fp8x2_to_halfraw2(
-            (__nv_fp8x2_storage_t)((word_of(R, w >> 1) >> (16 * (w & 1))) & 0xFFFFu), __NV_E4M3);
-        const __half2_raw ch = __nv_cvt_fp8x2_to_halfraw2(
-            (__nv_fp8x2_storage_t)((word_of(C, w >> 1) >> (16 * (w & 1))) & 0xFFFFu), __NV_E4M3);
-        rw = (uint32_t)rh.x | ((uint32_t)rh.y << 16);
-        cw = (uint32_t)ch.x | ((uint32_t)ch.y << 16);
+        rw = fp8x2_to_half2_bits<DT>(word_of(R, w >> 1) >> (16 * (w & 1)));
+        cw = fp8x2_to_half2_bits<DT>(word_of(C, w >> 1) >> (16 * (w & 1)));
       }
       const __half2 s2 = __hsub2(*reinterpret_cast<const __half2 *>(&cw),
                                  *reinterpret_cast<const __half2 *>(&rw));
@@ -518,6 +560,12 @@ __device__ __forceinline__ Hot run_dispatch(const CmpParams &p, const CmpRegion 
     case kF8: return ASMV_RUN(kF8, p.tol[kF8]);
     case kI32: return ASMV_RUN(kI32, p.tol[0]);
     case kI8: return ASMV_RUN(kI8, p.tol[0]);
+    case kF8E5M2: return ASMV_RUN(kF8E5M2, p.tol[kF8E5M2]);
+    case kF8E4FNUZ: return ASMV_RUN(kF8E4FNUZ, p.tol[kF8E4FNUZ]);
+    case kF8E5FNUZ: return ASMV_RUN(kF8E5FNUZ, p.tol[kF8E5FNUZ]);
+    case kF64: return ASMV_RUN(kF64, p.tol[kF64]);
+    case kI16: return ASMV_RUN(kI16, p.tol[0]);
+    case kI64: return ASMV_RUN(kI64, p.tol[0]);
     default: return ASMV_RUN(kU8, p.tol[0]);
   }
 #undef ASMV_RUN

@@ -131,6 +131,45 @@ __device__ __forceinline__ uint32_t pack_f8x4(float a, float b, float c, float d
   return (lo & 0xFFFFu) | (hi << 16);
 }
 
+// OCP E5M2: hardware conversion, saturating at +-57344.
+__device__ __forceinline__ uint32_t pack_e5m2x4(float a, float b, float c, float d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E5M2);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c, d), __NV_SATFINITE, __NV_E5M2);
+  return (lo & 0xFFFFu) | (hi << 16);
+}
+
+// The fnuz formats hold half the value of the OCP format with the same bits
+// (bias one higher), except that they are finite at the top exponent, have
+// no negative zero and keep 0x80 for NaN.  So x is converted as 2x by the
+// hardware (round to nearest even), then:
+//   NaN -> 0x80; a zero result -> +0;
+//   E4M3FNUZ: above 232 (halfway between 224 and the top value 240) -> 240
+//     (0x7F, a NaN in the OCP format);
+//   E5M2FNUZ: from 30720 (halfway between 28672 and 32768) the top binade
+//     (4..7) * 8192 is chosen directly, nearest with ties to even, capped at
+//     57344 -- values the OCP format holds as Inf and NaN.
+__device__ __forceinline__ uint32_t enc_e4m3fnuz(float x) {
+  const float ax = fabsf(x);
+  const uint32_t sign = (__float_as_uint(x) >> 24) & 0x80u;
+  if (isnan(x)) return 0x80u;
+  if (ax > 232.0f) return sign | 0x7Fu;
+  const uint32_t b =
+      __nv_cvt_float2_to_fp8x2(make_float2(__fmul_rn(x, 2.0f), 0.0f), __NV_SATFINITE, __NV_E4M3) & 0xFFu;
+  return (b & 0x7Fu) ? b : 0u;
+}
+__device__ __forceinline__ uint32_t enc_e5m2fnuz(float x) {
+  const float ax = fabsf(x);
+  const uint32_t sign = (__float_as_uint(x) >> 24) & 0x80u;
+  if (isnan(x)) return 0x80u;
+  if (ax >= 30720.0f) {
+    const int q = min(__float2int_rn(__fmul_rn(fminf(ax, 1e9f), 0x1p-13f)), 7);
+    return sign | 0x7Cu | (uint32_t)(q - 4);
+  }
+  const uint32_t b =
+      __nv_cvt_float2_to_fp8x2(make_float2(__fmul_rn(x, 2.0f), 0.0f), __NV_SATFINITE, __NV_E5M2) & 0xFFu;
+  return (b & 0x7Fu) ? b : 0u;
+}
+
 // ---------------------------------------------------------------- decoders
 __device__ __forceinline__ float2 f16x2_to_f32(uint32_t w) {
   return __half22float2(*reinterpret_cast<const __half2 *>(&w));
@@ -139,6 +178,29 @@ __device__ __forceinline__ float2 f8x2_to_f32(uint32_t w16) {
   const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(w16 & 0xFFFFu), __NV_E4M3);
   uint32_t u = (uint32_t)h.x | ((uint32_t)h.y << 16);
   return f16x2_to_f32(u);
+}
+
+// Two fp8 values (low byte first) as an exact half2, per format.  The fnuz
+// formats are half the value of the OCP format with the same bits, finite
+// at the top exponent (E4M3: 0x7F is 240; E5M2: exponent 31 holds
+// (4..7) * 8192), with 0x80 the NaN.
+__device__ __forceinline__ uint32_t half_bits_fnuz(uint32_t b, uint32_t hw, bool e5) {
+  const uint32_t sign = (b & 0x80u) << 8;
+  if (b == 0x80u) return 0x7E00u;
+  if (!e5 && (b & 0x7Fu) == 0x7Fu) return sign | 0x5B80u;                   // 240
+  if (e5 && (b & 0x7Cu) == 0x7Cu) return sign | 0x7800u | ((b & 3u) << 8);  // (4+m) 2^13
+  const __half h = __hmul(__ushort_as_half((unsigned short)hw), __float2half(0.5f));
+  return (uint32_t)__half_as_ushort(h);
+}
+
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t fp8x2_to_half2_bits(uint32_t w16) {
+  const __nv_fp8x2_storage_t s = (__nv_fp8x2_storage_t)(w16 & 0xFFFFu);
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(
+      s, (DT == kF8 || DT == kF8E4FNUZ) ? __NV_E4M3 : __NV_E5M2);
+  if (DT == kF8 || DT == kF8E5M2) return (uint32_t)h.x | ((uint32_t)h.y << 16);
+  const bool e5 = DT == kF8E5FNUZ;
+  return half_bits_fnuz(w16 & 0xFFu, h.x, e5) | (half_bits_fnuz((w16 >> 8) & 0xFFu, h.y, e5) << 16);
 }
 
 // ---------------------------------------------------------------- integers

@@ -333,9 +333,15 @@ __device__ __forceinline__ uint32_t byte_of(const uint4 &v, int k) {
   const uint32_t w = k < 4 ? v.x : k < 8 ? v.y : k < 12 ? v.z : v.w;
   return (w >> (8 * (k & 3))) & 0xFFu;
 }
+// Element k of a chunk of E5M2 / fnuz fp8 as the bits of its exact fp16 value.
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t fp8_half(const uint4 &v, int k) {
+  return fp8x2_to_half2_bits<DT>(byte_of(v, k)) & 0xFFFFu;
+}
 
 // One tile of an fp16 or fp8 region: S_rr once, then the candidates two at
-// a time (the reference chunk is decoded once per pair).
+// a time (the reference chunk is decoded once per pair).  E5M2 and the fnuz
+// formats go through their exact fp16 values (and fp16's binary point).
 template <int DT>
 __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R, uint32_t region,
                                            uint64_t a, uint32_t nb, long long *sdig) {
@@ -357,12 +363,15 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
       if (DT == kF16) {
 #pragma unroll
         for (int k = 0; k < 8; ++k) sq(rr, fix_f16(half_of(rv, k)));
+      } else if (DT != kF8) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) sq(rr, fix_f16(fp8_half<DT>(rv, k)));
       } else {
 #pragma unroll
         for (int k = 0; k < 16; ++k) { const int x = fix_f8(byte_of(rv, k)); r8 = mad_wide(x, x, r8); }
       }
     }
-    if (DT == kF16) flush3(rr, sdig); else flush1(r8, sdig);
+    if (DT != kF8) flush3(rr, sdig); else flush1(r8, sdig);
   }
   for (uint32_t j = 0; j < p.K; j += 2) {
     const bool two = j + 1 < p.K;                    // uniform
@@ -389,6 +398,15 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
           mac(rc0, x, y0); sq(cc0, y0);
           mac(rc1, x, y1); sq(cc1, y1);
         }
+      } else if (DT != kF8) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const Limbs x = fix_f16(fp8_half<DT>(rv, k));
+          const Limbs y0 = fix_f16(fp8_half<DT>(v0, k));
+          const Limbs y1 = fix_f16(fp8_half<DT>(v1, k));
+          mac(rc0, x, y0); sq(cc0, y0);
+          mac(rc1, x, y1); sq(cc1, y1);
+        }
       } else {
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -399,7 +417,7 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
         }
       }
     }
-    if (DT == kF16) {
+    if (DT != kF8) {
       flush3(rc0, sdig + (1 + 2 * j) * kWin);
       flush3(cc0, sdig + (2 + 2 * j) * kWin);
       if (two) { flush3(rc1, sdig + (3 + 2 * j) * kWin); flush3(cc1, sdig + (4 + 2 * j) * kWin); }
@@ -415,7 +433,7 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
 __device__ void cta_flush(const EqParams &p, uint32_t region, uint32_t dtype, long long *sdig) {
   __syncthreads();
   const int dig0 = dtype == kF32 ? Fmt<kF32>::kDig : dtype == kBF16 ? Fmt<kBF16>::kDig
-                 : dtype == kF16 ? Fmt<kF16>::kDig : Fmt<kF8>::kDig;
+                 : dtype == kF8 ? Fmt<kF8>::kDig : Fmt<kF16>::kDig;   // other fp8: fp16's point
   const uint32_t nloc = 1u + 2u * p.K;
   for (uint32_t x = threadIdx.x; x < nloc * kWin; x += blockDim.x) {
     const long long v = sdig[x];
@@ -451,6 +469,9 @@ __global__ void __launch_bounds__(kThreads) eq_kernel(EqParams p) {
       case kF32: eq_tile<kF32>(p, R, i, a, nb, sdig); break;
       case kBF16: eq_tile<kBF16>(p, R, i, a, nb, sdig); break;
       case kF16: eq_tile_fixed<kF16>(p, R, i, a, nb, sdig); break;
+      case kF8E5M2: eq_tile_fixed<kF8E5M2>(p, R, i, a, nb, sdig); break;
+      case kF8E4FNUZ: eq_tile_fixed<kF8E4FNUZ>(p, R, i, a, nb, sdig); break;
+      case kF8E5FNUZ: eq_tile_fixed<kF8E5FNUZ>(p, R, i, a, nb, sdig); break;
       default: eq_tile_fixed<kF8>(p, R, i, a, nb, sdig); break;
     }
   }

@@ -63,6 +63,24 @@ template <uint32_t DIST, uint32_t DT>
 __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, uint64_t c) {
   if (DIST == kRaw) return payload_block(K, r.region_id, c);
   if (DIST == kIntRange) {
+    if (DT == kI64) {                           // 2 elements: words 2(c mod 2), +1 of block c/2
+      const uint4 w = payload_block(K, r.region_id, c >> 1);
+      const uint32_t wa = (c & 1) ? w.z : w.x, wb = (c & 1) ? w.w : w.y;
+      const int64_t a = r.ilo + (int64_t)(((uint64_t)wa * r.ispan) >> 32);
+      const int64_t b = r.ilo + (int64_t)(((uint64_t)wb * r.ispan) >> 32);
+      return make_uint4((uint32_t)a, (uint32_t)((uint64_t)a >> 32), (uint32_t)b,
+                        (uint32_t)((uint64_t)b >> 32));
+    }
+    if (DT == kI16) {                           // 8 elements: blocks 2c, 2c+1
+      uint32_t out[4];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint4 w = payload_block(K, r.region_id, 2 * c + q);
+        out[2 * q] = (int_of(w.x, r.ilo, r.ispan) & 0xFFFFu) | (int_of(w.y, r.ilo, r.ispan) << 16);
+        out[2 * q + 1] = (int_of(w.z, r.ilo, r.ispan) & 0xFFFFu) | (int_of(w.w, r.ilo, r.ispan) << 16);
+      }
+      return make_uint4(out[0], out[1], out[2], out[3]);
+    }
     if (DT == kI32) {
       const uint4 w = payload_block(K, r.region_id, c);
       return make_uint4(int_of(w.x, r.ilo, r.ispan), int_of(w.y, r.ilo, r.ispan),
@@ -79,6 +97,23 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     }
   }
   // UNIFORM / NORMAL on float dtypes
+  if (DT == kF64) {                             // 2 elements: words 2(c mod 2), +1 of block c/2
+    const uint4 w = payload_block(K, r.region_id, c >> 1);
+    float v0, v1;
+    if (DIST == kNormal) {
+      float z0, z1;
+      if (c & 1) box_muller(w.z, w.w, K.lntab, z0, z1);
+      else box_muller(w.x, w.y, K.lntab, z0, z1);
+      v0 = __fadd_rn(r.f0, __fmul_rn(r.f1, z0));
+      v1 = __fadd_rn(r.f0, __fmul_rn(r.f1, z1));
+    } else {
+      v0 = uniform_of((c & 1) ? w.z : w.x, r.f0, r.f1);
+      v1 = uniform_of((c & 1) ? w.w : w.y, r.f0, r.f1);
+    }
+    const unsigned long long a = (unsigned long long)__double_as_longlong((double)v0);
+    const unsigned long long b = (unsigned long long)__double_as_longlong((double)v1);
+    return make_uint4((uint32_t)a, (uint32_t)(a >> 32), (uint32_t)b, (uint32_t)(b >> 32));
+  }
   if (DT == kF32) {
     float v[4];
     float4_of<DIST>(payload_block(K, r.region_id, c), r, K, v);
@@ -100,7 +135,14 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     for (int q = 0; q < 4; ++q) {
       float v[4];
       float4_of<DIST>(payload_block(K, r.region_id, 4 * c + q), r, K, v);
-      out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
+      if (DT == kF8) out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
+      else if (DT == kF8E5M2) out[q] = pack_e5m2x4(v[0], v[1], v[2], v[3]);
+      else if (DT == kF8E4FNUZ)
+        out[q] = enc_e4m3fnuz(v[0]) | (enc_e4m3fnuz(v[1]) << 8) | (enc_e4m3fnuz(v[2]) << 16) |
+                 (enc_e4m3fnuz(v[3]) << 24);
+      else
+        out[q] = enc_e5m2fnuz(v[0]) | (enc_e5m2fnuz(v[1]) << 8) | (enc_e5m2fnuz(v[2]) << 16) |
+                 (enc_e5m2fnuz(v[3]) << 24);
     }
     return make_uint4(out[0], out[1], out[2], out[3]);
   }
@@ -125,14 +167,22 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
   switch (r.dist) {
     case kRaw: fill_tile<kRaw, kU8>(r, K, t); break;
     case kIntRange:
-      if (r.dtype == kI32) fill_tile<kIntRange, kI32>(r, K, t);
-      else fill_tile<kIntRange, kI8>(r, K, t);
+      switch (r.dtype) {
+        case kI32: fill_tile<kIntRange, kI32>(r, K, t); break;
+        case kI16: fill_tile<kIntRange, kI16>(r, K, t); break;
+        case kI64: fill_tile<kIntRange, kI64>(r, K, t); break;
+        default: fill_tile<kIntRange, kI8>(r, K, t); break;
+      }
       break;
     case kUniform:
       switch (r.dtype) {
         case kF32: fill_tile<kUniform, kF32>(r, K, t); break;
         case kBF16: fill_tile<kUniform, kBF16>(r, K, t); break;
         case kF16: fill_tile<kUniform, kF16>(r, K, t); break;
+        case kF8E5M2: fill_tile<kUniform, kF8E5M2>(r, K, t); break;
+        case kF8E4FNUZ: fill_tile<kUniform, kF8E4FNUZ>(r, K, t); break;
+        case kF8E5FNUZ: fill_tile<kUniform, kF8E5FNUZ>(r, K, t); break;
+        case kF64: fill_tile<kUniform, kF64>(r, K, t); break;
         default: fill_tile<kUniform, kF8>(r, K, t); break;
       }
       break;
@@ -141,6 +191,10 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
         case kF32: fill_tile<kNormal, kF32>(r, K, t); break;
         case kBF16: fill_tile<kNormal, kBF16>(r, K, t); break;
         case kF16: fill_tile<kNormal, kF16>(r, K, t); break;
+        case kF8E5M2: fill_tile<kNormal, kF8E5M2>(r, K, t); break;
+        case kF8E4FNUZ: fill_tile<kNormal, kF8E4FNUZ>(r, K, t); break;
+        case kF8E5FNUZ: fill_tile<kNormal, kF8E5FNUZ>(r, K, t); break;
+        case kF64: fill_tile<kNormal, kF64>(r, K, t); break;
         default: fill_tile<kNormal, kF8>(r, K, t); break;
       }
       break;
@@ -148,7 +202,7 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
   }
 }
 
-__global__ void __launch_bounds__(kThreads) fill_kernel(const FillParams p) {
+__global__ void __launch_bounds__(kThreads, 6) fill_kernel(const FillParams p) {
   __shared__ float4 lntab[ASMV_LN_TABLE_ROWS];
   for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS; i += kThreads) lntab[i] = kLnTableInit[i];
   __syncthreads();

@@ -28,7 +28,16 @@ constexpr int kConsumerWarps = 16;      // compare: checking warps per CTA
 constexpr int kStages = 4;              // compare: shared-memory pipeline depth
 constexpr int kCmpThreads = (kConsumerWarps + 1) * 32;   // + one producer warp
 
-enum : uint32_t { kF32 = 0, kBF16 = 1, kF16 = 2, kF8 = 3, kI32 = 4, kI8 = 5, kU8 = 6 };
+enum : uint32_t { kF32 = 0, kBF16 = 1, kF16 = 2, kF8 = 3, kI32 = 4, kI8 = 5, kU8 = 6,
+                  kF8E5M2 = 7, kF8E4FNUZ = 8, kF8E5FNUZ = 9, kF64 = 10, kI16 = 11, kI64 = 12,
+                  kNDtypes = 13 };
+
+__host__ __device__ constexpr bool is_fp8(uint32_t dt) {
+  return dt == kF8 || dt == kF8E5M2 || dt == kF8E4FNUZ || dt == kF8E5FNUZ;
+}
+__host__ __device__ constexpr bool is_float_dt(uint32_t dt) {
+  return dt <= kF8 || (dt >= kF8E5M2 && dt <= kF64);
+}
 enum : uint32_t { kRaw = 0, kUniform = 1, kNormal = 2, kIntRange = 3, kNone = 4 };
 enum : uint32_t { kSegFill = 0, kSegSelf = 1, kSegCand = 2, kSegRef = 3 };
 
@@ -107,7 +116,7 @@ struct CmpParams {
   uint32_t nsegs;
   uint32_t K;
   uint32_t tile_bytes;         // payload bytes per tile (multiple of 16)
-  TolF tol[7];
+  TolF tol[kNDtypes];
 };
 
 // The Eq. 1 sums (eqsum.cu).  Each sum of a region is kept as kEqDigits
@@ -115,8 +124,9 @@ struct CmpParams {
 // digits of one region are [slot][kEqDigits] with slot 0 = S_rr and slots
 // 1 + 2j, 2 + 2j = S_rc, S_cc of candidate j.
 constexpr int kEqDigits = 20;
+// fp8 formats other than E4M3 are summed through their exact fp16 value.
 constexpr int eq_digit_base(uint32_t dtype) {
-  return dtype == kF32 ? -318 : dtype == kBF16 ? -286 : dtype == kF16 ? -112 : -82;
+  return dtype == kF32 ? -318 : dtype == kBF16 ? -286 : dtype == kF8 ? -82 : -112;
 }
 
 struct EqParams {

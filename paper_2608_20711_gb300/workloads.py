@@ -22,14 +22,19 @@ from typing import List, Optional, Sequence
 
 import numpy as np
 
-DTYPES = ("f32", "bf16", "f16", "f8e4m3", "i32", "i8", "u8")
-DTYPE_SIZE = {"f32": 4, "bf16": 2, "f16": 2, "f8e4m3": 1, "i32": 4, "i8": 1, "u8": 1}
-FLOAT_DTYPES = ("f32", "bf16", "f16", "f8e4m3")
+DTYPES = ("f32", "bf16", "f16", "f8e4m3", "i32", "i8", "u8", "f8e5m2", "f8e4m3fnuz",
+          "f8e5m2fnuz", "f64", "i16", "i64")
+DTYPE_SIZE = {"f32": 4, "bf16": 2, "f16": 2, "f8e4m3": 1, "i32": 4, "i8": 1, "u8": 1,
+              "f8e5m2": 1, "f8e4m3fnuz": 1, "f8e5m2fnuz": 1, "f64": 8, "i16": 2, "i64": 8}
+FLOAT_DTYPES = ("f32", "bf16", "f16", "f8e4m3", "f8e5m2", "f8e4m3fnuz", "f8e5m2fnuz", "f64")
 DISTS = ("raw", "uniform", "normal", "int_range", "none")
 
 # largest finite value's bit pattern, per float format (sign-magnitude)
-_MAX_FINITE_BITS = {"f32": 0x7F7FFFFF, "bf16": 0x7F7F, "f16": 0x7BFF, "f8e4m3": 0x7E}
-_BITS = {"f32": 32, "bf16": 16, "f16": 16, "f8e4m3": 8, "i32": 32, "i8": 8, "u8": 8}
+_MAX_FINITE_BITS = {"f32": 0x7F7FFFFF, "bf16": 0x7F7F, "f16": 0x7BFF, "f8e4m3": 0x7E,
+                    "f8e5m2": 0x7B, "f8e4m3fnuz": 0x7F, "f8e5m2fnuz": 0x7F,
+                    "f64": 0x7FEFFFFFFFFFFFFF}
+_BITS = {"f32": 32, "bf16": 16, "f16": 16, "f8e4m3": 8, "i32": 32, "i8": 8, "u8": 8,
+         "f8e5m2": 8, "f8e4m3fnuz": 8, "f8e5m2fnuz": 8, "f64": 64, "i16": 16, "i64": 64}
 
 ARENA_ALIGN = 256
 
@@ -104,6 +109,10 @@ DEFAULT_TOL = {
     "bf16": Tolerance(1e-5, 1.6e-2),
     "f16": Tolerance(1e-5, 1e-3),
     "f8e4m3": Tolerance(1e-5, 0.125),
+    "f8e5m2": Tolerance(1e-5, 0.25),
+    "f8e4m3fnuz": Tolerance(1e-5, 0.125),
+    "f8e5m2fnuz": Tolerance(1e-5, 0.25),
+    "f64": Tolerance(1e-7, 1e-7),
 }
 
 

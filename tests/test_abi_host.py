@@ -62,7 +62,7 @@ def test_region_table_validation():
     ok = dict(alloc=1 << 20, n_elems=100, dtype="f32", dist="uniform", p0=-1.0, p1=1.0,
               guard_lo=64, guard_hi=64)
     assert asmv.check_regions([ok], for_fill=True) == asmv.OK
-    bad = [dict(ok, dtype=9), dict(ok, dist=7), dict(ok, dist="int_range", p0=0, p1=5),
+    bad = [dict(ok, dtype=13), dict(ok, dist=7), dict(ok, dist="int_range", p0=0, p1=5),
            dict(ok, p0=2.0, p1=1.0), dict(ok, n_elems=1 << 62), dict(ok, alloc=0)]
     for b in bad:
         assert asmv.check_regions([b], for_fill=True) == asmv.EINVAL, b
