@@ -190,6 +190,45 @@ def regions_in_arena(specs: Iterable, base: int) -> List[Region]:
                         s.region_id, s.canary, s.p0, s.p1) for s in specs]
 
 
+def strided_regions(base: int, shape: Sequence[int], strides: Sequence[int], dtype,
+                    region_id0: int = 0, canary: int = 0xA5) -> List[Region]:
+    """A non-contiguous tensor (element strides, row-major shape) as one
+    region per contiguous run of its innermost dimension(s): runs are merged
+    while the strides are those of a contiguous block.  Region ids count up
+    from region_id0 in row-major order; no guard bands (the gaps between runs
+    belong to other data)."""
+    shape, strides = list(shape), list(strides)
+    if len(shape) != len(strides) or any(n < 0 for n in shape):
+        raise ValueError("shape and strides must have the same length")
+    code = DTYPE_CODE[dtype] if isinstance(dtype, str) else int(dtype)
+    size = [4, 2, 2, 1, 4, 1, 1, 1, 1, 1, 8, 2, 8][code]
+    if 0 in shape:
+        return []
+    # innermost dimensions that form one contiguous run
+    run, k = 1, len(shape)
+    while k > 0 and strides[k - 1] == run:
+        run *= shape[k - 1]
+        k -= 1
+    if k == len(shape):               # innermost stride not 1: runs of one element
+        run = 1
+    outer = shape[:k]
+    out = []
+    idx = [0] * len(outer)
+    while True:
+        off = sum(i * st for i, st in zip(idx, strides[:k]))
+        out.append(make_region(base + off * size, run, code, "raw", 0, 0,
+                               region_id0 + len(out), canary))
+        d = len(outer) - 1
+        while d >= 0:
+            idx[d] += 1
+            if idx[d] < outer[d]:
+                break
+            idx[d] = 0
+            d -= 1
+        if d < 0:
+            return out
+
+
 def tol_array(tol: Optional[Dict] = None) -> ctypes.Array:
     """Per-dtype tolerances: dict of dtype name/code -> (atol, rtol) or an
     object with .atol/.rtol; unspecified float dtypes get (0, 0)."""

@@ -130,3 +130,24 @@ def test_no_gpu_means_no_context():
     _lib()
     with pytest.raises(asmv.AsmvError):
         asmv.Context(0)
+
+
+def test_strided_regions_cover_each_element_once():
+    """The regions of a strided view cover exactly its elements' bytes."""
+    import numpy as np
+    base = 1 << 30
+    a = np.zeros((6, 10, 12), np.float16)
+    for view in (a, a[:, 2:9, :], a[::2, :, 3:7], a.transpose(1, 0, 2)[:, :, ::3], a[:, :, 5]):
+        strides = [s // a.itemsize for s in view.strides]
+        off0 = (view.__array_interface__["data"][0] - a.__array_interface__["data"][0]) // 2
+        regs = asmv.strided_regions(base + 2 * off0, view.shape, strides, "f16")
+        covered = []
+        for r in regs:
+            start = (r.alloc - base) // 2
+            covered.extend(range(start, start + r.n_elems))
+        idx = np.arange(a.size).reshape(a.shape)
+        # element offsets of the view, in row-major order of the view
+        view_idx = np.lib.stride_tricks.as_strided(idx.ravel()[off0:], view.shape,
+                                                   [s // 2 * 8 for s in view.strides])
+        assert covered == view_idx.ravel().tolist()
+        assert len(regs) <= view.size

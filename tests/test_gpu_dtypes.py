@@ -186,3 +186,32 @@ def test_restore_wide_types(ctx, oracle):
                               snap_h[r.payload_offset:r.payload_offset + r.payload_bytes])
     np.testing.assert_array_equal(to_host(arena), want)
     torch.cuda.synchronize()
+
+
+def test_strided_view_compare(ctx, oracle):
+    """A non-contiguous fp16 view (a slice of a transposed tensor) checked
+    as one region per contiguous run; each run's statistics equal the
+    oracle's on the same bytes."""
+    torch = torch_cuda()
+    g = torch.Generator(device="cpu").manual_seed(3)
+    host = torch.randn(64, 48, 40, generator=g).to(torch.float16)
+    cand = host.clone()
+    cand.view(-1)[::97] += 0.01
+    dref, dcand = host.cuda(), cand.cuda()
+    view_r = dref.transpose(0, 1)[5:40, ::2, 3:29]
+    view_c = dcand.transpose(0, 1)[5:40, ::2, 3:29]
+    regs_r = asmv.strided_regions(view_r.data_ptr(), view_r.shape, view_r.stride(), "f16")
+    regs_c = asmv.strided_regions(view_c.data_ptr(), view_c.shape, view_c.stride(), "f16")
+    assert len(regs_r) == 35 * 32
+    got = ctx.compare(regs_r, regs_c, W.DEFAULT_TOL)
+    hr, hc = host.numpy().view(np.uint8).ravel(), cand.numpy().view(np.uint8).ravel()
+    base_r = dref.data_ptr()
+    t = W.DEFAULT_TOL["f16"]
+    total = 0
+    for r, s in zip(regs_r, got):
+        off = r.alloc - base_r
+        want = oracle.compare_region(hr[off:], 0, 0, 0xA5, hc[off:], 0, 0, 0xA5, r.n_elems,
+                                     ORACLE_DTYPE["f16"], t.atol, t.rtol)
+        assert_stats_equal(s, want)
+        total += want["mismatches"]
+    assert total > 0
