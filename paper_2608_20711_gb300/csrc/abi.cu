@@ -1133,7 +1133,8 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   p.nsegs = (uint32_t)ks;
   p.K = 1;
   p.tile_bytes = tile_bytes;
-  for (int d = 0; d <= ASMV_F8E4M3; ++d) p.tol[d] = make_tolf(tol[d]);
+  for (int d = 0; d < ASMV_NDTYPES; ++d)
+    if (is_float((uint32_t)d)) p.tol[d] = make_tolf(tol[d]);
   const uint64_t per_cta = kConsumerWarps + 1;
   const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(
       std::max<uint64_t>(tile, (ks + per_cta - 1) / per_cta), (uint64_t)g_noalloc_sms[dev]));

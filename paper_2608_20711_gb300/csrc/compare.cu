@@ -30,23 +30,31 @@
 //      maximum of RN64(D).  max_abs = max(m32, that maximum).
 //  (4) max_rel: a thread keeps its exact maximum Rmax and T <= Rmax(1-2^-19)
 //      in fp32.  An element can exceed Rmax only if as > T*|r| (the
-//      relative error of as/|r| against d/|r| is below 2^-23), which
-//      one fma decides exactly in sign; those elements get the exact
-//      RN64(d/|r|).
+//      relative error of as/|r| against d/|r| is below 2^-23).  The screen
+//      flags as >= y, y = RD32(Tp*|r| + 2^-149) (one fma rounded down),
+//      Tp = min(T, 1/2 -).  as lies on the fp32 grid, whose spacing is at
+//      least 2^-149: if as > Tp*|r| then either as >= Tp*|r| + 2^-149 >= y,
+//      or Tp*|r| + 2^-149 lies in (as, as + 2^-149) and rounds down to as;
+//      as = 0 (relative error 0) is never flagged, since y >= 2^-149.
+//      Flagged elements get the exact RN64(d/|r|) (one fma decides
+//      as > T*|r| exactly in sign).  Since y < |r|/2 for normal r, and a
+//      subnormal r makes every nonzero inexact difference exceed y, every
+//      element whose c - r may be inexact is flagged as well.
 // The maxima are order-independent (max of exact values), counts are sums
 // and first_mismatch a minimum, so any grid gives bit-identical results.
 //
-// Work split: a CTA's 8 warps are divided among the K candidates (G = 8/K
-// warps each).  For K > 1 the reference tile is staged once in shared
-// memory and every candidate's warps read it from there, so device memory
-// sees the reference once per tile.  Each lane keeps its statistics in
-// registers and a warp merges them into the global entries with atomics
-// when its CTA moves to the next region.
+// Work split: one CTA of 17 warps per SM.  The last warp streams each tile
+// of the reference and of the K <= 8 candidates into shared memory with
+// bulk copies (four stages, mbarrier-completed); the 16 checking warps are
+// divided among the candidates, so device memory sees the reference once
+// per tile.  Chunks the screen cannot settle are queued per warp and
+// drained lane-parallel.  Each lane keeps its statistics in registers and
+// a warp merges them into the global entries with atomics when its CTA
+// moves to the next region.
 //
 // Roofline: HBM reads of reference + candidate payloads (reference once per
-// launch of up to 8 candidates); the screen costs ~10 fp32/integer
-// operations per differing element, so dense small differences are also
-// ALU-heavy.
+// launch of up to 8 candidates); the screen costs about 10 fp32 operations
+// per differing element, so dense small differences are also ALU-heavy.
 #include <float.h>
 #include <math_constants.h>
 #include "device.cuh"
@@ -287,7 +295,7 @@ __device__ __forceinline__ uint32_t screen(float r, float s, float Tp, const Tol
   const float as = fabsf(s), ar = fabsf(r);
   const float lo = __fmaf_rn(t.rlo, ar, t.alo);
   const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
-  const float y = __fmaf_rn(Tp, ar, 0x1p-149f);
+  const float y = __fmaf_rd(Tp, ar, 0x1p-149f);
   const bool ok = as < lo;
   const bool bad = as > hi;
   rare |= (!(ok | bad)) | (as >= y);
