@@ -823,11 +823,17 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
       if (flt) {
         const long long *d = digits.data() + i * nslots * kEqDigits;
         const int base = eq_digit_base(ref[i].dtype);
-        if (exact_to_double_impl((const int64_t *)(d + (1 + 2 * j) * kEqDigits), kEqDigits, base,
-                                 &q.sum_rc) != ASMV_OK ||
-            exact_to_double_impl((const int64_t *)d, kEqDigits, base, &q.sum_rr) != ASMV_OK ||
-            exact_to_double_impl((const int64_t *)(d + (2 + 2 * j) * kEqDigits), kEqDigits, base,
-                                 &q.sum_cc) != ASMV_OK)
+        int64_t rc[kEqDigits], cc[kEqDigits];
+        const long long *rr = d, *s1 = d + (1 + 2 * j) * kEqDigits, *s2 = d + (2 + 2 * j) * kEqDigits;
+        const bool diff = eq_difference_form(ref[i].dtype);
+        for (int k = 0; k < kEqDigits; ++k) {
+          // digits stay far below 2^61, so these sums cannot overflow
+          rc[k] = diff ? (int64_t)rr[k] + s1[k] : s1[k];
+          cc[k] = diff ? (int64_t)rr[k] + 2 * (int64_t)s1[k] + s2[k] : s2[k];
+        }
+        if (exact_to_double_impl(rc, kEqDigits, base, &q.sum_rc) != ASMV_OK ||
+            exact_to_double_impl((const int64_t *)rr, kEqDigits, base, &q.sum_rr) != ASMV_OK ||
+            exact_to_double_impl(cc, kEqDigits, base, &q.sum_cc) != ASMV_OK)
           return ASMV_ECUDA;                         // digits out of range: a device fault
         q.cos = eq_cosine(q.sum_rc, q.sum_rr, q.sum_cc);
       } else {

@@ -296,6 +296,30 @@ __device__ __forceinline__ void sq(Acc3 &a, const Limbs &x) {
   a.s0 = mad_wide(x.lo, x.lo, a.s0);
 }
 
+// The difference form: with d = c - r formed exactly on the limbs,
+//   S_rc = S_rr + sum r d,   S_cc = S_rr + 2 sum r d + sum d^2,
+// so a candidate element adds r*d and d*d.  When |X_d| <= 2^28 (every
+// candidate within a few thousand units in the last place of the
+// reference) that is 3 multiply-adds instead of 7 (|X_d|^2 <= 2^56 and at
+// most 64 adds per flush keep every accumulator below 2^63).
+__device__ __forceinline__ void diff_add(Acc3 &rd, Acc3 &dd, const Limbs &x, const Limbs &y) {
+  const int dh = y.hi - x.hi, dl = y.lo - x.lo;
+  if ((unsigned)(dh + 255) <= 510u) {
+    const int xd = dh * (1 << 20) + dl;            // |xd| <= 2^28
+    rd.s1 = mad_wide(x.hi, xd, rd.s1);
+    rd.s0 = mad_wide(x.lo, xd, rd.s0);
+    dd.s0 = mad_wide(xd, xd, dd.s0);
+  } else {
+    rd.s2 = mad_wide(x.hi, dh, rd.s2);
+    rd.s1 = mad_wide(x.hi, dl, rd.s1);
+    rd.s1 = mad_wide(x.lo, dh, rd.s1);
+    rd.s0 = mad_wide(x.lo, dl, rd.s0);
+    dd.s2 = mad_wide(dh, dh, dd.s2);
+    dd.s1 = mad_wide(dh, 2 * dl, dd.s1);
+    dd.s0 = mad_wide(dl, dl, dd.s0);
+  }
+}
+
 // Warp-sum a digit vector and add it to the CTA's shared digits.
 template <int N>
 __device__ __forceinline__ void warp_add_digits(long long (&d)[N], long long *sdig) {
@@ -342,6 +366,8 @@ __device__ __forceinline__ uint32_t fp8_half(const uint4 &v, int k) {
 // One tile of an fp16 or fp8 region: S_rr once, then the candidates two at
 // a time (the reference chunk is decoded once per pair).  E5M2 and the fnuz
 // formats go through their exact fp16 values (and fp16's binary point).
+// For fp16 and those formats the candidate slots hold the difference-form
+// sums sum r d and sum d^2 (diff_add); the host forms S_rc and S_cc.
 template <int DT>
 __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R, uint32_t region,
                                            uint64_t a, uint32_t nb, long long *sdig) {
@@ -395,8 +421,8 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
           const Limbs x = fix_f16(half_of(rv, k));
           const Limbs y0 = fix_f16(half_of(v0, k));
           const Limbs y1 = fix_f16(half_of(v1, k));
-          mac(rc0, x, y0); sq(cc0, y0);
-          mac(rc1, x, y1); sq(cc1, y1);
+          diff_add(rc0, cc0, x, y0);
+          diff_add(rc1, cc1, x, y1);
         }
       } else if (DT != kF8) {
 #pragma unroll
@@ -404,8 +430,8 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
           const Limbs x = fix_f16(fp8_half<DT>(rv, k));
           const Limbs y0 = fix_f16(fp8_half<DT>(v0, k));
           const Limbs y1 = fix_f16(fp8_half<DT>(v1, k));
-          mac(rc0, x, y0); sq(cc0, y0);
-          mac(rc1, x, y1); sq(cc1, y1);
+          diff_add(rc0, cc0, x, y0);
+          diff_add(rc1, cc1, x, y1);
         }
       } else {
 #pragma unroll

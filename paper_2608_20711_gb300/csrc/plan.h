@@ -122,11 +122,17 @@ struct CmpParams {
 // The Eq. 1 sums (eqsum.cu).  Each sum of a region is kept as kEqDigits
 // signed 64-bit digits, digit k weighing 2^(32k + eq_digit_base(dtype)); the
 // digits of one region are [slot][kEqDigits] with slot 0 = S_rr and slots
-// 1 + 2j, 2 + 2j = S_rc, S_cc of candidate j.
+// 1 + 2j, 2 + 2j = S_rc, S_cc of candidate j -- or, for the formats of
+// eq_difference_form, sum r d and sum d^2 with d = c - r, from which
+// S_rc = S_rr + sum r d and S_cc = S_rr + 2 sum r d + sum d^2.
 constexpr int kEqDigits = 20;
 // fp8 formats other than E4M3 are summed through their exact fp16 value.
 constexpr int eq_digit_base(uint32_t dtype) {
   return dtype == kF32 ? -318 : dtype == kBF16 ? -286 : dtype == kF8 ? -82 : -112;
+}
+
+constexpr bool eq_difference_form(uint32_t dtype) {
+  return dtype == kF16 || dtype == kF8E5M2 || dtype == kF8E4FNUZ || dtype == kF8E5FNUZ;
 }
 
 struct EqParams {
