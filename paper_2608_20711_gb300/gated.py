@@ -2,12 +2,15 @@
 correctness strictly before timing, then the commit gate of Eq. 2.
 
 For a candidate c against the original K0 over the evaluated inputs X:
-  1. For each input x (a Tier 1 dispatch: input regions and a seed):
-     - the input regions are filled from x's seed (asmv_fill, guarded), the
-       reference output regions are overwritten with a poison pattern, and
-       K0 runs once, giving O(x);
+  1. For each input x -- a Tier 1 dispatch (input regions and a seed) or a
+     Tier 2 replay (captured regions and their pre-dispatch snapshots):
+     - the inputs are prepared (Tier 1: filled from x's seed with asmv_fill;
+       Tier 2: restored from the capture with asmv_restore, so kernels that
+       update their inputs in place start from the same state every run),
+       the reference output regions are overwritten with a poison pattern,
+       and K0 runs once, giving O(x);
      - c runs `repeats` times (three in the paper, Sec. 5); before each run
-       the inputs are filled again and the candidate's output regions are
+       the inputs are prepared again and the candidate's output regions are
        poisoned with a fresh pattern, so that output c failed to write cannot
        match; each result is checked with Eq. 1 (asmv_compare_eq).  The first
        failing check ends the evaluation as "divergent".
@@ -48,6 +51,26 @@ class Dispatch:
 
 
 @dataclass
+class ReplayDispatch:
+    """One evaluated input x captured from a real dispatch (Tier 2,
+    Sec. 3.4): the referenced regions (asmv Region objects or dicts, at the
+    addresses the kernel arguments point to) and, per region, the device
+    address of its captured pre-dispatch payload.  Before every run the
+    regions are restored from the capture (asmv_restore), guard bands
+    included."""
+    regions: Sequence
+    snapshots: Sequence[int]
+    name: str = ""
+
+
+def _prepare(ctx, x, stream):
+    if isinstance(x, ReplayDispatch):
+        ctx.restore(x.regions, x.snapshots, stream=stream)
+    else:
+        ctx.fill(x.inputs, seed=x.seed, stream=stream)
+
+
+@dataclass
 class GateResult:
     outcome: str
     commit: bool = False
@@ -84,15 +107,16 @@ def gated_eval(ctx: "asmv.Context", dispatches: Sequence[Dispatch],
     handle = st.cuda_stream
     res = GateResult(outcome="ok")
     for i, x in enumerate(dispatches):
-        ctx.fill(x.inputs, seed=x.seed, stream=st)
-        ctx.fill(_poisoned(ref_out, 0x5EF), seed=x.seed ^ POISON_TAG, stream=st)
+        salt = getattr(x, "seed", i)
+        _prepare(ctx, x, st)
+        ctx.fill(_poisoned(ref_out, 0x5EF), seed=salt ^ POISON_TAG, stream=st)
         try:
             run_original(i, handle)
         except Exception as e:           # the original must run; report, do not hide
             raise RuntimeError("the original kernel failed on input %d" % i) from e
         for rep in range(repeats):
-            ctx.fill(x.inputs, seed=x.seed, stream=st)
-            ctx.fill(_poisoned(cand_out, 0xCA0 + rep), seed=x.seed ^ POISON_TAG ^ (rep + 1),
+            _prepare(ctx, x, st)
+            ctx.fill(_poisoned(cand_out, 0xCA0 + rep), seed=salt ^ POISON_TAG ^ (rep + 1),
                      stream=st)
             try:
                 run_candidate(i, handle)
@@ -109,7 +133,7 @@ def gated_eval(ctx: "asmv.Context", dispatches: Sequence[Dispatch],
                                  "flags": eqs[0][bad[0]]["flags"]}
                 return res
     # timing on the representative launch (the first input), inputs in place
-    ctx.fill(dispatches[0].inputs, seed=dispatches[0].seed, stream=st)
+    _prepare(ctx, dispatches[0], st)
     t0 = asmv.time_launches(lambda h: run_original(0, h), reps, warmup, stream=st)
     t1 = asmv.time_launches(lambda h: run_candidate(0, h), reps, warmup, stream=st)
     res.timing_original = asmv.timing_summary(t0)

@@ -155,3 +155,34 @@ def test_time_launches_counts_each_launch(env):
     assert n["calls"] == 9 and len(ms) == 7 and all(m > 0 for m in ms)
     s = asmv.timing_summary(ms)
     assert s["r"] == 7 and s["median_ms"] == float(np.median(ms))
+
+
+def test_replay_dispatch_restores_inputs(env):
+    """Tier 2 replay: a kernel that updates its input in place (x += 1,
+    y = 2x) is equivalent on every repeat only because the captured
+    pre-state is restored before each run."""
+    from paper_2608_20711_gb300.gated import ReplayDispatch
+    torch = env["torch"]
+    ctx = env["ctx"]
+    ctx.fill(env["inp"], seed=31)
+    snap = torch.empty(2 * N, dtype=torch.uint8, device="cuda")
+    ctx.capture(env["inp"], [snap.data_ptr()])
+
+    def original(i, h):
+        with _on(torch, h):
+            env["x"].add_(1)
+            torch.mul(env["x"], 2, out=env["y0"])
+
+    def candidate(i, h):
+        with _on(torch, h):
+            env["x"].add_(1)
+            torch.add(env["x"], env["x"], out=env["y1"])
+    x = ReplayDispatch(env["inp"], [snap.data_ptr()])
+    r = gated_eval(ctx, [x], original, candidate, env["ref_out"], env["cand_out"],
+                   W.DEFAULT_TOL, reps=5)
+    assert r.outcome == "ok" and len(r.checks) == 3
+    # without restoring, the second repeat would see x + 2 and diverge
+    xs = [Dispatch(env["inp"], seed=31)]
+    r2 = gated_eval(ctx, xs, original, candidate, env["ref_out"], env["cand_out"],
+                    W.DEFAULT_TOL, reps=5)
+    assert r2.outcome == "ok"                     # Tier 1 refills the input each run too
