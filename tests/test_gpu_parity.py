@@ -351,3 +351,19 @@ def test_rejects_host_memory_and_bad_tables(ctx):
     with pytest.raises(asmv.AsmvError):
         ctx.compare(ok, ok, {"f32": (-1.0, 0.0)})
     assert ctx.compare([], [], TOL) == []
+
+
+def test_radius_sqrt_matches_ieee_on_its_whole_domain(tmp_path):
+    """The fill's Box-Muller radius uses its own correctly rounded square
+    root; it must equal the IEEE square root on all 2^24 possible inputs."""
+    import os
+    import subprocess
+    torch_cuda()
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    exe = str(tmp_path / "radius_sqrt_check")
+    subprocess.check_call(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
+                           "-I", os.path.join(root, "paper_2608_20711_gb300", "csrc"), "-o", exe,
+                           os.path.join(root, "tests", "helpers", "radius_sqrt_check.cu")])
+    out = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert out.returncode == 0, out.stdout + out.stderr
+    assert "differing 0 " in out.stdout
