@@ -359,6 +359,20 @@ int asmv_ctx_cuda_error(const asmv_ctx *ctx);
 /* Number of kernels this context has launched since creation. */
 uint64_t asmv_ctx_launches(const asmv_ctx *ctx);
 
+/* Every device wait of the compare pipeline is bounded: ASMV_WAIT_ROUNDS
+ * tries of up to 100 us.  A wait that runs out sets the launch's error word,
+ * the kernel lets the copies it issued land and returns, and the call
+ * returns ASMV_ETIMEOUT with out_host untouched and the context usable.
+ * This sets, per context, the bound of one of those waits: the copy
+ * producer's wait for a stage the checking warps have released.  Meant for
+ * tests of the timeout path: with 0 the producer gives up as soon as it
+ * needs a stage back (in any CTA with more than four tiles), its checking
+ * warps then wait in vain for the next tile until their own default bound
+ * runs out (about 2 s), and the call returns ASMV_ETIMEOUT.  EINVAL for a
+ * null ctx. */
+#define ASMV_WAIT_ROUNDS 20000u
+int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds);
+
 /* Static description of a status code. */
 const char *asmv_strerror(int status);
 

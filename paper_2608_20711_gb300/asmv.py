@@ -86,8 +86,9 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double",
                  "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches",
                  "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
-                 "asmv_va_address", "asmv_va_size", "asmv_va_unmap")
+                 "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds")
 NOALLOC_SCRATCH_BYTES = 1 << 20
+WAIT_ROUNDS = 20000                      # default bound of the compare's device waits
 
 
 class AsmvError(RuntimeError):
@@ -123,6 +124,7 @@ def lib():
         L.asmv_ctx_cuda_error.argtypes = [vp]
         L.asmv_ctx_launches.argtypes = [vp]
         L.asmv_ctx_launches.restype = ctypes.c_uint64
+        L.asmv_ctx_set_wait_rounds.argtypes = [vp, ctypes.c_uint32]
         L.asmv_strerror.argtypes = [ctypes.c_int]
         L.asmv_strerror.restype = ctypes.c_char_p
         L.asmv_abi_version.argtypes = []
@@ -300,6 +302,13 @@ class Context:
     @property
     def launches(self) -> int:
         return int(self._lib.asmv_ctx_launches(self._h))
+
+    def set_wait_rounds(self, rounds: int = None):
+        """Bound of the compare pipeline's device waits (tries of up to
+        100 us); None restores the default.  0 makes every compare with a
+        non-empty payload return ETIMEOUT (a test of that path)."""
+        r = WAIT_ROUNDS if rounds is None else int(rounds)
+        self._check(self._lib.asmv_ctx_set_wait_rounds(self._h, r))
 
     def set_timing(self, enable: bool = True):
         self._check(self._lib.asmv_ctx_set_timing(self._h, 1 if enable else 0))

@@ -27,6 +27,7 @@ static_assert(sizeof(asmv_stats) == 64, "asmv_stats layout");
 static_assert(sizeof(asmv_eq) == 40, "asmv_eq layout");
 static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
 static_assert(sizeof(CopyRegion) == 48, "copy region layout");
+static_assert(kWaitRounds == ASMV_WAIT_ROUNDS, "default wait bound");
 static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
               "plan layouts");
 
@@ -217,6 +218,7 @@ struct asmv_ctx {
   cudaEvent_t t0 = nullptr, t1 = nullptr;
   int cuda_err = 0;
   uint64_t launches = 0;
+  uint32_t wait_rounds = kWaitRounds;
   AddrRangeFn addr_range = nullptr;
 };
 
@@ -499,6 +501,12 @@ int asmv_ctx_cuda_error(const asmv_ctx *ctx) { return ctx ? ctx->cuda_err : 0; }
 
 uint64_t asmv_ctx_launches(const asmv_ctx *ctx) { return ctx ? ctx->launches : 0; }
 
+int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds) {
+  if (ctx == nullptr) return ASMV_EINVAL;
+  ctx->wait_rounds = rounds;
+  return ASMV_OK;
+}
+
 int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed,
               asmv_stream_t stream) {
   if (ctx == nullptr) return ASMV_EINVAL;
@@ -637,6 +645,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   p.ntiles = tile;
   p.nregions = (uint32_t)n;
   p.tile_bytes = tile_bytes;
+  p.wait_rounds = ctx->wait_rounds;
   for (int d = 0; d < ASMV_NDTYPES; ++d) {
     if (is_float((uint32_t)d) && tol) p.tol[d] = make_tolf(tol[d]);
   }
@@ -1139,6 +1148,7 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   p.nsegs = (uint32_t)ks;
   p.K = 1;
   p.tile_bytes = tile_bytes;
+  p.wait_rounds = kWaitRounds;
   for (int d = 0; d < ASMV_NDTYPES; ++d)
     if (is_float((uint32_t)d)) p.tol[d] = make_tolf(tol[d]);
   const uint64_t per_cta = kConsumerWarps + 1;

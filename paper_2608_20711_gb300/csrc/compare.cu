@@ -422,8 +422,11 @@ __device__ __forceinline__ uint4 load_chunk(uint64_t base, uint64_t c, uint64_t 
 
 // ---------------------------------------------------------------- pipeline
 // mbarrier helpers (shared::cta addresses).  Waits are bounded: after
-// kWaitRounds tries of up to kWaitHintNs each, the wait reports failure.
-constexpr uint32_t kWaitRounds = 20000;
+// `rounds` tries of up to kWaitHintNs each, the wait reports failure.  The
+// producer's wait for a free stage takes the launch's bound
+// (CmpParams::wait_rounds; 0 gives up without trying, which makes its
+// consumers' waits run out: the test of this path); every other wait takes
+// kWaitRounds.
 constexpr uint32_t kWaitHintNs = 100000;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -439,8 +442,8 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t tx) {
   asm volatile("{ .reg .b64 st; mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1; }"
                :: "r"(bar), "r"(tx) : "memory");
 }
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kWaitRounds; ++i) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t rounds) {
+  for (uint32_t i = 0; i < rounds; ++i) {
     uint32_t done;
     asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;"
                  " selp.u32 %0, 1, 0, p; }"
@@ -519,7 +522,7 @@ __device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, u
   uint32_t u = cur->u;
   for (; t < t_end; ++t, ++u) {
     const uint32_t s = u % kStages;
-    if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u)) { cur->ok = 0; break; }
+    if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u, kWaitRounds)) { cur->ok = 0; break; }
     if (active) {
       const TileInfo ti = tile_info(r, t, tile_bytes);
       const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
@@ -641,7 +644,8 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
       for (uint64_t t = t0; t < t1 && ok; ++t, ++u) {
         while (p.regions[ri + 1].tile0 <= t) ++ri;
         const uint32_t s = u % kStages;
-        if (u >= (uint32_t)kStages && !mbar_wait(smem_addr(&empty[s]), ((u / kStages) & 1u) ^ 1u)) {
+        if (u >= (uint32_t)kStages &&
+            !mbar_wait(smem_addr(&empty[s]), ((u / kStages) & 1u) ^ 1u, p.wait_rounds)) {
           ok = false;
           break;
         }
@@ -657,12 +661,13 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
             bulk_load(dst + (1 + k) * TB, p.cands[(size_t)k * p.nregions + ri] + ti.off, nb, fb);
         }
       }
-      if (!ok) {
-        atomicOr(p.err, 1u);
-        // let copies already issued land before the CTA exits
-        for (uint32_t v = (u >= (uint32_t)kStages ? u - kStages : 0); v < u; ++v)
-          mbar_wait(smem_addr(&full[v % kStages]), (v / kStages) & 1u);
-      }
+      if (!ok) atomicOr(p.err, 1u);
+      // Let every copy issued land before the CTA can exit: consumers that
+      // gave up on a wait leave their stages unread.  Each stage's latest
+      // phase is the one awaited; in a run without errors these have
+      // completed already.
+      for (uint32_t v = (u >= (uint32_t)kStages ? u - kStages : 0); v < u; ++v)
+        mbar_wait(smem_addr(&full[v % kStages]), (v / kStages) & 1u, kWaitRounds);
     }
   } else if (t0 < t1) {
     // consumers: one call per run of tiles of the same region

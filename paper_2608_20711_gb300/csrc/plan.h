@@ -27,6 +27,7 @@ constexpr int kMaxCands = 8;            // candidates per batched launch
 constexpr int kConsumerWarps = 16;      // compare: checking warps per CTA
 constexpr int kStages = 4;              // compare: shared-memory pipeline depth
 constexpr int kCmpThreads = (kConsumerWarps + 1) * 32;   // + one producer warp
+constexpr uint32_t kWaitRounds = 20000;  // compare: default bound of a pipeline wait, in tries
 
 enum : uint32_t { kF32 = 0, kBF16 = 1, kF16 = 2, kF8 = 3, kI32 = 4, kI8 = 5, kU8 = 6,
                   kF8E5M2 = 7, kF8E4FNUZ = 8, kF8E5FNUZ = 9, kF64 = 10, kI16 = 11, kI64 = 12,
@@ -116,6 +117,7 @@ struct CmpParams {
   uint32_t nsegs;
   uint32_t K;
   uint32_t tile_bytes;         // payload bytes per tile (multiple of 16)
+  uint32_t wait_rounds;        // bound of the producer's wait for a free stage (tries)
   TolF tol[kNDtypes];
 };
 

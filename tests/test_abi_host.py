@@ -45,6 +45,8 @@ def test_layouts_and_version():
     assert ctypes.sizeof(asmv.EqResult) == 40
     ver = int(re.search(r"#define ASMV_ABI_VERSION (\d+)", text).group(1))
     assert _lib().asmv_abi_version() == ver
+    assert int(re.search(r"#define ASMV_WAIT_ROUNDS (\d+)u", text).group(1)) == asmv.WAIT_ROUNDS
+    assert _lib().asmv_ctx_set_wait_rounds(None, 0) == asmv.EINVAL
     for name, code in (("ASMV_EQ_COS", asmv.EQ_COS), ("ASMV_EQ_LINF", asmv.EQ_LINF),
                        ("ASMV_EQ_INT", asmv.EQ_INT), ("ASMV_EQ_GUARD", asmv.EQ_GUARD)):
         assert int(re.search(r"#define %s +(\d+)u" % name, text).group(1)) == code
