@@ -20,10 +20,11 @@
 //   global digits with 64-bit atomics; values between about 2^-24 and 2^24
 //   stay in the window.
 //
-// Reduction.  Every tile, each warp carries its lanes' accumulators into
-// 32-bit digits, sums them over the warp with shuffles and adds them to the
-// CTA's shared digits; the CTA adds those to the region's global digits when
-// it leaves the region.  Global digit k of a sum weighs 2^(32k + base), base
+// Reduction.  Every tile, each warp cuts its lanes' accumulated sums into
+// 16-bit pieces whose warp sums fit in 32 bits, sums each piece over the
+// warp with one redux, and adds the recombined digits to the CTA's shared
+// digits; the CTA adds those to the region's global digits when it leaves
+// the region.  Three CTAs of 256 threads share an SM (80 registers).  Global digit k of a sum weighs 2^(32k + base), base
 // = eq_digit_base(dtype); the host rounds the digits to fp64.
 //
 // Work split: like the compare, a persistent grid over 16 KiB tiles of the
@@ -141,6 +142,18 @@ __device__ __forceinline__ void add_product(long long (&a)[Fmt<DT>::kNacc], cons
   }
 }
 
+// Warp sum of one lane value |v| < 2^32 added to one shared digit: v is
+// cut into its low 16 bits and the signed rest (|rest| < 2^16), whose warp
+// sums fit in 32 bits and take one redux each.
+__device__ __forceinline__ void warp_add_digit(long long v, long long *sd) {
+  const uint32_t a = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)v & 0xFFFFu);
+  const int b = __reduce_add_sync(0xFFFFFFFFu, (int)(v >> 16));
+  if ((threadIdx.x & 31) == 0) {
+    const long long s = (long long)a + (long long)b * 65536ll;
+    if (s != 0) atomicAdd(reinterpret_cast<unsigned long long *>(sd), (unsigned long long)s);
+  }
+}
+
 // Carry the lane's accumulators into N+1 digits, sum them over the warp and
 // add them to the CTA's shared digits of one sum.  All 32 lanes call this.
 template <int N>
@@ -156,13 +169,7 @@ __device__ __forceinline__ void warp_flush(long long (&a)[N], long long *sdig) {
   }
   d[N] = carry;
 #pragma unroll
-  for (int k = 0; k <= N; ++k) {
-    long long v = d[k];
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    if ((threadIdx.x & 31) == 0 && v != 0)
-      atomicAdd(reinterpret_cast<unsigned long long *>(sdig + k), (unsigned long long)v);
-  }
+  for (int k = 0; k <= N; ++k) warp_add_digit(d[k], sdig + k);
 }
 
 __device__ __forceinline__ long long *global_digits(const EqParams &p, uint32_t region, uint32_t slot) {
@@ -271,6 +278,26 @@ __device__ __forceinline__ Limbs fix_f16(uint32_t b) {
           __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic)) - kMagicBits};
 }
 
+// The same limbs, each plus kMagicBits, for a value known to be finite:
+// for a candidate only the differences of its limbs from the reference's
+// are used, so the offsets cancel and need no subtraction.
+__device__ __forceinline__ Limbs fix_f16_biased(uint32_t b) {
+  const float x = __half2float(__ushort_as_half((unsigned short)b));
+  const float hf = __fmaf_rn(x, 16.0f, kMagic);
+  const float l = __fmaf_rn(__fsub_rn(hf, kMagic), -0.0625f, x);
+  return {__float_as_int(hf), __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic))};
+}
+
+// A pair of fp16 values with the non-finite ones replaced by zero: x - x is
+// zero exactly for finite x and a NaN for an infinity or a NaN.
+__device__ __forceinline__ uint32_t finite_f16x2(uint32_t w) {
+  const __half2 h = *reinterpret_cast<const __half2 *>(&w);
+  return w & __heq2_mask(__hsub2(h, h), __float2half2_rn(0.0f));
+}
+__device__ __forceinline__ uint4 finite_f16x8(uint4 v) {
+  return make_uint4(finite_f16x2(v.x), finite_f16x2(v.y), finite_f16x2(v.z), finite_f16x2(v.w));
+}
+
 // fp8 e4m3 bits -> X = x 2^9 (|X| < 2^18), exactly.
 __device__ __forceinline__ int fix_f8(uint32_t b) {
   b = ((b & 0x7Fu) == 0x7Fu) ? 0u : b;                          // NaN -> 0
@@ -301,9 +328,12 @@ __device__ __forceinline__ void sq(Acc3 &a, const Limbs &x) {
 // so a candidate element adds r*d and d*d.  When |X_d| <= 2^28 (every
 // candidate within a few thousand units in the last place of the
 // reference) that is 3 multiply-adds instead of 7 (|X_d|^2 <= 2^56 and at
-// most 64 adds per flush keep every accumulator below 2^63).
-__device__ __forceinline__ void diff_add(Acc3 &rd, Acc3 &dd, const Limbs &x, const Limbs &y) {
-  const int dh = y.hi - x.hi, dl = y.lo - x.lo;
+// most 64 adds per flush keep every accumulator below 2^63).  x holds the
+// reference's limbs; xo and y the reference's and the candidate's limbs
+// with one common offset, which cancels in the differences.
+__device__ __forceinline__ void diff_add(Acc3 &rd, Acc3 &dd, const Limbs &x, const Limbs &xo,
+                                         const Limbs &y) {
+  const int dh = y.hi - xo.hi, dl = y.lo - xo.lo;
   if ((unsigned)(dh + 255) <= 510u) {
     const int xd = dh * (1 << 20) + dl;            // |xd| <= 2^28
     rd.s1 = mad_wide(x.hi, xd, rd.s1);
@@ -320,32 +350,44 @@ __device__ __forceinline__ void diff_add(Acc3 &rd, Acc3 &dd, const Limbs &x, con
   }
 }
 
-// Warp-sum a digit vector and add it to the CTA's shared digits.
-template <int N>
-__device__ __forceinline__ void warp_add_digits(long long (&d)[N], long long *sdig) {
+// Warp sum of one lane value T, |T| < 2^95, added to three of the CTA's
+// shared digits (digit k weighs 2^32k).  T is cut into six 16-bit pieces,
+// five unsigned and the top one signed:
+//   T = p0 + p1 2^16 + p2 2^32 + p3 2^48 + p4 2^64 + p5 2^80,
+// so every piece's warp sum fits in 32 bits (below 2^21) and takes one
+// redux; lane 0 recombines the sums two by two into the digits.
+__device__ __forceinline__ void warp_add_t(__int128 T, long long *sdig) {
+  const unsigned long long lo = (unsigned long long)T;
+  const long long hi = (long long)(T >> 64);             // |hi| < 2^31
+  const uint32_t a0 = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)lo & 0xFFFFu);
+  const uint32_t a1 = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)(lo >> 16) & 0xFFFFu);
+  const uint32_t a2 = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)(lo >> 32) & 0xFFFFu);
+  const uint32_t a3 = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)(lo >> 48));
+  const uint32_t a4 = __reduce_add_sync(0xFFFFFFFFu, (uint32_t)hi & 0xFFFFu);
+  const int a5 = __reduce_add_sync(0xFFFFFFFFu, (int)(hi >> 16));    // |piece| < 2^15
+  if ((threadIdx.x & 31) == 0) {
+    const long long d[3] = {(long long)a0 + ((long long)a1 << 16), (long long)a2 + ((long long)a3 << 16),
+                            (long long)a4 + ((long long)a5 * 65536ll)};
 #pragma unroll
-  for (int k = 0; k < N; ++k) {
-    long long v = d[k];
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    if ((threadIdx.x & 31) == 0 && v != 0)
-      atomicAdd(reinterpret_cast<unsigned long long *>(sdig + k), (unsigned long long)v);
+    for (int k = 0; k < 3; ++k)
+      if (d[k] != 0) atomicAdd(reinterpret_cast<unsigned long long *>(sdig + k), (unsigned long long)d[k]);
   }
 }
 
-// sum = s2 2^40 + s1 2^20 + s0 (|s| < 2^63) as four digits of 32 bits.
+// sum = s2 2^40 + s1 2^20 + s0.  Between two flushes a lane adds at most 64
+// products (one tile), each |r d|, |d d| <= 2^56 in the short form and each
+// partial product <= 2^42 in the limb form, so |s0| < 2^63, |s1| < 2^56,
+// |s2| < 2^49 and |sum| < 2^90.
 __device__ __forceinline__ void flush3(Acc3 &a, long long *sdig) {
   const __int128 T = (__int128)a.s0 + (__int128)a.s1 * ((__int128)1 << 20) +
                     (__int128)a.s2 * ((__int128)1 << 40);
-  long long d[4] = {(long long)(T & 0xFFFFFFFF), (long long)((T >> 32) & 0xFFFFFFFF),
-                    (long long)((T >> 64) & 0xFFFFFFFF), (long long)(T >> 96)};
-  warp_add_digits(d, sdig);
+  warp_add_t(T, sdig);
   a.s2 = a.s1 = a.s0 = 0;
 }
 
+// fp8 e4m3 products are below 2^36, so a tile's sum is below 2^42.
 __device__ __forceinline__ void flush1(long long &s, long long *sdig) {
-  long long d[2] = {s & 0xFFFFFFFFll, s >> 32};
-  warp_add_digits(d, sdig);
+  warp_add_t((__int128)s, sdig);
   s = 0;
 }
 
@@ -416,22 +458,22 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
         if (two) v1 = load_chunk(cb1 + 16ull * c, bytes, R.vec, false);
       }
       if (DT == kF16) {
+        rv = finite_f16x8(rv);
+        v0 = finite_f16x8(v0);
+        v1 = finite_f16x8(v1);
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-          const Limbs x = fix_f16(half_of(rv, k));
-          const Limbs y0 = fix_f16(half_of(v0, k));
-          const Limbs y1 = fix_f16(half_of(v1, k));
-          diff_add(rc0, cc0, x, y0);
-          diff_add(rc1, cc1, x, y1);
+          const Limbs xb = fix_f16_biased(half_of(rv, k));
+          const Limbs x = {xb.hi - kMagicBits, xb.lo - kMagicBits};
+          diff_add(rc0, cc0, x, xb, fix_f16_biased(half_of(v0, k)));
+          diff_add(rc1, cc1, x, xb, fix_f16_biased(half_of(v1, k)));
         }
       } else if (DT != kF8) {
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           const Limbs x = fix_f16(fp8_half<DT>(rv, k));
-          const Limbs y0 = fix_f16(fp8_half<DT>(v0, k));
-          const Limbs y1 = fix_f16(fp8_half<DT>(v1, k));
-          diff_add(rc0, cc0, x, y0);
-          diff_add(rc1, cc1, x, y1);
+          diff_add(rc0, cc0, x, x, fix_f16(fp8_half<DT>(v0, k)));
+          diff_add(rc1, cc1, x, x, fix_f16(fp8_half<DT>(v1, k)));
         }
       } else {
 #pragma unroll
@@ -474,7 +516,7 @@ __device__ void cta_flush(const EqParams &p, uint32_t region, uint32_t dtype, lo
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kThreads) eq_kernel(EqParams p) {
+__global__ void __launch_bounds__(kThreads, 3) eq_kernel(EqParams p) {   // 3 CTAs per SM
   __shared__ long long sdig[(1 + 2 * kMaxCands) * kWin];
   for (uint32_t x = threadIdx.x; x < (1 + 2 * kMaxCands) * kWin; x += blockDim.x) sdig[x] = 0;
   __syncthreads();
