@@ -119,7 +119,7 @@ def kernel_traffic(kernel, workload):
 
 
 # the source files each kernel is compiled from
-KERNEL_SOURCES = {"fill": ("fill.cu", "device.cuh", "ln_table.h", "plan.h"),
+KERNEL_SOURCES = {"fill": ("fill.cu", "fill_math.cuh", "device.cuh", "ln_table.h", "plan.h"),
                   "compare": ("compare.cu", "device.cuh", "plan.h"),
                   "eqsum": ("eqsum.cu", "device.cuh", "plan.h"),
                   "copy": ("copy.cu", "device.cuh", "plan.h")}

@@ -11,7 +11,7 @@
 // Roofline: HBM writes of payload + guard bytes; Philox (about 80 integer
 // operations per 16-byte block) and Box-Muller for NORMAL also load the
 // ALUs, so 16-bit and 8-bit NORMAL fills are arithmetic-bound.
-#include "device.cuh"
+#include "fill_math.cuh"
 #include "ln_table.h"
 
 namespace asmv {
@@ -22,19 +22,23 @@ __device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
   return __fadd_rn(lo, __fmul_rn(f, width));
 }
 
+// v = mean + sd*z for the four normals of a block, two per packed
+// instruction: v[0], v[2] from z0 of the two pairs, v[1], v[3] from z1.
 __device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const float4 *tab, float v[4]) {
-  float z[4];
-  box_muller(w.x, w.y, tab, z[0], z[1]);
-  box_muller(w.z, w.w, tab, z[2], z[3]);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) v[j] = __fadd_rn(mean, __fmul_rn(sd, z[j]));
+  float2 z0, z1;
+  box_muller2(w, tab, z0, z1);
+  const float2 a = __fadd2_rn(f2(mean), __fmul2_rn(f2(sd), z0));
+  const float2 b = __fadd2_rn(f2(mean), __fmul2_rn(f2(sd), z1));
+  v[0] = a.x; v[1] = b.x; v[2] = a.y; v[3] = b.y;
 }
 
+// uniform_of for the four words of a block, two per packed instruction.
 __device__ __forceinline__ void uniform4(uint4 w, float lo, float width, float v[4]) {
-  v[0] = uniform_of(w.x, lo, width);
-  v[1] = uniform_of(w.y, lo, width);
-  v[2] = uniform_of(w.z, lo, width);
-  v[3] = uniform_of(w.w, lo, width);
+  const float2 fa = __fmul2_rn(make_float2(__uint2float_rn(w.x >> 8), __uint2float_rn(w.y >> 8)), f2(0x1p-24f));
+  const float2 fb = __fmul2_rn(make_float2(__uint2float_rn(w.z >> 8), __uint2float_rn(w.w >> 8)), f2(0x1p-24f));
+  const float2 a = __fadd2_rn(f2(lo), __fmul2_rn(fa, f2(width)));
+  const float2 b = __fadd2_rn(f2(lo), __fmul2_rn(fb, f2(width)));
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
 }
 
 __device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span) {

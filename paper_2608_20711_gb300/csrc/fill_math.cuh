@@ -1,0 +1,243 @@
+// fill_math.cuh -- the arithmetic of the Tier 1 fill (AsmEvo Sec. 3.4):
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), the fp32 Box-Muller
+// transform of the NORMAL distribution and the encoders to the stored
+// formats.  Every floating-point step uses an explicit _rn intrinsic (one
+// or two IEEE operations) so that nvcc cannot contract or reorder it; the
+// sequence of IEEE operations is the one the library's specification
+// states, which makes the filled bytes reproducible on any IEEE machine.
+#pragma once
+#include "device.cuh"
+
+namespace asmv {
+
+// ---------------------------------------------------------------- Philox
+// Philox4x32-10 round: (x0,x1,x2,x3) -> (hi(B*x2)^x1^k0, lo(B*x2), hi(A*x0)^x3^k1,
+// lo(A*x0)) with A = 0xD2511F53, B = 0xCD9E8D57; round r uses the key
+// (k0 + r*0x9E3779B9, k1 + r*0xBB67AE85) (SC'11, Sec. 3).
+// Ten rounds with the round keys given (one 64-bit product per multiplier;
+// the keys are kernel-parameter operands of the XORs).
+__device__ __forceinline__ void mul_wide(uint32_t a, uint32_t m, uint32_t &hi, uint32_t &lo) {
+  asm("{ .reg .u64 t; mul.wide.u32 t, %2, %3; mov.b64 {%1, %0}, t; }"
+      : "=r"(hi), "=r"(lo) : "r"(a), "r"(m));
+}
+
+__device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, const uint32_t *k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    uint32_t ahi, alo, bhi, blo;
+    mul_wide(x.x, 0xD2511F53u, ahi, alo);
+    mul_wide(x.z, 0xCD9E8D57u, bhi, blo);
+    x = make_uint4(bhi ^ x.y ^ k0[r], blo, ahi ^ x.w ^ k1[r], alo);
+  }
+  return x;
+}
+
+// ---------------------------------------------------------------- Box-Muller
+// ln(u), u = k 2^-24: u = m 2^e with m in [1, 2); j = round(128 (m - 1));
+// r = m*inv_j - 1 exactly (fma); ln u = e ln2 + (-ln inv_j) + log1p(r), with
+// ln 2 and -ln inv_j split into a 2^-9-multiple head (exact sum) and an fp32
+// tail, and log1p(r) = r + r^2 (-1/2 + r (1/3 - r/4)) for |r| < 2^-7.  The
+// table lives in shared memory (ln_table.h).
+// sin/cos(2 pi u): nearest quarter turn removed exactly in integers, then the
+// Taylor series of sin(pi/2 r) and cos(pi/2 r) for r in [-1/2, 1/2); each
+// coefficient is the fp32 rounding of +-(pi/2)^j / j!.
+#define ASMV_LN2_HI 0x1.63p-1f
+#define ASMV_LN2_LO (-0x1.bd0106p-13f)
+#define ASMV_THIRD 0x1.555556p-2f
+#define ASMV_S1 0x1.921fb6p+0f
+#define ASMV_S3 (-0x1.4abbcep-1f)
+#define ASMV_S5 0x1.466bc6p-4f
+#define ASMV_S7 (-0x1.32d2ccp-8f)
+#define ASMV_S9 0x1.507834p-13f
+#define ASMV_C2 (-0x1.3bd3ccp+0f)
+#define ASMV_C4 0x1.03c1f0p-2f
+#define ASMV_C6 (-0x1.55d3c8p-6f)
+#define ASMV_C8 0x1.e1f506p-11f
+#define ASMV_C10 (-0x1.a6d1f2p-16f)
+
+__device__ __forceinline__ float ln_u24(uint32_t k, const float4 *tab) {
+  const float u = __fmul_rn(__uint2float_rn(k), 0x1p-24f);   // exact
+  const uint32_t bits = __float_as_uint(u);
+  const int e = (int)(bits >> 23) - 127;
+  const uint32_t mb = bits & 0x7FFFFFu;
+  const float m = __uint_as_float(mb | 0x3F800000u);
+  const float4 t = tab[(mb + (1u << 15)) >> 16];             // inv, hi, lo
+  const float r = __fmaf_rn(m, t.x, -1.0f);                  // exact
+  const float r2 = __fmul_rn(r, r);
+  float p = __fmaf_rn(r, -0.25f, ASMV_THIRD);
+  p = __fmaf_rn(r, p, -0.5f);
+  const float lp = __fmaf_rn(r2, p, r);
+  // exact int -> float for |e| < 2^22: 1.5*2^23 + e has unit spacing
+  const float ef = __fsub_rn(__int_as_float(0x4B400000 + e), 12582912.0f);
+  const float hi = __fmaf_rn(ef, ASMV_LN2_HI, t.y);           // exact
+  const float lo = __fmaf_rn(ef, ASMV_LN2_LO, t.z);
+  return __fadd_rn(hi, __fadd_rn(lo, lp));
+}
+
+// sin and cos of 2 pi k 2^-24, k in [0, 2^24).
+__device__ __forceinline__ void sincos_u24(uint32_t k, float &sn, float &cs) {
+  const uint32_t q = (k + (1u << 21)) >> 22;                 // nearest quarter turn
+  const int32_t ri = (int32_t)k - (int32_t)(q << 22);
+  // r = ri * 2^-22 exactly: floats in [2, 4) are spaced 2^-22 apart
+  const float r = __fsub_rn(__int_as_float(0x40400000 + ri), 3.0f);
+  const float r2 = __fmul_rn(r, r);
+  float sp = __fmaf_rn(r2, ASMV_S9, ASMV_S7);
+  sp = __fmaf_rn(r2, sp, ASMV_S5);
+  sp = __fmaf_rn(r2, sp, ASMV_S3);
+  sp = __fmaf_rn(r2, sp, ASMV_S1);
+  const float s = __fmul_rn(r, sp);
+  float cp = __fmaf_rn(r2, ASMV_C10, ASMV_C8);
+  cp = __fmaf_rn(r2, cp, ASMV_C6);
+  cp = __fmaf_rn(r2, cp, ASMV_C4);
+  cp = __fmaf_rn(r2, cp, ASMV_C2);
+  const float c = __fmaf_rn(r2, cp, 1.0f);
+  // quarter turn q: (sin, cos) = (s, c), (c, -s), (-s, -c), (-c, s)
+  const bool odd = q & 1u;
+  const float a = odd ? c : s, b = odd ? s : c;
+  sn = __uint_as_float(__float_as_uint(a) ^ ((q & 2u) << 30));
+  cs = __uint_as_float(__float_as_uint(b) ^ (((q + 1u) & 2u) << 30));
+}
+
+// sqrt(x), correctly rounded, for the radii of Box-Muller: x = -2 ln(u1)
+// lies in [-0, 33.3].  Markstein's method (P. Markstein, "IA-64 and
+// Elementary Functions", 2000): s = x * rsqrt(x) from the hardware
+// approximation, then one Newton step on the exact residual x - s*s (one
+// fma).  Equal to the IEEE square root on every one of the 2^24 inputs the
+// fill can produce (checked exhaustively on the GPU against __fsqrt_rn; the
+// test suite repeats the check); zero is returned as is, keeping -0.
+__device__ __forceinline__ float sqrt_radius(float x) {
+  const float r = rsqrtf(x);
+  const float s = __fmul_rn(x, r);
+  const float e = __fmaf_rn(-s, s, x);
+  const float y = __fmaf_rn(e, __fmul_rn(0.5f, r), s);
+  return x == 0.0f ? x : y;
+}
+
+__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const float4 *tab, float &z0,
+                                           float &z1) {
+  const float l = ln_u24((w0 >> 8) + 1u, tab);
+  const float rho = sqrt_radius(__fmul_rn(-2.0f, l));
+  float sn, cs;
+  sincos_u24(w1 >> 8, sn, cs);
+  z0 = __fmul_rn(rho, cs);
+  z1 = __fmul_rn(rho, sn);
+}
+
+// Two Box-Muller pairs at once, (w.x, w.y) and (w.z, w.w): the sequence of
+// box_muller with every fp32 step of the two pairs in one packed
+// instruction (f32x2: two IEEE operations, each rounded exactly as its
+// scalar form), the integer steps and the reciprocal square root per lane.
+// z0 = (z0 of pair a, z0 of pair b), z1 likewise.
+__device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
+
+__device__ __forceinline__ void box_muller2(uint4 w, const float4 *tab, float2 &z0, float2 &z1) {
+  // ln(k 2^-24), k = (w >> 8) + 1
+  const uint32_t ka = (w.x >> 8) + 1u, kb = (w.z >> 8) + 1u;
+  const float2 u = __fmul2_rn(make_float2(__uint2float_rn(ka), __uint2float_rn(kb)), f2(0x1p-24f));
+  const uint32_t ba = __float_as_uint(u.x), bb = __float_as_uint(u.y);
+  const uint32_t ma = ba & 0x7FFFFFu, mb = bb & 0x7FFFFFu;
+  const float4 ta = tab[(ma + (1u << 15)) >> 16], tb = tab[(mb + (1u << 15)) >> 16];
+  const float2 m = make_float2(__uint_as_float(ma | 0x3F800000u), __uint_as_float(mb | 0x3F800000u));
+  const float2 r = __ffma2_rn(m, make_float2(ta.x, tb.x), f2(-1.0f));
+  const float2 r2 = __fmul2_rn(r, r);
+  float2 p = __ffma2_rn(r, f2(-0.25f), f2(ASMV_THIRD));
+  p = __ffma2_rn(r, p, f2(-0.5f));
+  const float2 lp = __ffma2_rn(r2, p, r);
+  const float2 ef = __fadd2_rn(make_float2(__int_as_float(0x4B400000 + (int)(ba >> 23) - 127),
+                                           __int_as_float(0x4B400000 + (int)(bb >> 23) - 127)),
+                               f2(-12582912.0f));
+  const float2 hi = __ffma2_rn(ef, f2(ASMV_LN2_HI), make_float2(ta.y, tb.y));
+  const float2 lo = __ffma2_rn(ef, f2(ASMV_LN2_LO), make_float2(ta.z, tb.z));
+  const float2 l = __fadd2_rn(hi, __fadd2_rn(lo, lp));
+  // radius: sqrt_radius of -2 ln(u) per lane
+  const float2 x = __fmul2_rn(f2(-2.0f), l);
+  const float2 rs = make_float2(rsqrtf(x.x), rsqrtf(x.y));
+  const float2 s = __fmul2_rn(x, rs);
+  const float2 e = __ffma2_rn(make_float2(-s.x, -s.y), s, x);
+  const float2 y = __ffma2_rn(e, __fmul2_rn(f2(0.5f), rs), s);
+  const float2 rho = make_float2(x.x == 0.0f ? x.x : y.x, x.y == 0.0f ? x.y : y.y);
+  // sin and cos of 2 pi k 2^-24, k = w >> 8
+  const uint32_t kc = w.y >> 8, kd = w.w >> 8;
+  const uint32_t qa = (kc + (1u << 21)) >> 22, qb = (kd + (1u << 21)) >> 22;
+  const int32_t ra = (int32_t)kc - (int32_t)(qa << 22), rb = (int32_t)kd - (int32_t)(qb << 22);
+  const float2 t = __fadd2_rn(make_float2(__int_as_float(0x40400000 + ra), __int_as_float(0x40400000 + rb)),
+                              f2(-3.0f));
+  const float2 t2 = __fmul2_rn(t, t);
+  float2 sp = __ffma2_rn(t2, f2(ASMV_S9), f2(ASMV_S7));
+  sp = __ffma2_rn(t2, sp, f2(ASMV_S5));
+  sp = __ffma2_rn(t2, sp, f2(ASMV_S3));
+  sp = __ffma2_rn(t2, sp, f2(ASMV_S1));
+  const float2 sv = __fmul2_rn(t, sp);
+  float2 cp = __ffma2_rn(t2, f2(ASMV_C10), f2(ASMV_C8));
+  cp = __ffma2_rn(t2, cp, f2(ASMV_C6));
+  cp = __ffma2_rn(t2, cp, f2(ASMV_C4));
+  cp = __ffma2_rn(t2, cp, f2(ASMV_C2));
+  const float2 cv = __ffma2_rn(t2, cp, f2(1.0f));
+  // quarter turn q: (sin, cos) = (s, c), (c, -s), (-s, -c), (-c, s)
+  const float sa = (qa & 1u) ? cv.x : sv.x, ca = (qa & 1u) ? sv.x : cv.x;
+  const float sb = (qb & 1u) ? cv.y : sv.y, cb = (qb & 1u) ? sv.y : cv.y;
+  const float2 sn = make_float2(__uint_as_float(__float_as_uint(sa) ^ ((qa & 2u) << 30)),
+                                __uint_as_float(__float_as_uint(sb) ^ ((qb & 2u) << 30)));
+  const float2 cs = make_float2(__uint_as_float(__float_as_uint(ca) ^ (((qa + 1u) & 2u) << 30)),
+                                __uint_as_float(__float_as_uint(cb) ^ (((qb + 1u) & 2u) << 30)));
+  z0 = __fmul2_rn(rho, cs);
+  z1 = __fmul2_rn(rho, sn);
+}
+
+// ---------------------------------------------------------------- encoders
+// Hardware round-to-nearest-even conversions (fp8: saturating to +-448).
+// (one packed conversion per pair; a goes to the low half)
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t *>(&v);
+}
+__device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
+  const __half2 v = __floats2half2_rn(a, b);
+  return *reinterpret_cast<const uint32_t *>(&v);
+}
+__device__ __forceinline__ uint32_t pack_f8x4(float a, float b, float c, float d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c, d), __NV_SATFINITE, __NV_E4M3);
+  return (lo & 0xFFFFu) | (hi << 16);
+}
+
+// OCP E5M2: hardware conversion, saturating at +-57344.
+__device__ __forceinline__ uint32_t pack_e5m2x4(float a, float b, float c, float d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E5M2);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c, d), __NV_SATFINITE, __NV_E5M2);
+  return (lo & 0xFFFFu) | (hi << 16);
+}
+
+// The fnuz formats hold half the value of the OCP format with the same bits
+// (bias one higher), except that they are finite at the top exponent, have
+// no negative zero and keep 0x80 for NaN.  So x is converted as 2x by the
+// hardware (round to nearest even), then:
+//   NaN -> 0x80; a zero result -> +0;
+//   E4M3FNUZ: above 232 (halfway between 224 and the top value 240) -> 240
+//     (0x7F, a NaN in the OCP format);
+//   E5M2FNUZ: from 30720 (halfway between 28672 and 32768) the top binade
+//     (4..7) * 8192 is chosen directly, nearest with ties to even, capped at
+//     57344 -- values the OCP format holds as Inf and NaN.
+__device__ __forceinline__ uint32_t enc_e4m3fnuz(float x) {
+  const float ax = fabsf(x);
+  const uint32_t sign = (__float_as_uint(x) >> 24) & 0x80u;
+  if (isnan(x)) return 0x80u;
+  if (ax > 232.0f) return sign | 0x7Fu;
+  const uint32_t b =
+      __nv_cvt_float2_to_fp8x2(make_float2(__fmul_rn(x, 2.0f), 0.0f), __NV_SATFINITE, __NV_E4M3) & 0xFFu;
+  return (b & 0x7Fu) ? b : 0u;
+}
+__device__ __forceinline__ uint32_t enc_e5m2fnuz(float x) {
+  const float ax = fabsf(x);
+  const uint32_t sign = (__float_as_uint(x) >> 24) & 0x80u;
+  if (isnan(x)) return 0x80u;
+  if (ax >= 30720.0f) {
+    const int q = min(__float2int_rn(__fmul_rn(fminf(ax, 1e9f), 0x1p-13f)), 7);
+    return sign | 0x7Cu | (uint32_t)(q - 4);
+  }
+  const uint32_t b =
+      __nv_cvt_float2_to_fp8x2(make_float2(__fmul_rn(x, 2.0f), 0.0f), __NV_SATFINITE, __NV_E5M2) & 0xFFu;
+  return (b & 0x7Fu) ? b : 0u;
+}
+
+}  // namespace asmv

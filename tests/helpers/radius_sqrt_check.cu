@@ -4,7 +4,7 @@
 // there are none.  Built and run by tests/test_gpu_parity.py.
 #include <cstdio>
 #include <cuda_runtime.h>
-#include "device.cuh"
+#include "fill_math.cuh"
 #include "ln_table.h"
 
 __global__ void check(unsigned long long *bad, unsigned int *first) {
