@@ -28,6 +28,11 @@ DTYPE_CODE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32
 DIST_CODE = {"raw": DIST_RAW, "uniform": DIST_UNIFORM, "normal": DIST_NORMAL,
              "int_range": DIST_INT_RANGE, "none": DIST_NONE}
 OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM = 0, -1, -2, -3, -4
+
+
+def dtype_code(dtype) -> int:
+    """The ABI code of a dtype name (or a code, returned as is)."""
+    return DTYPE_CODE[dtype] if isinstance(dtype, str) else int(dtype)
 U64_NONE = (1 << 64) - 1
 
 
@@ -86,7 +91,9 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_compare_noalloc", "asmv_compare_eq", "asmv_exact_to_double",
                  "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches",
                  "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
-                 "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds")
+                 "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds",
+                 "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base")
+EQ_DIGITS = 20                           # signed 64-bit digits per exact Eq. 1 sum
 NOALLOC_SCRATCH_BYTES = 1 << 20
 WAIT_ROUNDS = 20000                      # default bound of the compare's device waits
 
@@ -131,6 +138,11 @@ def lib():
         L.asmv_compare_noalloc.argtypes = [RP, RP, sz, TP, SP, vp]
         L.asmv_compare_eq.argtypes = [vp, RP, ctypes.POINTER(RP), sz, sz, TP, ctypes.c_double,
                                       ctypes.c_double, SP, ctypes.POINTER(EqResult), vp]
+        i64p = ctypes.POINTER(ctypes.c_int64)
+        L.asmv_compare_eq_digits.argtypes = [vp, RP, ctypes.POINTER(RP), sz, sz, TP, SP, i64p, vp]
+        L.asmv_eq_from_digits.argtypes = [ctypes.POINTER(ctypes.c_uint32), sz, sz, SP, i64p,
+                                          ctypes.c_double, ctypes.c_double, ctypes.POINTER(EqResult)]
+        L.asmv_eq_digit_base.argtypes = [ctypes.c_uint32, ctypes.POINTER(ctypes.c_int)]
         L.asmv_exact_to_double.argtypes = [ctypes.POINTER(ctypes.c_int64), ctypes.c_int,
                                            ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
         dp = ctypes.POINTER(ctypes.c_double)
@@ -385,6 +397,67 @@ class Context:
         eqs = [{f: getattr(eq[x], f) for f in EQ_FIELDS} for x in range(k * n)]
         return ([flat[j * n:(j + 1) * n] for j in range(k)],
                 [eqs[j * n:(j + 1) * n] for j in range(k)])
+
+    def compare_eq_digits(self, ref: Sequence, cands: Sequence[Sequence], tol, stream=None):
+        """asmv_compare_eq_digits: (stats, digits) with stats[j][i] as
+        compare_batched and digits[i, slot, d] the unrounded Eq. 1 sums
+        (int64, shape (n, 1 + 2k, EQ_DIGITS)): the per-shard result of a
+        check split across processes (see eq_from_digits)."""
+        n, k = len(ref), len(cands)
+        ra = region_array(ref)
+        cas = [region_array(c) for c in cands]
+        ptrs = (ctypes.POINTER(Region) * max(1, k))(*[ctypes.cast(c, ctypes.POINTER(Region))
+                                                      for c in cas])
+        st = (Stats * max(1, k * n))()
+        dig = np.zeros(max(1, n * (1 + 2 * k) * EQ_DIGITS), np.int64)
+        self._check(self._lib.asmv_compare_eq_digits(
+            self._h, ra, ptrs, k, n,
+            tol_array(tol) if not isinstance(tol, ctypes.Array) else tol,
+            st, dig.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), _stream_handle(stream)))
+        flat = stats_dicts(st, k * n)
+        return ([flat[j * n:(j + 1) * n] for j in range(k)],
+                dig[:n * (1 + 2 * k) * EQ_DIGITS].reshape(n, 1 + 2 * k, EQ_DIGITS))
+
+
+def stats_array(stats: Sequence[dict]) -> ctypes.Array:
+    """asmv_stats entries from statistics dicts (as stats_dicts returns them)."""
+    arr = (Stats * max(1, len(stats)))()
+    for i, d in enumerate(stats):
+        for f in STATS_FIELDS:
+            setattr(arr[i], f, d[f])
+    return arr
+
+
+def eq_from_digits(dtypes: Sequence, stats: Sequence[Sequence[dict]], digits: np.ndarray,
+                   theta: float = None, tau: float = None) -> List[List[dict]]:
+    """asmv_eq_from_digits: eq[j][i] of candidate j on region i from
+    statistics stats[j][i] and the digit vectors digits[i, slot, d] (as
+    Context.compare_eq_digits returns them, possibly summed over shards).
+    Host only."""
+    theta = THETA if theta is None else theta
+    tau = TAU if tau is None else tau
+    n, k = len(dtypes), len(stats)
+    codes = (ctypes.c_uint32 * max(1, n))(*[dtype_code(d) for d in dtypes])
+    st = stats_array([s for row in stats for s in row])
+    dig = np.ascontiguousarray(np.asarray(digits, dtype=np.int64).reshape(-1))
+    if dig.size != n * (1 + 2 * k) * EQ_DIGITS:
+        raise ValueError("digits must have shape (n, 1 + 2k, %d)" % EQ_DIGITS)
+    out = (EqResult * max(1, k * n))()
+    rc = lib().asmv_eq_from_digits(codes, k, n, st, dig.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                                   float(theta), float(tau), out)
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    eqs = [{f: getattr(out[x], f) for f in EQ_FIELDS} for x in range(k * n)]
+    return [eqs[j * n:(j + 1) * n] for j in range(k)]
+
+
+def eq_digit_base(dtype) -> int:
+    """asmv_eq_digit_base: the binary weight of digit 0 of a float dtype's sums."""
+    out = ctypes.c_int()
+    rc = lib().asmv_eq_digit_base(dtype_code(dtype), ctypes.byref(out))
+    if rc != OK:
+        raise AsmvError(rc, strerror(rc))
+    return out.value
 
 
 def exact_to_double(digits: Sequence[int], base_exp: int) -> float:

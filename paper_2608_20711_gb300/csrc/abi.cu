@@ -28,6 +28,7 @@ static_assert(sizeof(asmv_eq) == 40, "asmv_eq layout");
 static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
 static_assert(sizeof(CopyRegion) == 48, "copy region layout");
 static_assert(kWaitRounds == ASMV_WAIT_ROUNDS, "default wait bound");
+static_assert(kEqDigits == ASMV_EQ_DIGITS, "Eq. 1 digits");
 static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
               "plan layouts");
 
@@ -799,13 +800,16 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   return ASMV_OK;
 }
 
-int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
-                    size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
-                    asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// Validation shared by asmv_compare_eq and asmv_compare_eq_digits.
+int check_eq_call(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands, size_t k,
+                  size_t n, const asmv_tol *tol, const void *stats_host, const void *out_host) {
   if (ctx == nullptr || k == 0 || cands == nullptr || !tol_ok(tol) ||
-      (n > 0 && (stats_host == nullptr || eq_host == nullptr)))
+      (n > 0 && (stats_host == nullptr || out_host == nullptr)))
     return ASMV_EINVAL;
-  if (!std::isfinite(theta) || !std::isfinite(tau) || tau < 0.0) return ASMV_EINVAL;
   if (k > (size_t)0x7FFFFFFF / (n ? n : 1)) return ASMV_EINVAL;
   int rc = check_pairs(ref, cands, k, n);
   if (rc != ASMV_OK) return rc;
@@ -813,37 +817,59 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
     if (is_float(ref[i].dtype) &&
         (ref[i].dtype == ASMV_F64 || ref[i].n_elems > ((uint64_t)1 << 31)))
       return ASMV_EINVAL;
-  if (n == 0) return ASMV_OK;
+  return ASMV_OK;
+}
+
+// The statistics and the digit vectors of the Eq. 1 sums (the kernels).
+int run_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands, size_t k,
+                   size_t n, const asmv_tol *tol, asmv_stream_t stream, std::vector<asmv_stats> &stats,
+                   std::vector<long long> &digits) {
   DeviceScope ds(ctx->device);
   if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
   const cudaStream_t s = (cudaStream_t)stream;
-  std::vector<asmv_stats> stats(k * n);
+  stats.assign(k * n, asmv_stats());
+  int rc;
   if ((rc = run_compare(ctx, ref, cands, k, n, tol, stats.data(), s, false)) != ASMV_OK) return rc;
-  std::vector<long long> digits;
-  if ((rc = run_eq(ctx, ref, cands, k, n, s, digits)) != ASMV_OK) return rc;
-  std::vector<asmv_eq> res(k * n);
+  return run_eq(ctx, ref, cands, k, n, s, digits);
+}
+
+// Eq. 1 of every (candidate, region) from statistics and digit vectors: the
+// three sums rounded once each, the cosine and the four terms.  The digit
+// vectors of the difference-form dtypes hold sum r d and sum d^2, from which
+// S_rc = S_rr + sum r d and S_cc = S_rr + 2 sum r d + sum d^2, digit by
+// digit; a digit sum that would leave the int64 range is rejected.
+int eq_combine(const uint32_t *dtypes, size_t k, size_t n, const asmv_stats *stats,
+               const long long *digits, double theta, double tau, asmv_eq *res) {
   const size_t nslots = 1 + 2 * k;
   for (size_t j = 0; j < k; ++j) {
     for (size_t i = 0; i < n; ++i) {
       const asmv_stats &st = stats[j * n + i];
       asmv_eq &q = res[j * n + i];
       std::memset(&q, 0, sizeof q);
-      const bool flt = is_float(ref[i].dtype);
+      const bool flt = is_float(dtypes[i]);
       if (flt) {
-        const long long *d = digits.data() + i * nslots * kEqDigits;
-        const int base = eq_digit_base(ref[i].dtype);
+        const long long *d = digits + i * nslots * kEqDigits;
+        const int base = eq_digit_base(dtypes[i]);
         int64_t rc[kEqDigits], cc[kEqDigits];
         const long long *rr = d, *s1 = d + (1 + 2 * j) * kEqDigits, *s2 = d + (2 + 2 * j) * kEqDigits;
-        const bool diff = eq_difference_form(ref[i].dtype);
-        for (int k = 0; k < kEqDigits; ++k) {
-          // digits stay far below 2^61, so these sums cannot overflow
-          rc[k] = diff ? (int64_t)rr[k] + s1[k] : s1[k];
-          cc[k] = diff ? (int64_t)rr[k] + 2 * (int64_t)s1[k] + s2[k] : s2[k];
+        const bool diff = eq_difference_form(dtypes[i]);
+        for (int m = 0; m < kEqDigits; ++m) {
+          if (diff) {
+            long long a, b, c;
+            if (__builtin_add_overflow(rr[m], s1[m], &a) || __builtin_add_overflow(a, s1[m], &b) ||
+                __builtin_add_overflow(b, s2[m], &c))
+              return ASMV_EINVAL;
+            rc[m] = a;
+            cc[m] = c;
+          } else {
+            rc[m] = s1[m];
+            cc[m] = s2[m];
+          }
         }
         if (exact_to_double_impl(rc, kEqDigits, base, &q.sum_rc) != ASMV_OK ||
             exact_to_double_impl((const int64_t *)rr, kEqDigits, base, &q.sum_rr) != ASMV_OK ||
             exact_to_double_impl(cc, kEqDigits, base, &q.sum_cc) != ASMV_OK)
-          return ASMV_ECUDA;                         // digits out of range: a device fault
+          return ASMV_EINVAL;
         q.cos = eq_cosine(q.sum_rc, q.sum_rr, q.sum_cc);
       } else {
         q.cos = NAN;
@@ -857,8 +883,70 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
       q.eq = f == (ASMV_EQ_COS | ASMV_EQ_LINF | ASMV_EQ_INT | ASMV_EQ_GUARD);
     }
   }
+  return ASMV_OK;
+}
+
+bool theta_tau_ok(double theta, double tau) {
+  return std::isfinite(theta) && std::isfinite(tau) && tau >= 0.0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                    size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
+                    asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream) {
+  int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, eq_host);
+  if (rc != ASMV_OK) return rc;
+  if (!theta_tau_ok(theta, tau)) return ASMV_EINVAL;
+  if (n == 0) return ASMV_OK;
+  std::vector<asmv_stats> stats;
+  std::vector<long long> digits;
+  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits)) != ASMV_OK) return rc;
+  std::vector<uint32_t> dt(n);
+  for (size_t i = 0; i < n; ++i) dt[i] = ref[i].dtype;
+  std::vector<asmv_eq> res(k * n);
+  if (eq_combine(dt.data(), k, n, stats.data(), digits.data(), theta, tau, res.data()) != ASMV_OK)
+    return ASMV_ECUDA;                                // digits out of range: a device fault
   std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
   std::memcpy(eq_host, res.data(), res.size() * sizeof(asmv_eq));
+  return ASMV_OK;
+}
+
+int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
+                           size_t k, size_t n, const asmv_tol *tol, asmv_stats *stats_host,
+                           int64_t *digits_host, asmv_stream_t stream) {
+  int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, digits_host);
+  if (rc != ASMV_OK) return rc;
+  if (n == 0) return ASMV_OK;
+  std::vector<asmv_stats> stats;
+  std::vector<long long> digits;
+  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits)) != ASMV_OK) return rc;
+  std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
+  std::memcpy(digits_host, digits.data(), digits.size() * sizeof(int64_t));
+  return ASMV_OK;
+}
+
+int asmv_eq_from_digits(const uint32_t *dtypes, size_t k, size_t n, const asmv_stats *stats,
+                        const int64_t *digits, double theta, double tau, asmv_eq *eq_out) {
+  if (k == 0 || !theta_tau_ok(theta, tau)) return ASMV_EINVAL;
+  if (n == 0) return ASMV_OK;
+  if (dtypes == nullptr || stats == nullptr || digits == nullptr || eq_out == nullptr) return ASMV_EINVAL;
+  if (k > (size_t)0x7FFFFFFF / n) return ASMV_EINVAL;
+  for (size_t i = 0; i < n; ++i)
+    if (dtypes[i] >= (uint32_t)ASMV_NDTYPES || dtypes[i] == ASMV_F64) return ASMV_EINVAL;
+  std::vector<asmv_eq> res(k * n);
+  int rc = eq_combine(dtypes, k, n, stats, (const long long *)digits, theta, tau, res.data());
+  if (rc != ASMV_OK) return rc;
+  std::memcpy(eq_out, res.data(), res.size() * sizeof(asmv_eq));
+  return ASMV_OK;
+}
+
+int asmv_eq_digit_base(uint32_t dtype, int *base) {
+  if (base == nullptr || dtype >= (uint32_t)ASMV_NDTYPES || !is_float(dtype) || dtype == ASMV_F64)
+    return ASMV_EINVAL;
+  *base = eq_digit_base(dtype);
   return ASMV_OK;
 }
 

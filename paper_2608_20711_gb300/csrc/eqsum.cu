@@ -288,6 +288,17 @@ __device__ __forceinline__ Limbs fix_f16_biased(uint32_t b) {
   return {__float_as_int(hf), __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic))};
 }
 
+// fix_f16_biased for the two fp16 values of a word (low half first), on
+// packed fp32: each lane rounds exactly as the scalar form.
+__device__ __forceinline__ void fix_f16x2_biased(uint32_t w, Limbs &a, Limbs &b) {
+  const float2 x = __half22float2(*reinterpret_cast<const __half2 *>(&w));
+  const float2 hf = __ffma2_rn(x, make_float2(16.0f, 16.0f), make_float2(kMagic, kMagic));
+  const float2 l = __ffma2_rn(__fadd2_rn(hf, make_float2(-kMagic, -kMagic)), make_float2(-0.0625f, -0.0625f), x);
+  const float2 lo = __ffma2_rn(l, make_float2(16777216.0f, 16777216.0f), make_float2(kMagic, kMagic));
+  a = {__float_as_int(hf.x), __float_as_int(lo.x)};
+  b = {__float_as_int(hf.y), __float_as_int(lo.y)};
+}
+
 // A pair of fp16 values with the non-finite ones replaced by zero: x - x is
 // zero exactly for finite x and a NaN for an infinity or a NaN.
 __device__ __forceinline__ uint32_t finite_f16x2(uint32_t w) {
@@ -461,12 +472,21 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
         rv = finite_f16x8(rv);
         v0 = finite_f16x8(v0);
         v1 = finite_f16x8(v1);
+        const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+        const uint32_t w0[4] = {v0.x, v0.y, v0.z, v0.w};
+        const uint32_t w1[4] = {v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const Limbs xb = fix_f16_biased(half_of(rv, k));
-          const Limbs x = {xb.hi - kMagicBits, xb.lo - kMagicBits};
-          diff_add(rc0, cc0, x, xb, fix_f16_biased(half_of(v0, k)));
-          diff_add(rc1, cc1, x, xb, fix_f16_biased(half_of(v1, k)));
+        for (int q = 0; q < 4; ++q) {
+          Limbs xb[2], y0[2], y1[2];
+          fix_f16x2_biased(rw[q], xb[0], xb[1]);
+          fix_f16x2_biased(w0[q], y0[0], y0[1]);
+          fix_f16x2_biased(w1[q], y1[0], y1[1]);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const Limbs x = {xb[h].hi - kMagicBits, xb[h].lo - kMagicBits};
+            diff_add(rc0, cc0, x, xb[h], y0[h]);
+            diff_add(rc1, cc1, x, xb[h], y1[h]);
+          }
         }
       } else if (DT != kF8) {
 #pragma unroll

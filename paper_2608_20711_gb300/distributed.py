@@ -9,6 +9,11 @@ the split.  This module does the host side of that: slice regions by rank,
 shift indices back to region coordinates, and all-reduce the statistics
 with torch.distributed (any backend; the tests use gloo on CPU).
 
+The exact sums behind Eq. 1's cosine split the same way: every process
+returns its sums as unrounded digit vectors (asmv_compare_eq_digits), the
+vectors are added over the processes, and the verdict is formed once from
+the total (asmv_eq_from_digits), so the cosine is that of the whole region.
+
 Guard bands belong to whole allocations: the slice that starts the
 payload keeps the low band, the slice that ends it keeps the high band,
 and every other slice carries none, so each guard byte is checked once.
@@ -128,3 +133,31 @@ def allreduce_stats(per_region: Sequence[Dict], group=None) -> List[Dict]:
             "ref_guard_bad_bytes": int(sums[i, 3]),
         })
     return out
+
+
+def normalize_digits(digits, ndigits: int = 20):
+    """Carry every digit vector along its last axis so that each digit but
+    the top one lies in [0, 2^32) (the integer it represents is unchanged):
+    a sum over many processes then keeps every digit far inside int64."""
+    import numpy as np
+    d = np.asarray(digits, dtype=np.int64)
+    flat = d.reshape(-1, ndigits)
+    out = np.zeros_like(flat)
+    for r in range(flat.shape[0]):
+        v = sum(int(flat[r, k]) << (32 * k) for k in range(ndigits))
+        for k in range(ndigits - 1):
+            out[r, k] = (v >> (32 * k)) & 0xFFFFFFFF
+        out[r, ndigits - 1] = v >> (32 * (ndigits - 1))
+    return out.reshape(d.shape)
+
+
+def allreduce_digits(digits, group=None):
+    """Sum the Eq. 1 digit vectors of every rank (numpy int64, the same
+    shape on every rank), after normalising them: the exact sums of the
+    whole split check."""
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    t = torch.from_numpy(np.ascontiguousarray(normalize_digits(digits)))
+    dist.all_reduce(t, op=dist.ReduceOp.SUM, group=group)
+    return t.numpy()

@@ -117,3 +117,61 @@ def test_merge_is_order_independent():
     for p in reversed(parts):
         b = D.merge_stats(p, b)
     assert a == b == _region_stats(O, ref, cand, r, 0, r)
+
+
+def _eq_worker(rank, world, port, out):
+    """Each rank: its element range of every float region, as unrounded Eq. 1
+    digit vectors (built from the oracle's exact sums, in the library's
+    layout) and statistics; both all-reduced."""
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        from oracle import oracle as O
+        from tests.test_eq_digits import full_stats, shard_digits
+        regs, ref, cand = _workload()
+        flt = [r for r in regs if r.dtype in W.FLOAT_DTYPES]
+        digs, parts = [], []
+        for r in flt:
+            a, b = D.slice_bounds(r.n_elems, W.DTYPE_SIZE[r.dtype], rank, world)
+            off = r.payload_offset
+            rp, cp = ref[off:off + r.payload_bytes], cand[off:off + r.payload_bytes]
+            digs.append(shard_digits(O, rp, [cp], r.dtype, a, b))
+            t = TOL[r.dtype]
+            parts.append(D.to_region_coordinates(full_stats(O, rp, cp, r.dtype, a, b, t), a, 0))
+        merged_digits = D.allreduce_digits(np.stack(digs))
+        merged_stats = D.allreduce_stats(parts)
+        if rank == 0:
+            out.put((merged_digits, merged_stats))
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world", [2])
+def test_sharded_eq1_verdict_is_exact(world):
+    """Eq. 1 of regions split over gloo ranks, formed once from the summed
+    digit vectors, equals the oracle's verdict on the whole regions."""
+    from oracle import oracle as O
+    from paper_2608_20711_gb300 import asmv
+    from tests.test_eq_digits import ONAME, full_stats
+    regs, ref, cand = _workload()
+    flt = [r for r in regs if r.dtype in W.FLOAT_DTYPES]
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_eq_worker, args=(k, world, port, q)) for k in range(world)]
+    for p in procs:
+        p.start()
+    digits, stats = q.get(timeout=240)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    got = asmv.eq_from_digits([r.dtype for r in flt], [stats], digits)[0]
+    for r, g in zip(flt, got):
+        off = r.payload_offset
+        rp, cp = ref[off:off + r.payload_bytes], cand[off:off + r.payload_bytes]
+        code = getattr(O, ONAME[r.dtype])
+        whole = full_stats(O, rp, cp, r.dtype, 0, r.n_elems, TOL[r.dtype])
+        want = O.eq_verdict(whole, O.eq_sums(rp, cp, code, r.n_elems), code)
+        for f in ("sum_rc", "sum_rr", "sum_cc", "cos", "flags", "eq"):
+            assert g[f] == want[f], (r.name, f)

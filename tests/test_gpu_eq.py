@@ -246,3 +246,62 @@ def test_eq_batched_gemm_full(ctx, oracle):
         assert_stats_equal(stats[j][0], st, "candidate %d" % j)
         assert_stats_equal(eqs[j][0], want, "candidate %d" % j)
         del ch
+
+
+def test_eq_split_over_shards_equals_whole(ctx, oracle):
+    """A check split into element ranges (as processes of a multi-GPU run
+    would take them): the digit vectors of asmv_compare_eq_digits summed
+    over three shards and the merged statistics give, through
+    asmv_eq_from_digits, exactly the result of asmv_compare_eq on the whole
+    regions -- every float dtype, a mixed table, three candidates."""
+    from paper_2608_20711_gb300 import distributed as D
+    dts = ("f32", "bf16", "f16", "f8e4m3", "f8e5m2", "f8e4m3fnuz", "f8e5m2fnuz", "i32", "u8")
+    rng = np.random.default_rng(13)
+    regs = []
+    for rid, dt in enumerate(dts):
+        n = (3 * TILE + 4099) // W.DTYPE_SIZE[dt] + int(rng.integers(0, 40))
+        dist, p0, p1 = {"i32": ("int_range", 0, 1000), "u8": ("raw", 0, 0)}.get(dt, ("normal", 0.0, 1.0))
+        regs.append(W.Region("r%d" % rid, dt, n, dist, p0, p1, 64, 64, 0xA5, rid))
+    nbytes = _layout(regs)
+    ref = oracle_fill_arena(oracle, regs, nbytes, seed=12)
+    for r in regs:
+        if r.dtype in W.FLOAT_DTYPES:
+            _plant_specials(ref, r, rng)
+    cands = []
+    for j in range(3):
+        c = ref.copy()
+        for r in regs:
+            if W.DTYPE_SIZE[r.dtype] in (1, 2, 4):
+                _perturb(c, ref, r, rng, j)
+        cands.append(c)
+    dref = to_device(ref)
+    dc = [to_device(c) for c in cands]
+    rr = asmv.regions_in_arena(regs, dref.data_ptr())
+    cc = [asmv.regions_in_arena(regs, d.data_ptr()) for d in dc]
+    whole_stats, whole_eq = ctx.compare_eq(rr, cc, W.DEFAULT_TOL)
+    world = 3
+    digits = 0
+    stats = [[D.empty_stats() for _ in regs] for _ in cands]
+    for rank in range(world):
+        sr, firsts, shifts = [], [], []
+        for r in rr:
+            s, first, shift = D.shard_region(r, W.DTYPE_SIZE[regs[len(sr)].dtype], rank, world)
+            sr.append(s)
+            firsts.append(first)
+            shifts.append(shift)
+        sc = []
+        for c in cc:
+            sc.append([D.shard_region(r, W.DTYPE_SIZE[regs[i].dtype], rank, world)[0]
+                       for i, r in enumerate(c)])
+        st, dig = ctx.compare_eq_digits(sr, sc, W.DEFAULT_TOL)
+        digits = digits + D.normalize_digits(dig)
+        for j in range(len(cands)):
+            for i in range(len(regs)):
+                stats[j][i] = D.merge_stats(stats[j][i],
+                                            D.to_region_coordinates(st[j][i], firsts[i], shifts[i]))
+    got = asmv.eq_from_digits([r.dtype for r in regs], stats, digits)
+    for j in range(len(cands)):
+        for i, r in enumerate(regs):
+            where = "cand %d region %s (%s)" % (j, r.name, r.dtype)
+            assert_stats_equal(stats[j][i], whole_stats[j][i], where)
+            assert_stats_equal(got[j][i], whole_eq[j][i], where)
