@@ -258,15 +258,16 @@ def _timed_until(budget_s, fn, n0, nmax):
     return n, total_t, total_w
 
 
-def cpu_oracle_sample(setup, budget_s=12.0):
-    """The oracle as it stands, on the host cores, over a bounded sample of
-    the same workload: element prefixes of the fill regions (one of each
-    dtype/distribution kind) and of the reference/candidate payloads.  The
-    two measured rates are combined over the step's byte mix."""
+def cpu_oracle_sample(setup, budget_s=12.0, threads=None):
+    """The oracle as it stands, on the host cores (all of them unless
+    `threads` is given), over a bounded sample of the same workload: element
+    prefixes of the fill regions (one of each dtype/distribution kind) and
+    of the reference/candidate payloads.  The two measured rates are
+    combined over the step's byte mix."""
     from oracle import oracle as O
     ORACLE_DTYPE, ORACLE_DIST = O.CODE_OF_DTYPE, O.CODE_OF_DIST
     W = setup.W
-    threads = O.host_threads()
+    threads = O.host_threads() if threads is None else int(threads)
     kinds = {}
     for r in setup.fill_specs:
         kinds.setdefault((r.dtype, r.dist), r)
@@ -433,6 +434,9 @@ def run_mine(args):
         line["restore"] = run_restore(setup, args, peak)
     if rank == 0 and world == 1 and args.cpu:
         line["cpu_baseline"] = cpu_oracle_sample(setup)
+        one = cpu_oracle_sample(setup, budget_s=4.0, threads=1)
+        line["cpu_baseline"]["single_thread"] = {k: one[k] for k in ("value", "fill_gbs", "verify_gbs",
+                                                                      "seconds")}
     if rank == 0:
         mism = sum(int(s["mismatches"]) for cs in stats for s in cs)
         line["check"] = {"total_mismatches": mism}
