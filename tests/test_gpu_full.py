@@ -175,3 +175,32 @@ def test_batched_gemm_fp16_full(ctx, oracle):
         if wl.ulp_magnitudes[j] == 0:
             assert want["mismatches"] == 0 and want["max_abs_err"] == 0.0
         del ch
+
+
+def test_region_beyond_2_pow_32_elements(ctx, oracle):
+    """One fp16 NORMAL region of 2^32 + 1029 elements (8 GiB): element
+    indices and byte offsets past 2^32.  The GPU fill matches the oracle
+    on sampled ranges including the tail; a compare whose reference is the
+    oracle's own fill and whose candidate carries mismatches on both sides
+    of element 2^32 gives the oracle's statistics (count, first index,
+    exact maxima, guard damage past byte 2^33)."""
+    n = (1 << 32) + 1029
+    r = W.Region("big", "f16", n, "normal", 0.0, 1.0, 512, 4096, 0x5A, 3)
+    r.offset = 0
+    size = r.alloc_bytes + 64
+    seed = 31
+    torch = torch_cuda()
+    dev = torch.zeros(size, dtype=torch.uint8, device="cuda")
+    ctx.fill(asmv.regions_in_arena([r], dev.data_ptr()), seed=seed)
+    torch.cuda.synchronize()
+    _sampled_fill_check(oracle, None, [r], dev, seed, samples=4)
+    del dev
+    torch.cuda.empty_cache()
+    ref = oracle_fill_arena(oracle, [r], size, seed)
+    cand = ref.copy()
+    pay = cand[r.payload_offset:r.payload_offset + r.payload_bytes].view(np.uint16)
+    pos = np.array([5, 1 << 31, (1 << 32) - 1, 1 << 32, (1 << 32) + 7, n - 1], np.int64)
+    pay[pos] ^= np.array([1, 0x40, 2, 0x300, 1, 0x7C00], np.uint16)
+    cand[r.payload_offset + r.payload_bytes + 4000] ^= 0xFF          # high guard, past 2^33 bytes
+    import types
+    _check_compare(ctx, oracle, types.SimpleNamespace(tol=W.DEFAULT_TOL), ref, cand, regions=[r])
