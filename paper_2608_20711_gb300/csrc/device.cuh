@@ -15,12 +15,6 @@ namespace asmv {
 __device__ __forceinline__ float2 f16x2_to_f32(uint32_t w) {
   return __half22float2(*reinterpret_cast<const __half2 *>(&w));
 }
-__device__ __forceinline__ float2 f8x2_to_f32(uint32_t w16) {
-  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(w16 & 0xFFFFu), __NV_E4M3);
-  uint32_t u = (uint32_t)h.x | ((uint32_t)h.y << 16);
-  return f16x2_to_f32(u);
-}
-
 // Two fp8 values (low byte first) as an exact half2, per format.  The fnuz
 // formats are half the value of the OCP format with the same bits, finite
 // at the top exponent (E4M3: 0x7F is 240; E5M2: exponent 31 holds

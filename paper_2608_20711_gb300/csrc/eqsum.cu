@@ -278,18 +278,11 @@ __device__ __forceinline__ Limbs fix_f16(uint32_t b) {
           __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic)) - kMagicBits};
 }
 
-// The same limbs, each plus kMagicBits, for a value known to be finite:
-// for a candidate only the differences of its limbs from the reference's
-// are used, so the offsets cancel and need no subtraction.
-__device__ __forceinline__ Limbs fix_f16_biased(uint32_t b) {
-  const float x = __half2float(__ushort_as_half((unsigned short)b));
-  const float hf = __fmaf_rn(x, 16.0f, kMagic);
-  const float l = __fmaf_rn(__fsub_rn(hf, kMagic), -0.0625f, x);
-  return {__float_as_int(hf), __float_as_int(__fmaf_rn(l, 16777216.0f, kMagic))};
-}
-
-// fix_f16_biased for the two fp16 values of a word (low half first), on
-// packed fp32: each lane rounds exactly as the scalar form.
+// The limbs of fix_f16, each plus kMagicBits, for the two fp16 values of
+// a word (low half first) known to be finite, on packed fp32 (each lane
+// rounds exactly as fix_f16's scalar steps).  For a candidate only the
+// differences of its limbs from the reference's are used, so the offsets
+// cancel and need no subtraction.
 __device__ __forceinline__ void fix_f16x2_biased(uint32_t w, Limbs &a, Limbs &b) {
   const float2 x = __half22float2(*reinterpret_cast<const __half2 *>(&w));
   const float2 hf = __ffma2_rn(x, make_float2(16.0f, 16.0f), make_float2(kMagic, kMagic));
@@ -319,13 +312,6 @@ __device__ __forceinline__ int fix_f8(uint32_t b) {
 
 __device__ __forceinline__ long long mad_wide(int a, int b, long long c) {
   return (long long)a * (long long)b + c;
-}
-
-__device__ __forceinline__ void mac(Acc3 &a, const Limbs &x, const Limbs &y) {
-  a.s2 = mad_wide(x.hi, y.hi, a.s2);
-  a.s1 = mad_wide(x.hi, y.lo, a.s1);
-  a.s1 = mad_wide(x.lo, y.hi, a.s1);
-  a.s0 = mad_wide(x.lo, y.lo, a.s0);
 }
 
 __device__ __forceinline__ void sq(Acc3 &a, const Limbs &x) {
