@@ -656,6 +656,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   for (size_t g = 0; g < groups; ++g) {
     const size_t kg = guard_only ? 1 : std::min<size_t>(kMaxCands, k - g * kMaxCands);
     p.K = (uint32_t)kg;
+    p.nstages = compare_stages(p.K, tile_bytes);
     p.cands = (const uint64_t *)(dev + o_cand) + g * kMaxCands * n;
     p.stats = (StatsDev *)(dev + o_stats) + g * kMaxCands * n;
     p.nsegs = (g == 0) ? (uint32_t)segs.size() : 0u;
@@ -1236,6 +1237,7 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   p.nsegs = (uint32_t)ks;
   p.K = 1;
   p.tile_bytes = tile_bytes;
+  p.nstages = compare_stages(1, tile_bytes);
   p.wait_rounds = kWaitRounds;
   for (int d = 0; d < ASMV_NDTYPES; ++d)
     if (is_float((uint32_t)d)) p.tol[d] = make_tolf(tol[d]);

@@ -45,7 +45,8 @@
 //
 // Work split: one CTA of 17 warps per SM.  The last warp streams each tile
 // of the reference and of the K <= 8 candidates into shared memory with
-// bulk copies (four stages, mbarrier-completed); the 16 checking warps are
+// bulk copies (two or four stages, as fit, mbarrier-completed; the kernel
+// is instantiated per depth); the 16 checking warps are
 // divided among the candidates, so device memory sees the reference once
 // per tile.  Chunks the screen cannot settle are queued per warp and
 // drained lane-parallel.  Each lane keeps its statistics in registers and
@@ -509,7 +510,8 @@ __device__ __noinline__ Hot tail_rows(const CmpRegion r, uint64_t cbase, const T
 // for every tile, wait for its stage, check chunks part*32 + lane + j*32*W
 // (staged chunks from shared memory, the rest from global), release the
 // stage.  One call per run of tiles keeps the per-tile cost to the waits.
-template <uint32_t DT>
+// NST is the launch's pipeline depth (stage u % NST, phase (u / NST) & 1).
+template <uint32_t DT, uint32_t NST>
 __device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, uint64_t t_end,
                                 const unsigned char *bufs, uint32_t stage_bytes, uint32_t cand_off,
                                 uint64_t *full, uint64_t *empty, uint32_t tile_bytes, uint32_t part,
@@ -521,8 +523,8 @@ __device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, u
   const uint32_t lane = threadIdx.x & 31;
   uint32_t u = cur->u;
   for (; t < t_end; ++t, ++u) {
-    const uint32_t s = u % kStages;
-    if (!mbar_wait(smem_addr(&full[s]), (u / kStages) & 1u, kWaitRounds)) { cur->ok = 0; break; }
+    const uint32_t s = u % NST;
+    if (!mbar_wait(smem_addr(&full[s]), (u / NST) & 1u, kWaitRounds)) { cur->ok = 0; break; }
     if (active) {
       const TileInfo ti = tile_info(r, t, tile_bytes);
       const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
@@ -556,13 +558,14 @@ __device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, u
   return h;
 }
 
+template <uint32_t NST>
 __device__ __forceinline__ Hot run_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
                                             uint64_t t, uint64_t t_end, const unsigned char *bufs,
                                             uint32_t stage_bytes, uint32_t cand_off, uint64_t *full,
                                             uint64_t *empty, uint32_t part, uint32_t W, bool active,
                                             Hot h, Queue *q, Cursor *cur) {
   const uint32_t TB = p.tile_bytes;
-#define ASMV_RUN(DT, TOL) run<DT>(r, cbase, t, t_end, bufs, stage_bytes, cand_off, full, empty, TB, \
+#define ASMV_RUN(DT, TOL) run<DT, NST>(r, cbase, t, t_end, bufs, stage_bytes, cand_off, full, empty, TB, \
                                   part, W, active, h, TOL, q, cur)
   switch (r.dtype) {
     case kF32: return ASMV_RUN(kF32, p.tol[kF32]);
@@ -615,10 +618,12 @@ __device__ void guard_phase(const CmpParams &p, uint32_t warp, uint32_t nwarps) 
 // holds the reference tile and the K candidate tiles (tile_bytes each);
 // full[s] completes when its bulk copies land, empty[s] when every
 // consumer warp has finished with it.
+template <uint32_t NST>
 __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams p) {
   extern __shared__ __align__(128) unsigned char smem[];
   uint64_t *full = reinterpret_cast<uint64_t *>(smem);
   uint64_t *empty = full + kStages;
+  constexpr uint32_t nst = NST;                              // pipeline depth, 2 or 4
   Queue *queues = reinterpret_cast<Queue *>(smem + 128);
   unsigned char *bufs = smem + 128 + kConsumerWarps * sizeof(Queue);
   const uint32_t K = p.K, TB = p.tile_bytes;
@@ -626,7 +631,7 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x < kConsumerWarps) queues[threadIdx.x].count = 0;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (uint32_t s = 0; s < nst; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
       mbar_init(smem_addr(&empty[s]), kConsumerWarps);
     }
@@ -643,9 +648,8 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
       uint32_t u = 0;
       for (uint64_t t = t0; t < t1 && ok; ++t, ++u) {
         while (p.regions[ri + 1].tile0 <= t) ++ri;
-        const uint32_t s = u % kStages;
-        if (u >= (uint32_t)kStages &&
-            !mbar_wait(smem_addr(&empty[s]), ((u / kStages) & 1u) ^ 1u, p.wait_rounds)) {
+        const uint32_t s = u % nst;
+        if (u >= nst && !mbar_wait(smem_addr(&empty[s]), ((u / nst) & 1u) ^ 1u, p.wait_rounds)) {
           ok = false;
           break;
         }
@@ -666,8 +670,8 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
       // gave up on a wait leave their stages unread.  Each stage's latest
       // phase is the one awaited; in a run without errors these have
       // completed already.
-      for (uint32_t v = (u >= (uint32_t)kStages ? u - kStages : 0); v < u; ++v)
-        mbar_wait(smem_addr(&full[v % kStages]), (v / kStages) & 1u, kWaitRounds);
+      for (uint32_t v = (u >= nst ? u - nst : 0); v < u; ++v)
+        mbar_wait(smem_addr(&full[v % nst]), (v / nst) & 1u, kWaitRounds);
     }
   } else if (t0 < t1) {
     // consumers: one call per run of tiles of the same region
@@ -685,8 +689,9 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
       while (p.regions[ri + 1].tile0 <= t) ++ri;
       const uint64_t t_end = umin64(t1, p.regions[ri + 1].tile0);
       const CmpRegion r = p.regions[ri];
-      h = run_dispatch(p, r, p.cands[(size_t)k * p.nregions + ri], t, t_end, bufs, stage_bytes,
-                       (1 + k) * TB, full, empty, part, W, active, h, &queues[warp], &cur);
+      const uint64_t cbase = p.cands[(size_t)k * p.nregions + ri];
+      h = run_dispatch<NST>(p, r, cbase, t, t_end, bufs, stage_bytes, (1 + k) * TB, full, empty,
+                            part, W, active, h, &queues[warp], &cur);
       t = t_end;
       if (active && cur.ok) flush(h, p, k, ri);
     }
@@ -697,24 +702,35 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
 
 }  // namespace
 
-size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes) {
-  return 128 + kConsumerWarps * sizeof(Queue) + (size_t)kStages * (1 + K) * tile_bytes;
+size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes, uint32_t nstages) {
+  return 128 + kConsumerWarps * sizeof(Queue) + (size_t)nstages * (1 + K) * tile_bytes;
 }
 
+// Tiles of a launch group of up to K candidates: 16 KiB for one candidate,
+// 8 KiB otherwise, over as many stages as fit (compare_stages).  Larger
+// tiles mean fewer per-tile waits and less bookkeeping per chunk.  On a
+// 1 GiB fp16 reference (GB/s of reference + candidates read):
+//   K            2     3     4     5     6     7     8
+//   before    3051  2911  2582  2265  2654  2768  3051   (4 KiB tiles from K = 4, 4 stages)
+//   now       3143  2958  2940  3089  3062  3167  3498
+// and with one candidate, 4 stages of 16 KiB beat 2 stages by a fifth.
+// Tiles of whole warp rows (no tail rows) were measured too: better at
+// K = 2, worse at K = 3 and 5.
 uint32_t compare_tile_bytes(uint32_t K) {
-  // stage = (1 + K) tiles; keep a stage near 32-36 KiB
-  if (K <= 1) return 16384;
-  if (K == 2) return 12288;
-  if (K == 3) return 8192;
-  return 4096;
+  return K <= 1 ? 16384u : 8192u;
+}
+
+// The deepest pipeline (4, else 2 stages) whose shared memory fits a CTA.
+uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
+  return compare_smem_bytes(K, tile_bytes, 4) <= kMaxSmemPerCta ? 4u : 2u;
 }
 
 int launch_compare(const CmpParams &p, int grid, void *stream) {
-  const size_t smem = compare_smem_bytes(p.K, p.tile_bytes);
-  cudaError_t e = cudaFuncSetAttribute(compare_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  const size_t smem = compare_smem_bytes(p.K, p.tile_bytes, p.nstages);
+  auto kern = p.nstages == 2 ? compare_kernel<2> : compare_kernel<4>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return (int)e;
-  compare_kernel<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
+  kern<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }
 
