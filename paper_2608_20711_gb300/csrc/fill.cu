@@ -206,17 +206,31 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
   }
 }
 
+// The region of tile t when it lies past region ri: a binary search over
+// the regions after ri (the table's sentinel entry bounds it).
+__device__ __noinline__ uint32_t next_region(const FillRegion *regs, uint32_t n, uint32_t ri,
+                                             uint64_t t) {
+  uint32_t lo = ri + 1, hi = n;     // regs[lo].tile0 <= t < regs[hi].tile0
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (regs[mid].tile0 <= t) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
 __global__ void __launch_bounds__(kThreads, 6) fill_kernel(const FillParams p) {
   __shared__ float4 lntab[ASMV_LN_TABLE_ROWS];
   for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS; i += kThreads) lntab[i] = kLnTableInit[i];
   __syncthreads();
   const uint64_t G = gridDim.x, b = blockIdx.x;
-  const uint64_t t0 = p.ntiles * b / G, t1 = p.ntiles * (b + 1) / G;
-  if (t0 < t1) {
+  // Tiles b, b + G, b + 2G, ...: every CTA gets its share of every region,
+  // so regions of very different cost per tile (NORMAL against RAW) spread
+  // evenly over the SMs.
+  if (b < p.ntiles) {
     const Keys K = {p.key0, p.key1, lntab};
-    uint32_t ri = find_region(p.regions, p.nregions, t0);
-    for (uint64_t t = t0; t < t1; ++t) {
-      while (p.regions[ri + 1].tile0 <= t) ++ri;
+    uint32_t ri = find_region(p.regions, p.nregions, b);
+    for (uint64_t t = b; t < p.ntiles; t += G) {
+      if (p.regions[ri + 1].tile0 <= t) ri = next_region(p.regions, p.nregions, ri, t);
       const FillRegion r = p.regions[ri];
       fill_tile_dispatch(r, K, t - r.tile0);
     }

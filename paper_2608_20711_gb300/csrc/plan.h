@@ -5,10 +5,13 @@
 // kTileBytes for the fill, and of a per-launch tile size for the compare
 // (the last tile of a region may be short).  Tiles of all
 // regions form one index space; region i owns tiles [tile0[i], tile0[i+1]).
-// A launch runs a persistent grid; CTA b takes the contiguous tile range
-// [T*b/G, T*(b+1)/G), so a CTA crosses few region boundaries and flushes its
-// per-region partial statistics once per boundary.  Inside a tile, thread t
-// handles 16-byte chunks t, t+256, ... (coalesced 128-bit accesses).
+// A launch runs a persistent grid.  In the compare and the Eq. 1 sums CTA b
+// takes the contiguous tile range [T*b/G, T*(b+1)/G), so a CTA crosses few
+// region boundaries and flushes its per-region partial statistics once per
+// boundary; the fill, which keeps no per-region state, takes tiles b, b+G,
+// b+2G, ..., so that regions of very different cost per tile spread evenly
+// over the SMs.  Inside a tile, thread t handles 16-byte chunks t, t+256,
+// ... (coalesced 128-bit accesses).
 //
 // Guard bands are cut into segments of at most kGuardSegBytes and handled
 // one warp per segment after the payload tiles.
