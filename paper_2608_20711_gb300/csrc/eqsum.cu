@@ -402,8 +402,89 @@ __device__ __forceinline__ uint32_t fp8_half(const uint4 &v, int k) {
   return fp8x2_to_half2_bits<DT>(byte_of(v, k)) & 0xFFFFu;
 }
 
-// One tile of an fp16 or fp8 region: S_rr once, then the candidates two at
-// a time (the reference chunk is decoded once per pair).  E5M2 and the fnuz
+// The sums of candidates j and (if TWO) j + 1 over one tile's share of a
+// warp, added to the CTA's shared digits sd (slots 1 + 2j .. 4 + 2j), and
+// with RR also sum r*r into the reference's slot (sdig0) from the same
+// decoded values.  With an odd number of candidates the last call has
+// TWO = false and does no work for a second candidate.
+template <int DT, bool TWO, bool RR>
+__device__ __forceinline__ void pair_sums(const CmpRegion &R, uint64_t ref, uint64_t cb0, uint64_t cb1,
+                                          uint32_t c0, uint32_t c1, uint32_t rounds, uint32_t nb,
+                                          long long *sd, long long *sdig0) {
+  const uint32_t lane = threadIdx.x & 31;
+  Acc3 rc0 = {0, 0, 0}, cc0 = {0, 0, 0}, rc1 = {0, 0, 0}, cc1 = {0, 0, 0}, rr = {0, 0, 0};
+  long long rc8_0 = 0, cc8_0 = 0, rc8_1 = 0, cc8_1 = 0, r8 = 0;
+#pragma unroll 1
+  for (uint32_t r = 0; r < rounds; ++r) {
+    const uint32_t c = c0 + 32u * r + lane;
+    uint4 rv = make_uint4(0u, 0u, 0u, 0u), v0 = rv, v1 = rv;
+    if (c < c1) {
+      const uint32_t bytes = min(16u, nb - 16u * c);
+      rv = load_chunk(ref + 16ull * c, bytes, R.vec, true);     // L1 hit after the first pair
+      v0 = load_chunk(cb0 + 16ull * c, bytes, R.vec, false);
+      if (TWO) v1 = load_chunk(cb1 + 16ull * c, bytes, R.vec, false);
+    }
+    if (DT == kF16) {
+      rv = finite_f16x8(rv);
+      v0 = finite_f16x8(v0);
+      if (TWO) v1 = finite_f16x8(v1);
+      const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+      const uint32_t w0[4] = {v0.x, v0.y, v0.z, v0.w};
+      const uint32_t w1[4] = {v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        Limbs xb[2], y0[2], y1[2];
+        fix_f16x2_biased(rw[q], xb[0], xb[1]);
+        fix_f16x2_biased(w0[q], y0[0], y0[1]);
+        if (TWO) fix_f16x2_biased(w1[q], y1[0], y1[1]);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const Limbs x = {xb[h].hi - kMagicBits, xb[h].lo - kMagicBits};
+          if (RR) sq(rr, x);
+          diff_add(rc0, cc0, x, xb[h], y0[h]);
+          if (TWO) diff_add(rc1, cc1, x, xb[h], y1[h]);
+        }
+      }
+    } else if (DT != kF8) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const Limbs x = fix_f16(fp8_half<DT>(rv, k));
+        if (RR) sq(rr, x);
+        diff_add(rc0, cc0, x, x, fix_f16(fp8_half<DT>(v0, k)));
+        if (TWO) diff_add(rc1, cc1, x, x, fix_f16(fp8_half<DT>(v1, k)));
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int x = fix_f8(byte_of(rv, k));
+        if (RR) r8 = mad_wide(x, x, r8);
+        const int y0 = fix_f8(byte_of(v0, k));
+        rc8_0 = mad_wide(x, y0, rc8_0); cc8_0 = mad_wide(y0, y0, cc8_0);
+        if (TWO) {
+          const int y1 = fix_f8(byte_of(v1, k));
+          rc8_1 = mad_wide(x, y1, rc8_1); cc8_1 = mad_wide(y1, y1, cc8_1);
+        }
+      }
+    }
+  }
+  if (DT != kF8) {
+    if (RR) flush3(rr, sdig0);
+    flush3(rc0, sd);
+    flush3(cc0, sd + kWin);
+    if (TWO) { flush3(rc1, sd + 2 * kWin); flush3(cc1, sd + 3 * kWin); }
+  } else {
+    if (RR) flush1(r8, sdig0);
+    flush1(rc8_0, sd);
+    flush1(cc8_0, sd + kWin);
+    if (TWO) { flush1(rc8_1, sd + 2 * kWin); flush1(cc8_1, sd + 3 * kWin); }
+  }
+}
+
+// One tile of an fp16 or fp8 region: S_rr, then the candidates two at a
+// time (the reference chunk is decoded once per pair).  With a single
+// candidate S_rr is added in the candidate's pass, from the same decoded
+// reference values (with two candidates per pass the extra accumulator
+// costs more than the second decode saves).  E5M2 and the fnuz
 // formats go through their exact fp16 values (and fp16's binary point).
 // For fp16 and those formats the candidate slots hold the difference-form
 // sums sum r d and sum d^2 (diff_add); the host forms S_rc and S_cc.
@@ -417,7 +498,7 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
   const uint32_t c1 = min(c0 + per_warp, nchunks);
   const uint32_t rounds = (per_warp + 31u) >> 5;     // the same for every warp
   const uint64_t ref = R.ref + a;
-  if (p.do_rr) {
+  if (p.do_rr && p.K >= 2) {           // with one candidate S_rr rides on its pass
     Acc3 rr = {0, 0, 0};
     long long r8 = 0;
 #pragma unroll 1
@@ -439,67 +520,12 @@ __device__ __noinline__ void eq_tile_fixed(const EqParams &p, const CmpRegion &R
     if (DT != kF8) flush3(rr, sdig); else flush1(r8, sdig);
   }
   for (uint32_t j = 0; j < p.K; j += 2) {
-    const bool two = j + 1 < p.K;                    // uniform
     const uint64_t cb0 = p.cands[(size_t)j * p.nregions + region] + a;
-    const uint64_t cb1 = two ? p.cands[(size_t)(j + 1) * p.nregions + region] + a : cb0;
-    Acc3 rc0 = {0, 0, 0}, cc0 = {0, 0, 0}, rc1 = {0, 0, 0}, cc1 = {0, 0, 0};
-    long long rc8_0 = 0, cc8_0 = 0, rc8_1 = 0, cc8_1 = 0;
-#pragma unroll 1
-    for (uint32_t r = 0; r < rounds; ++r) {
-      const uint32_t c = c0 + 32u * r + lane;
-      uint4 rv = make_uint4(0u, 0u, 0u, 0u), v0 = rv, v1 = rv;
-      if (c < c1) {
-        const uint32_t bytes = min(16u, nb - 16u * c);
-        rv = load_chunk(ref + 16ull * c, bytes, R.vec, true);     // L1 hit after the first pair
-        v0 = load_chunk(cb0 + 16ull * c, bytes, R.vec, false);
-        if (two) v1 = load_chunk(cb1 + 16ull * c, bytes, R.vec, false);
-      }
-      if (DT == kF16) {
-        rv = finite_f16x8(rv);
-        v0 = finite_f16x8(v0);
-        v1 = finite_f16x8(v1);
-        const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
-        const uint32_t w0[4] = {v0.x, v0.y, v0.z, v0.w};
-        const uint32_t w1[4] = {v1.x, v1.y, v1.z, v1.w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          Limbs xb[2], y0[2], y1[2];
-          fix_f16x2_biased(rw[q], xb[0], xb[1]);
-          fix_f16x2_biased(w0[q], y0[0], y0[1]);
-          fix_f16x2_biased(w1[q], y1[0], y1[1]);
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const Limbs x = {xb[h].hi - kMagicBits, xb[h].lo - kMagicBits};
-            diff_add(rc0, cc0, x, xb[h], y0[h]);
-            diff_add(rc1, cc1, x, xb[h], y1[h]);
-          }
-        }
-      } else if (DT != kF8) {
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const Limbs x = fix_f16(fp8_half<DT>(rv, k));
-          diff_add(rc0, cc0, x, x, fix_f16(fp8_half<DT>(v0, k)));
-          diff_add(rc1, cc1, x, x, fix_f16(fp8_half<DT>(v1, k)));
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int x = fix_f8(byte_of(rv, k));
-          const int y0 = fix_f8(byte_of(v0, k)), y1 = fix_f8(byte_of(v1, k));
-          rc8_0 = mad_wide(x, y0, rc8_0); cc8_0 = mad_wide(y0, y0, cc8_0);
-          rc8_1 = mad_wide(x, y1, rc8_1); cc8_1 = mad_wide(y1, y1, cc8_1);
-        }
-      }
-    }
-    if (DT != kF8) {
-      flush3(rc0, sdig + (1 + 2 * j) * kWin);
-      flush3(cc0, sdig + (2 + 2 * j) * kWin);
-      if (two) { flush3(rc1, sdig + (3 + 2 * j) * kWin); flush3(cc1, sdig + (4 + 2 * j) * kWin); }
-    } else {
-      flush1(rc8_0, sdig + (1 + 2 * j) * kWin);
-      flush1(cc8_0, sdig + (2 + 2 * j) * kWin);
-      if (two) { flush1(rc8_1, sdig + (3 + 2 * j) * kWin); flush1(cc8_1, sdig + (4 + 2 * j) * kWin); }
-    }
+    long long *sd = sdig + (1 + 2 * j) * kWin;
+    const uint64_t cb1 = j + 1 < p.K ? p.cands[(size_t)(j + 1) * p.nregions + region] + a : cb0;
+    if (j + 1 < p.K) pair_sums<DT, true, false>(R, ref, cb0, cb1, c0, c1, rounds, nb, sd, sdig);
+    else if (p.K == 1 && p.do_rr) pair_sums<DT, false, true>(R, ref, cb0, cb1, c0, c1, rounds, nb, sd, sdig);
+    else pair_sums<DT, false, false>(R, ref, cb0, cb1, c0, c1, rounds, nb, sd, sdig);
   }
 }
 
