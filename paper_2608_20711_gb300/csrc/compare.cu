@@ -58,6 +58,8 @@
 // per differing element, so dense small differences are also ALU-heavy.
 #include <float.h>
 #include <math_constants.h>
+#include <atomic>
+#include <mutex>
 #include "device.cuh"
 
 namespace asmv {
@@ -714,7 +716,7 @@ size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes, uint32_t nstages) {
 // 1 GiB fp16 reference (GB/s of reference + candidates read):
 //   K            2     3     4     5     6     7     8
 //   before    3051  2911  2582  2265  2654  2768  3051   (4 KiB tiles from K = 4, 4 stages)
-//   now       3143  2958  2940  3089  3062  3167  3498
+//   now       3137  2960  3302  3053  3118  3194  3530   (stages: 4 4 4 3 2 2 2)
 // and with one candidate, 4 stages of 16 KiB beat 2 stages by a fifth.
 // Tiles of whole warp rows (no tail rows) were measured too: better at
 // K = 2, worse at K = 3 and 5.
@@ -722,16 +724,51 @@ uint32_t compare_tile_bytes(uint32_t K) {
   return K <= 1 ? 16384u : 8192u;
 }
 
-// The deepest pipeline (4, else 2 stages) whose shared memory fits a CTA.
+// The deepest pipeline (4, 3, else 2 stages) within kCmpSmemBudget of shared
+// memory.  The budget stays below the 227 KiB a CTA may take: the rest of
+// the SM's 256 KiB is L1, which holds the checking warps' spilled registers
+// (about 100 bytes a thread), and deeper pipelines that squeezed it were
+// slower (K = 5 at 4 stages and 217 KiB: 2348 GB/s against 3089 at 2 stages).
+constexpr size_t kCmpSmemBudget = 192 * 1024;
 uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
-  return compare_smem_bytes(K, tile_bytes, 4) <= kMaxSmemPerCta ? 4u : 2u;
+  for (uint32_t n = 4; n > 2; --n)
+    if (compare_smem_bytes(K, tile_bytes, n) <= kCmpSmemBudget) return n;
+  return 2u;
 }
+
+// The dynamic shared memory limit of both instances, raised once per device
+// to the most any launch uses (a per-launch call would add its host latency
+// to every compare).  0: not yet, 1: done; a failure is returned every time.
+namespace {
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_smem_set[kMaxDevices];
+std::mutex g_smem_mutex;
+
+int prepare_compare(size_t smem) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  if (dev < 0 || dev >= kMaxDevices || smem > kMaxSmemPerCta) return (int)cudaErrorInvalidValue;
+  if (g_smem_set[dev].load(std::memory_order_acquire)) return (int)cudaSuccess;
+  std::lock_guard<std::mutex> lock(g_smem_mutex);
+  if (g_smem_set[dev].load(std::memory_order_relaxed)) return (int)cudaSuccess;
+  if ((e = cudaFuncSetAttribute(compare_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kMaxSmemPerCta)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(compare_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kMaxSmemPerCta)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(compare_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kMaxSmemPerCta)) != cudaSuccess)
+    return (int)e;
+  g_smem_set[dev].store(1, std::memory_order_release);
+  return (int)cudaSuccess;
+}
+}  // namespace
 
 int launch_compare(const CmpParams &p, int grid, void *stream) {
   const size_t smem = compare_smem_bytes(p.K, p.tile_bytes, p.nstages);
-  auto kern = p.nstages == 2 ? compare_kernel<2> : compare_kernel<4>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return (int)e;
+  const int rc = prepare_compare(smem);
+  if (rc != (int)cudaSuccess) return rc;
+  auto kern = p.nstages == 2 ? compare_kernel<2> : p.nstages == 3 ? compare_kernel<3> : compare_kernel<4>;
   kern<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }

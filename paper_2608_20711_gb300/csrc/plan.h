@@ -28,7 +28,7 @@ constexpr uint64_t kTileBytes = (uint64_t)kChunkBytes * kTileChunks;  // 16 KiB
 constexpr uint32_t kGuardSegBytes = 4096;
 constexpr int kMaxCands = 8;            // candidates per batched launch
 constexpr int kConsumerWarps = 16;      // compare: checking warps per CTA
-constexpr int kStages = 4;              // compare: deepest shared-memory pipeline (2 or 4 stages per launch)
+constexpr int kStages = 4;              // compare: deepest shared-memory pipeline (2 to 4 stages per launch)
 constexpr size_t kMaxSmemPerCta = 232448;   // GB300: 227 KiB of shared memory per CTA (opt-in)
 constexpr int kCmpThreads = (kConsumerWarps + 1) * 32;   // + one producer warp
 constexpr uint32_t kWaitRounds = 20000;  // compare: default bound of a pipeline wait, in tries
@@ -122,7 +122,7 @@ struct CmpParams {
   uint32_t K;
   uint32_t tile_bytes;         // payload bytes per tile (multiple of 16)
   uint32_t wait_rounds;        // bound of the producer's wait for a free stage (tries)
-  uint32_t nstages;            // pipeline depth of this launch: 2 or 4 (compare_stages)
+  uint32_t nstages;            // pipeline depth of this launch: 2, 3 or 4 (compare_stages)
   TolF tol[kNDtypes];
 };
 
