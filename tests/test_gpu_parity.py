@@ -307,7 +307,7 @@ def test_partial_tiles_of_every_shape(ctx, oracle, k):
             assert_stats_equal(g, want, "cand %d %s" % (j, r.name))
 
 
-@pytest.mark.parametrize("k", [2, 8, 11])
+@pytest.mark.parametrize("k", [2, 5, 6, 7, 8, 11])
 def test_batched_matches_oracle(ctx, oracle, k):
     regs = _cmp_table(31, n_regions=14)
     size = _place(regs)
