@@ -125,12 +125,21 @@ KERNEL_SOURCES = {"fill": ("fill.cu", "fill_math.cuh", "device.cuh", "ln_table.h
                   "copy": ("copy.cu", "device.cuh", "plan.h")}
 
 
+def _code_only(src):
+    """A source's code with comments, blank lines and indentation removed:
+    an edit to comments alone leaves the compiled kernel, and so the hash,
+    unchanged."""
+    tok = re.compile(r'"(?:\\.|[^"\\])*"|\'(?:\\.|[^\'\\])*\'|/\*.*?\*/|//[^\n]*', re.S)
+    src = tok.sub(lambda m: m.group(0) if m.group(0)[0] in "\"'" else " ", src)
+    return "\n".join(line.strip() for line in src.splitlines() if line.strip())
+
+
 def source_hash(kernel):
     d = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_20711_gb300", "csrc")
     for f in KERNEL_SOURCES[kernel]:
-        with open(os.path.join(csrc, f), "rb") as fh:
-            d.update(f.encode() + fh.read())
+        with open(os.path.join(csrc, f)) as fh:
+            d.update(f.encode() + _code_only(fh.read()).encode())
     return d.hexdigest()[:16]
 
 
