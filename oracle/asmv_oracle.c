@@ -674,8 +674,8 @@ void oracle_restore_region(uint8_t *alloc, uint64_t payload_bytes, uint32_t glo,
  *      digits, digit k weighing 2^(32 k + OEQ_BASE).  The final rounding is
  *      done by the caller from the digits.
  * The range covers every product of two fp32 values (2^-298 .. 2^256) with
- * 2^64 of headroom for the sum.  Binary64 regions have no exact sums here
- * (their products need 106 bits): they return zeros.
+ * 2^64 of headroom for the sum.  Binary64 products need 106 bits: those
+ * regions are summed by oracle_eq64_sums_range (R11) and return zeros here.
  * ====================================================================== */
 #define OEQ_DIGITS 20
 #define OEQ_BASE (-320)
@@ -734,6 +734,91 @@ void oracle_eq_sums_range(const uint8_t *ref, const uint8_t *cand, int dt,
 
 int oracle_eq_digits(void) { return OEQ_DIGITS; }
 int oracle_eq_base(void) { return OEQ_BASE; }
+
+/* ======================================================================
+ * Eq. 1 sums of binary64 regions (R9 widened to binary64).
+ *   R11 A finite binary64 value is +-m 2^e with m an integer below 2^53
+ *       and e >= -1074, so a product of two is +-M 2^E with M = m_r m_c
+ *       below 2^106 and E >= -2148, and its magnitude is below 2^2048.
+ *       The sums are kept exactly in O64_DIGITS signed 64-bit digits, digit
+ *       k weighing 2^(32 k + O64_BASE): 2^-2148 .. 2^2048 and 2^64 of
+ *       headroom need 134 digits.  The caller rounds them (gradual
+ *       underflow and overflow to infinity included) and forms the cosine.
+ * ====================================================================== */
+#define O64_DIGITS 136
+#define O64_BASE (-2148)
+
+static void eq64_normalize(int64_t *acc) {
+  for (int k = 0; k < O64_DIGITS - 1; ++k) {
+    int64_t carry = acc[k] >> 32;          /* floor division by 2^32 */
+    acc[k] -= carry * 4294967296LL;
+    acc[k + 1] += carry;
+  }
+}
+
+/* |x| = m 2^e with m odd, for finite non-zero x; m = 0 for zeros and
+ * non-finite x. */
+static void eq64_split(double x, uint64_t *m, int *e) {
+  *m = 0;
+  *e = 0;
+  if (x == 0.0 || !isfinite(x)) return;
+  int ex;
+  double f = frexp(fabs(x), &ex);                  /* |x| = f 2^ex, f in [0.5, 1) */
+  uint64_t mm = (uint64_t)ldexp(f, 53);            /* exact: 53-bit integer */
+  int ee = ex - 53;
+  while ((mm & 1u) == 0) { mm >>= 1; ++ee; }       /* now ee >= -1074 */
+  *m = mm;
+  *e = ee;
+}
+
+/* Bits lo .. lo + 31 of M as an integer (lo may be negative: low bits 0). */
+static uint64_t eq64_bits(unsigned __int128 M, int lo) {
+  if (lo >= 128) return 0;
+  if (lo < 0) return (uint64_t)((M << -lo) & 0xFFFFFFFFu);
+  return (uint64_t)((M >> lo) & 0xFFFFFFFFu);
+}
+
+/* acc += (-1)^neg m1 m2 2^(e1 + e2), exactly. */
+static void eq64_add(int64_t *acc, int neg, uint64_t m1, int e1, uint64_t m2, int e2) {
+  if (m1 == 0 || m2 == 0) return;
+  unsigned __int128 M = (unsigned __int128)m1 * m2;      /* < 2^106 */
+  int pos = e1 + e2 - O64_BASE;                          /* >= 0 */
+  int q = pos / 32, b = pos % 32;
+  /* M 2^pos = sum over k of (bits 32k - b .. 32k - b + 31 of M) 2^(32 (q + k)) */
+  for (int k = 0; k < 5; ++k) {
+    int64_t dig = (int64_t)eq64_bits(M, 32 * k - b);
+    acc[q + k] += neg ? -dig : dig;
+  }
+}
+
+/* The three sums over elements [i0, i1) of two binary64 payloads, as
+ * normalized digits: out[0..D) = S_rc, out[D..2D) = S_rr, out[2D..3D) =
+ * S_cc, D = O64_DIGITS. */
+void oracle_eq64_sums_range(const uint8_t *ref, const uint8_t *cand, uint64_t i0, uint64_t i1,
+                            int64_t *out) {
+  int64_t *rc = out, *rr = out + O64_DIGITS, *cc = out + 2 * O64_DIGITS;
+  for (int k = 0; k < 3 * O64_DIGITS; ++k) out[k] = 0;
+  uint64_t since = 0;
+  for (uint64_t i = i0; i < i1; ++i) {
+    double r = decode_elem(ref, OD_F64, i), c = decode_elem(cand, OD_F64, i);
+    uint64_t mr, mc;
+    int er, ec;
+    eq64_split(r, &mr, &er);
+    eq64_split(c, &mc, &ec);
+    int nr = signbit(r) != 0, nc = signbit(c) != 0;
+    if (isfinite(r) && isfinite(c)) eq64_add(rc, nr != nc, mr, er, mc, ec);
+    if (isfinite(r)) eq64_add(rr, 0, mr, er, mr, er);
+    if (isfinite(c)) eq64_add(cc, 0, mc, ec, mc, ec);
+    if (++since == (1u << 20)) {     /* each digit grows by < 2^32 per add */
+      eq64_normalize(rc); eq64_normalize(rr); eq64_normalize(cc);
+      since = 0;
+    }
+  }
+  eq64_normalize(rc); eq64_normalize(rr); eq64_normalize(cc);
+}
+
+int oracle_eq64_digits(void) { return O64_DIGITS; }
+int oracle_eq64_base(void) { return O64_BASE; }
 
 /* ======================================================================
  * Batch entry points for the tests (plain loops over the functions above).

@@ -120,6 +120,7 @@ def _load(path):
                 c.POINTER(_RegionStats)]
             L.oracle_eq_sums_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
                                                c.c_uint64, _i64p]
+            L.oracle_eq64_sums_range.argtypes = [_u8p, _u8p, c.c_uint64, c.c_uint64, _i64p]
             L.oracle_restore_region.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
                                                 c.c_uint8, _u8p]
     return L
@@ -336,6 +337,57 @@ def exact_to_double(v):
     return v / (1 << -EQ_BASE)
 
 
+# Binary64 regions (reading R11 of the C oracle): products up to 106 bits,
+# sums kept exactly at the binary point 2^EQ64_BASE.
+EQ64_DIGITS, EQ64_BASE = 136, -2148
+
+
+def eq64_sums_range(ref_payload, cand_payload, i0, i1):
+    """Exact S_rc, S_rr, S_cc of two binary64 payloads over elements
+    [i0, i1), as Python integers scaled by 2^-EQ64_BASE."""
+    out = np.zeros(3 * EQ64_DIGITS, np.int64)
+    lib().oracle_eq64_sums_range(_ptr(ref_payload, _u8p), _ptr(cand_payload, _u8p), i0, i1,
+                                 _ptr(out, _i64p))
+    vals = []
+    for s in range(3):
+        d = out[s * EQ64_DIGITS:(s + 1) * EQ64_DIGITS]
+        vals.append(sum(int(d[k]) << (32 * k) for k in range(EQ64_DIGITS)))
+    return tuple(vals)
+
+
+def round_scaled(v, e):
+    """The integer v times 2^e rounded to the nearest fp64, ties to even,
+    with gradual underflow and overflow to an infinity of v's sign (Python's
+    int-to-float conversion and int / int division both round correctly and
+    raise OverflowError exactly when the rounded value overflows)."""
+    if v == 0:
+        return 0.0
+    try:
+        return float(v << e) if e >= 0 else v / (1 << -e)
+    except OverflowError:
+        return float("inf") if v > 0 else float("-inf")
+
+
+def eq_cos_exact(v_rc, v_rr, v_cc, base):
+    """c_x of Eq. 1 from exact sums S = v * 2^base, without overflow or
+    underflow of the intermediate sums: with 2p and 2q the even exponents
+    that bring S_rr and S_cc into [1, 4), the cosine is formed in fp64 from
+    RN(S_rc 2^-(p+q)), RN(S_rr 2^-2p) and RN(S_cc 2^-2q) -- the same number
+    as the plain formula, whose sums of binary64 values can leave the double
+    range.  1 when both sums of squares are 0, 0 when exactly one is."""
+    import math
+    if v_rr == 0 and v_cc == 0:
+        return 1.0
+    if v_rr == 0 or v_cc == 0:
+        return 0.0
+    p = (v_rr.bit_length() - 1 + base) // 2          # floor, also below zero
+    q = (v_cc.bit_length() - 1 + base) // 2
+    x = round_scaled(v_rc, base - p - q)
+    y = round_scaled(v_rr, base - 2 * p)
+    z = round_scaled(v_cc, base - 2 * q)
+    return x / (math.sqrt(y) * math.sqrt(z))
+
+
 def eq_cos(s_rc, s_rr, s_cc):
     """c_x of Eq. 1 from the rounded sums, in fp64: S_rc / (sqrt(S_rr) *
     sqrt(S_cc)); 1 when both vectors are zero, 0 when exactly one is."""
@@ -348,19 +400,30 @@ def eq_cos(s_rc, s_rr, s_cc):
 
 
 def eq_sums(ref_payload, cand_payload, dtype, n_elems, threads=1):
-    """The three sums of one float region, each exact then rounded to fp64
-    (not defined for binary64 regions)."""
-    if dtype == F64:
-        raise ValueError("Eq. 1 sums are not defined here for binary64 regions")
+    """The three sums of one float region, each exact then rounded to fp64,
+    and the cosine c_x.  Binary64 sums round with gradual underflow and
+    overflow to infinity, and their cosine comes from the scaled exact sums
+    (eq_cos_exact); for the other formats the sums stay well inside the
+    normal double range and c_x is eq_cos of the rounded sums."""
     spans = _split(n_elems, threads)
     parts = [None] * len(spans)
 
     def job(k, a, b):
-        parts[k] = eq_sums_range(ref_payload, cand_payload, dtype, a, b)
+        if dtype == F64:
+            parts[k] = eq64_sums_range(ref_payload, cand_payload, a, b)
+        else:
+            parts[k] = eq_sums_range(ref_payload, cand_payload, dtype, a, b)
     _run_threads([lambda k=k, a=a, b=b: job(k, a, b) for k, (a, b) in enumerate(spans)])
     tot = [sum(p[j] for p in parts) for j in range(3)]
-    return {"sum_rc": exact_to_double(tot[0]), "sum_rr": exact_to_double(tot[1]),
-            "sum_cc": exact_to_double(tot[2])}
+    if dtype == F64:
+        out = {"sum_rc": round_scaled(tot[0], EQ64_BASE), "sum_rr": round_scaled(tot[1], EQ64_BASE),
+               "sum_cc": round_scaled(tot[2], EQ64_BASE)}
+        out["cos"] = eq_cos_exact(tot[0], tot[1], tot[2], EQ64_BASE)
+        return out
+    out = {"sum_rc": exact_to_double(tot[0]), "sum_rr": exact_to_double(tot[1]),
+           "sum_cc": exact_to_double(tot[2])}
+    out["cos"] = eq_cos(out["sum_rc"], out["sum_rr"], out["sum_cc"])
+    return out
 
 
 def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
@@ -372,7 +435,10 @@ def eq_verdict(stats, sums, dtype, theta=THETA, tau=TAU):
     regions have no cosine (NaN) and pass the two float terms."""
     flt = dtype in FLOAT_DTYPES
     out = dict(sums) if flt else {"sum_rc": 0.0, "sum_rr": 0.0, "sum_cc": 0.0}
-    out["cos"] = eq_cos(out["sum_rc"], out["sum_rr"], out["sum_cc"]) if flt else float("nan")
+    if not flt:
+        out["cos"] = float("nan")
+    elif "cos" not in out:
+        out["cos"] = eq_cos(out["sum_rc"], out["sum_rr"], out["sum_cc"])
     flags = 0
     if not flt or out["cos"] >= theta:
         flags |= EQ_COS

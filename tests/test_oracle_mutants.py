@@ -21,7 +21,7 @@ from oracle import oracle as O
 PIN_MODULES = ("tests.test_oracle_codecs", "tests.test_oracle_philox",
                "tests.test_oracle_fill", "tests.test_oracle_compare",
                "tests.test_oracle_eq", "tests.test_oracle_dtypes", "tests.test_oracle_restore",
-               "tests.test_oracle_boxmuller")
+               "tests.test_oracle_boxmuller", "tests.test_oracle_eq64")
 # pins that take seconds run last, in this order
 EXPENSIVE = ("test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
              "test_ln_u24_all_inputs")
@@ -105,6 +105,19 @@ MUTANTS = [
     ("eq_sign_dropped", "int64_t sg = (p < 0.0) ? -1 : 1;", "int64_t sg = 1;"),
     ("eq_lsb_off_by_one", "int lsb = e - 53;", "int lsb = e - 52;"),
     ("eq_mid_digit_shift", "((m >> (32 - b)) & 0xFFFFFFFFu)", "((m >> (31 - b)) & 0xFFFFFFFFu)"),
+    # the exact sums of binary64 regions
+    ("eq64_digit_shift_off_by_one", "(int64_t)eq64_bits(M, 32 * k - b);",
+     "(int64_t)eq64_bits(M, 32 * k - b - 1);"),
+    ("eq64_top_digit_dropped", "for (int k = 0; k < 5; ++k) {\n    int64_t dig",
+     "for (int k = 0; k < 4; ++k) {\n    int64_t dig"),
+    ("eq64_low_bits_shifted_away", "if (lo < 0) return (uint64_t)((M << -lo) & 0xFFFFFFFFu);",
+     "if (lo < 0) return (uint64_t)((M >> -lo) & 0xFFFFFFFFu);"),
+    ("eq64_cross_sign_of_reference", "eq64_add(rc, nr != nc, mr, er, mc, ec);",
+     "eq64_add(rc, nr, mr, er, mc, ec);"),
+    ("eq64_rr_uses_candidate", "eq64_add(rr, 0, mr, er, mr, er);", "eq64_add(rr, 0, mr, er, mc, ec);"),
+    ("eq64_cc_needs_finite_pair", "if (isfinite(c)) eq64_add(cc, 0, mc, ec, mc, ec);",
+     "if (isfinite(r) && isfinite(c)) eq64_add(cc, 0, mc, ec, mc, ec);"),
+    ("eq64_exponent_off_by_one", "int ee = ex - 53;", "int ee = ex - 52;"),
     # further stored formats
     ("fnuz_negative_zero_kept", "if (fnuz && mag == 0) return 0;", ""),
     ("e5m2_saturates_to_inf", "encode_fp8(f, 5, 2, 15, 0x7Bu, 0)", "encode_fp8(f, 5, 2, 15, 0x7Cu, 0)"),
