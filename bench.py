@@ -12,8 +12,9 @@ Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|referenc
 
 Beside the step, the line carries `eq1`: Eq. 1 as a whole (the exact sums
 of the cosine term over the same reference and candidates), its kernel
-timed alone with CUDA events; and `restore`: the Tier 2 restore of the
-step's input regions from a captured snapshot, timed the same way.
+timed alone with CUDA events; `eq1_f64`: the same for binary64 outputs of
+the reference's size; and `restore`: the Tier 2 restore of the step's input
+regions from a captured snapshot, timed the same way.
 For N > 1 launch under torchrun; every rank runs its own replica (weak
 scaling, no data-path collective) and rank 0 prints one JSON line.
 """
@@ -122,7 +123,8 @@ def kernel_traffic(kernel, workload):
 KERNEL_SOURCES = {"fill": ("fill.cu", "fill_math.cuh", "device.cuh", "ln_table.h", "plan.h"),
                   "compare": ("compare.cu", "device.cuh", "plan.h"),
                   "eqsum": ("eqsum.cu", "device.cuh", "plan.h"),
-                  "copy": ("copy.cu", "device.cuh", "plan.h")}
+                  "copy": ("copy.cu", "device.cuh", "plan.h"),
+                  "eq64": ("eq64.cu", "eq64.h", "device.cuh", "plan.h")}
 
 
 def _code_only(src):
@@ -439,6 +441,7 @@ def run_mine(args):
     }
     if args.eq:
         line["eq1"] = run_eq1(setup, args, peak)
+        line["eq1_f64"] = run_eq1_f64(setup, args, peak)
     if args.restore:
         line["restore"] = run_restore(setup, args, peak)
     if rank == 0 and world == 1 and args.cpu:
@@ -481,6 +484,44 @@ def run_eq1(setup, args, peak):
             "pairs_per_s": round(elems * k / (avg / 1e3), 1),
             "theta": setup.asmv.THETA, "tau": setup.asmv.TAU,
             "passing": int(sum(e["eq"] for cs in eqs for e in cs)), "checks": k * len(eqs[0])}
+
+
+def run_eq1_f64(setup, args, peak, k=2):
+    """Eq. 1 over binary64 outputs of the same size as the step's reference
+    (a N(0, 1) reference from the guarded fill, k candidates with the last
+    bit flipped at every 7th element), through asmv_compare_eq; its binary64
+    sums kernel timed alone with CUDA events around its launches."""
+    torch, ctx, asmv = setup.torch, setup.ctx, setup.asmv
+    floats = ("f32", "bf16", "f16", "f8e4m3")
+    n = max(1, sum(r.payload_bytes for r in setup.wl.regions if r.dtype in floats) // 8)
+    ref = torch.empty(n, dtype=torch.float64, device=setup.device)
+
+    def table(t):
+        return [asmv.make_region(t.data_ptr(), n, "f64", "normal", 0, 0, region_id=1, p0=0.0, p1=1.0)]
+    ctx.fill(table(ref), seed=11)
+    cands = []
+    for j in range(k):
+        c = ref.clone()
+        c.view(torch.int64)[j::7] ^= 1
+        cands.append(c)
+    tol = {"f64": (1e-9, 1e-9)}
+    ctx.compare_eq(table(ref), [table(c) for c in cands], tol)
+    ctx.set_timing(True)
+    ms = []
+    for _ in range(max(3, args.steps)):
+        _, eqs = ctx.compare_eq(table(ref), [table(c) for c in cands], tol)
+        ms.append(ctx.kernel_ms())
+    ctx.set_timing(False)
+    avg = float(np.mean(ms))
+    nbytes = 8 * n * (1 + k)
+    gbs = nbytes / (avg / 1e3) / 1e9
+    traffic, _ = kernel_traffic("eq64", args.workload)
+    del ref, cands
+    return {"kernel": "eq64_kernel", "values": n, "candidates": k, "avg_launch_ms": round(avg, 4),
+            "algorithmic_bytes_per_launch": nbytes, "gbs": round(gbs, 1),
+            "hbm_frac": round(gbs / peak, 4), "traffic": traffic,
+            "pairs_per_s": round(n * k / (avg / 1e3), 1),
+            "passing": int(sum(e[0]["eq"] for e in eqs)), "cos": [e[0]["cos"] for e in eqs]}
 
 
 def run_restore(setup, args, peak):

@@ -233,8 +233,12 @@ typedef struct {
  * eq_host[j*n + i] the Eq. 1 result of candidate j on region i (k*n entries
  * each, caller-owned).  theta is any finite double; tau a finite double
  * >= 0.  Float regions of more than 2^31 elements are rejected (the exact
- * sums keep per-digit counts below 2^31), and so are binary64 regions (the
- * exact sums here cover formats whose products are exact in fp64).
+ * sums keep per-digit counts below 2^31).  Binary64 regions: the exact sums
+ * (products of 106 bits, 2^-2148 .. 2^2048) are rounded with gradual
+ * underflow and overflow to +-Inf, so sum_* may be Inf, subnormal or 0 for
+ * outputs near the ends of the double range; cos is formed from the exact
+ * sums scaled by powers of two (sum_rr by 2^-2p and sum_cc by 2^-2q into
+ * [1, 4), sum_rc by 2^-(p+q)), which is the same cosine and stays finite.
  * Synchronous.  Errors as asmv_compare_batched, plus EINVAL for a null
  * eq_host, a non-finite theta or tau, a negative tau, or such a region. */
 int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
@@ -246,6 +250,7 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
  * digit vectors are added element-wise over the processes and the
  * statistics merged, and asmv_eq_from_digits gives the verdict of the
  * whole -- the same result as one asmv_compare_eq over the whole regions.
+ * Binary64 regions are not taken here (EINVAL): their sums need 136 digits.
  *
  * asmv_compare_eq_digits: the statistics of asmv_compare_batched in
  * stats_host[j*n + i], and the exact sums of region i in

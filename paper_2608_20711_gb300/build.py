@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libasmv.so")
 BUILD = os.path.join(HERE, "_build")
-SOURCES = ["abi.cu", "fill.cu", "compare.cu", "eqsum.cu", "gate.cu", "copy.cu", "va.cu"]
+SOURCES = ["abi.cu", "fill.cu", "compare.cu", "eqsum.cu", "eq64.cu", "gate.cu", "copy.cu", "va.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

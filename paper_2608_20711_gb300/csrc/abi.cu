@@ -19,6 +19,7 @@
 
 #include "asmv.h"
 #include "plan.h"
+#include "eq64.h"
 
 using namespace asmv;
 
@@ -206,6 +207,7 @@ struct asmv_ctx {
   int sms = 0;
   int fill_ctas = 1;
   int eq_ctas = 1;
+  int eq64_ctas = 1;
   int copy_ctas = 1;
   void *dws = nullptr;
   size_t dws_cap = 0;
@@ -355,55 +357,96 @@ int readback(asmv_ctx *ctx, size_t stats_off, size_t img_bytes, size_t count, cu
   return ASMV_OK;
 }
 
-// The integer sum_k d[k] 2^(32k + base) rounded to the nearest double (ties
-// to even).  The digits are first carried into nd + 2 limbs of 32 bits in
-// two's complement; the magnitude's leading 64 bits and a sticky bit then
-// decide the rounding.
-int exact_to_double_impl(const int64_t *d, int nd, int base, double *out) {
-  if (d == nullptr || out == nullptr || nd < 1 || nd > 64) return ASMV_EINVAL;
-  const int nl = nd + 2;
-  uint32_t L[66];
+// The magnitude and sign of the integer sum_k d[k] 2^(32k): the digits are
+// carried into nd + 2 limbs of 32 bits in two's complement, and negated when
+// the top carry says the value is negative.  msb is the position of the
+// leading one bit, -1 for zero.
+constexpr int kMaxExactDigits = kEq64Digits;
+struct Magnitude {
+  uint32_t L[kMaxExactDigits + 2];
+  int nl;
+  int msb;
+  bool neg;
+  uint64_t bit(int pos) const {
+    return (pos < 0 || pos >= 32 * nl) ? 0u : (uint64_t)((L[pos >> 5] >> (pos & 31)) & 1u);
+  }
+  bool any_below(int pos) const {                 // some bit at a position < pos is set
+    if (pos <= 0) return false;
+    const int lim = std::min(pos >> 5, nl);
+    for (int k = 0; k < lim; ++k)
+      if (L[k] != 0) return true;
+    if (lim == nl || (pos & 31) == 0) return false;
+    return (L[lim] & ((1u << (pos & 31)) - 1u)) != 0;
+  }
+};
+
+void magnitude_of(const int64_t *d, int nd, Magnitude *m) {
+  m->nl = nd + 2;
   __int128 c = 0;
-  for (int k = 0; k < nl; ++k) {
+  for (int k = 0; k < m->nl; ++k) {
     const __int128 x = c + (k < nd ? (__int128)d[k] : (__int128)0);
-    L[k] = (uint32_t)(x & 0xFFFFFFFF);
+    m->L[k] = (uint32_t)(x & 0xFFFFFFFF);
     c = x >> 32;                                   // floor: arithmetic shift
   }
-  const bool neg = c < 0;                          // c is 0 or -1 here
-  if (neg) {
+  m->neg = c < 0;                                  // c is 0 or -1 here
+  if (m->neg) {
     uint64_t carry = 1;
-    for (int k = 0; k < nl; ++k) {
-      const uint64_t x = (uint64_t)(uint32_t)~L[k] + carry;
-      L[k] = (uint32_t)x;
+    for (int k = 0; k < m->nl; ++k) {
+      const uint64_t x = (uint64_t)(uint32_t)~m->L[k] + carry;
+      m->L[k] = (uint32_t)x;
       carry = x >> 32;
     }
   }
-  int top = nl - 1;
-  while (top >= 0 && L[top] == 0) --top;
-  if (top < 0) { *out = 0.0; return ASMV_OK; }
-  int msb = 32 * top;
-  for (uint32_t v = L[top]; v > 1; v >>= 1) ++msb;
-  auto bit = [&](int pos) -> uint64_t {
-    return pos < 0 ? 0u : (uint64_t)((L[pos >> 5] >> (pos & 31)) & 1u);
-  };
-  uint64_t m = 0;
-  for (int b = 0; b < 64; ++b) m = (m << 1) | bit(msb - b);
-  bool sticky = false;
-  const int below = msb - 64;                      // highest bit not in m
-  if (below >= 0) {
-    const int lim = below >> 5;
-    const uint32_t mask = (below & 31) == 31 ? 0xFFFFFFFFu : ((1u << ((below & 31) + 1)) - 1u);
-    sticky = (L[lim] & mask) != 0;
-    for (int k = 0; k < lim && !sticky; ++k) sticky = L[k] != 0;
+  int top = m->nl - 1;
+  while (top >= 0 && m->L[top] == 0) --top;
+  m->msb = -1;
+  if (top >= 0) {
+    m->msb = 32 * top;
+    for (uint32_t v = m->L[top]; v > 1; v >>= 1) ++m->msb;
   }
-  uint64_t keep = m >> 11;                         // 53 bits
-  const uint64_t rem = m & 0x7FFu, half = 0x400u;
-  if (rem > half || (rem == half && (sticky || (keep & 1u)))) keep += 1;
-  const int e = msb - 52 + base;                   // weight of keep's last bit
-  if (e + 52 < -1022 || e + 53 > 1024) return ASMV_EINVAL;
-  const double v = std::ldexp((double)keep, e);
-  *out = neg ? -v : v;
+}
+
+// |value| 2^scale rounded to the nearest double, ties to even, with gradual
+// underflow (the last kept bit weighs at least 2^-1074) and overflow to
+// infinity; the sign is not applied.
+double round_magnitude(const Magnitude &m, int scale) {
+  if (m.msb < 0) return 0.0;
+  if (m.msb + scale >= 1024) return INFINITY;
+  const int last = std::max(m.msb - 52, -1074 - scale);   // position of the last kept bit
+  uint64_t keep = 0;
+  for (int pos = m.msb; pos >= last; --pos) keep = (keep << 1) | m.bit(pos);
+  const bool half = m.bit(last - 1) != 0;
+  const bool sticky = m.any_below(last - 1);
+  if (half && (sticky || (keep & 1u))) keep += 1;
+  return std::ldexp((double)keep, last + scale);   // exact; 2^1024 becomes infinity
+}
+
+// The integer sum_k d[k] 2^(32k + base) rounded to the nearest double (ties
+// to even); EINVAL when the value lies outside the normal double range.
+int exact_to_double_impl(const int64_t *d, int nd, int base, double *out) {
+  if (d == nullptr || out == nullptr || nd < 1 || nd > 64) return ASMV_EINVAL;
+  Magnitude m;
+  magnitude_of(d, nd, &m);
+  if (m.msb < 0) { *out = 0.0; return ASMV_OK; }
+  if (m.msb + base < -1022 || m.msb + base >= 1024) return ASMV_EINVAL;
+  const double v = round_magnitude(m, base);
+  *out = m.neg ? -v : v;
   return ASMV_OK;
+}
+
+// c_x of a binary64 region from its exact sums (value = magnitude 2^base):
+// S_rr and S_cc scaled by 2^-2p and 2^-2q into [1, 4) and S_rc by
+// 2^-(p+q) before rounding, so no sum overflows or underflows, and the
+// cosine of the scaled sums is the cosine of the sums.
+double eq_cosine_scaled(const Magnitude &rc, const Magnitude &rr, const Magnitude &cc, int base) {
+  if (rr.msb < 0 && cc.msb < 0) return 1.0;
+  if (rr.msb < 0 || cc.msb < 0) return 0.0;
+  auto half_floor = [](int v) { return v >= 0 ? v / 2 : -((1 - v) / 2); };
+  const int p = half_floor(rr.msb + base), q = half_floor(cc.msb + base);
+  double x = round_magnitude(rc, base - p - q);
+  if (rc.neg) x = -x;
+  const double y = round_magnitude(rr, base - 2 * p), z = round_magnitude(cc, base - 2 * q);
+  return x / (std::sqrt(y) * std::sqrt(z));
 }
 
 double eq_cosine(double rc, double rr, double cc) {
@@ -457,6 +500,7 @@ int asmv_ctx_create(asmv_ctx **out, int device) {
   }
   ctx->fill_ctas = fill_max_ctas_per_sm();
   ctx->eq_ctas = eq_max_ctas_per_sm();
+  ctx->eq64_ctas = eq64_max_ctas_per_sm();
   ctx->copy_ctas = copy_max_ctas_per_sm();
   void *fn = nullptr;
   cudaDriverEntryPointQueryResult q;
@@ -727,13 +771,45 @@ int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref, const asmv_regio
   return run_compare(ctx, ref, cands, k, n, tol, out_host, (cudaStream_t)stream, false);
 }
 
-// The exact Eq. 1 sums of k candidates: fills digits[n][1 + 2k][kEqDigits].
+// The exact Eq. 1 sums of k candidates: fills digits[n][1 + 2k][kEqDigits]
+// for the float regions other than binary64, and digits64[m][1 + 2k]
+// [kEq64Digits] for the m-th binary64 region of the table.
 static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
-                  size_t k, size_t n, cudaStream_t s, std::vector<long long> &digits) {
+                  size_t k, size_t n, cudaStream_t s, std::vector<long long> &digits,
+                  std::vector<long long> &digits64) {
   const size_t nslots = 1 + 2 * k;
   digits.assign(n * nslots * kEqDigits, 0);
-  std::vector<CmpRegion> cr(n + 1);
-  std::vector<uint64_t> caddr(k * n);
+  std::vector<CmpRegion> cr(n + 1), cr64;
+  std::vector<uint64_t> caddr(k * n), caddr64;
+  std::vector<size_t> idx64;                       // table index of each binary64 region
+  for (size_t i = 0; i < n; ++i)
+    if (ref[i].dtype == ASMV_F64) idx64.push_back(i);
+  const size_t n64 = idx64.size();
+  digits64.assign(n64 * nslots * kEq64Digits, 0);
+  cr64.resize(n64 + 1);
+  caddr64.resize(k * n64);
+  uint64_t tile64 = 0;
+  for (size_t m = 0; m < n64; ++m) {
+    const asmv_region &r = ref[idx64[m]];
+    uint64_t pb, tot;
+    region_extent(r, &pb, &tot);
+    CmpRegion &c = cr64[m];
+    std::memset(&c, 0, sizeof c);
+    c.ref = r.alloc + r.guard_lo;
+    c.bytes = pb;
+    c.tile0 = tile64;
+    c.dtype = r.dtype;
+    bool vec = (c.ref % 16) == 0;
+    for (size_t j = 0; j < k; ++j) {
+      const uint64_t a = cands[j][idx64[m]].alloc + cands[j][idx64[m]].guard_lo;
+      caddr64[j * n64 + m] = a;
+      vec = vec && (a % 16) == 0;
+    }
+    c.vec = vec;
+    tile64 += (pb + kEq64TileBytes - 1) / kEq64TileBytes;
+  }
+  std::memset(&cr64[n64], 0, sizeof(CmpRegion));
+  cr64[n64].tile0 = tile64;
   uint64_t tile = 0;
   for (size_t i = 0; i < n; ++i) {
     const asmv_region &r = ref[i];
@@ -756,18 +832,23 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   }
   std::memset(&cr[n], 0, sizeof(CmpRegion));
   cr[n].tile0 = tile;
-  if (tile == 0) return ASMV_OK;                    // no float payload: all sums are zero
+  if (tile == 0 && tile64 == 0) return ASMV_OK;     // no float payload: all sums are zero
   const size_t dig_bytes = digits.size() * sizeof(long long);
+  const size_t dig64_bytes = digits64.size() * sizeof(long long);
+  const size_t o_dig64 = (dig_bytes + 255) & ~(size_t)255;     // from o_dig
+  const size_t all_dig = o_dig64 + dig64_bytes;
 
   Image img;
   const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CmpRegion));
   const size_t o_cand = img.add(caddr.data(), caddr.size() * sizeof(uint64_t));
+  const size_t o_regs64 = img.add(cr64.data(), cr64.size() * sizeof(CmpRegion));
+  const size_t o_cand64 = img.add(caddr64.data(), caddr64.size() * sizeof(uint64_t));
   const size_t o_dig = (img.bytes.size() + 255) & ~(size_t)255;
   unsigned char *dev = nullptr;
   int rc;
-  if ((rc = stage(ctx, img, dig_bytes, s, &dev, dig_bytes)) != ASMV_OK) return rc;
+  if ((rc = stage(ctx, img, all_dig, s, &dev, all_dig)) != ASMV_OK) return rc;
   cudaError_t e;
-  if ((e = cudaMemsetAsync(dev + o_dig, 0, dig_bytes, s)) != cudaSuccess) return fail_cuda(ctx, e);
+  if ((e = cudaMemsetAsync(dev + o_dig, 0, all_dig, s)) != cudaSuccess) return fail_cuda(ctx, e);
 
   EqParams p;
   std::memset(&p, 0, sizeof p);
@@ -777,14 +858,30 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   p.nregions = (uint32_t)n;
   p.nslots = (uint32_t)nslots;
   const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tile, (uint64_t)ctx->sms * ctx->eq_ctas));
+  Eq64Params p64;
+  std::memset(&p64, 0, sizeof p64);
+  p64.regions = (const CmpRegion *)(dev + o_regs64);
+  p64.digits = (long long *)(dev + o_dig + o_dig64);
+  p64.ntiles = tile64;
+  p64.nregions = (uint32_t)n64;
+  p64.nslots = (uint32_t)nslots;
+  const int grid64 =
+      (int)std::max<uint64_t>(1, std::min<uint64_t>(tile64, (uint64_t)ctx->sms * ctx->eq64_ctas));
   if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
   for (size_t g = 0; g * kMaxCands < k; ++g) {
-    p.K = (uint32_t)std::min<size_t>(kMaxCands, k - g * kMaxCands);
-    p.j0 = (uint32_t)(g * kMaxCands);
-    p.do_rr = g == 0;
+    p.K = p64.K = (uint32_t)std::min<size_t>(kMaxCands, k - g * kMaxCands);
+    p.j0 = p64.j0 = (uint32_t)(g * kMaxCands);
+    p.do_rr = p64.do_rr = g == 0;
     p.cands = (const uint64_t *)(dev + o_cand) + g * kMaxCands * n;
-    if ((e = (cudaError_t)launch_eq(p, grid, s)) != cudaSuccess) return fail_cuda(ctx, e);
-    ctx->launches += 1;
+    p64.cands = (const uint64_t *)(dev + o_cand64) + g * kMaxCands * n64;
+    if (tile > 0) {
+      if ((e = (cudaError_t)launch_eq(p, grid, s)) != cudaSuccess) return fail_cuda(ctx, e);
+      ctx->launches += 1;
+    }
+    if (tile64 > 0) {
+      if ((e = (cudaError_t)launch_eq64(p64, grid64, s)) != cudaSuccess) return fail_cuda(ctx, e);
+      ctx->launches += 1;
+    }
   }
   if (ctx->timing) {
     if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
@@ -792,12 +889,13 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   }
   if ((rc = after_launch(ctx, s)) != ASMV_OK) return rc;
   unsigned char *host = ctx->hst + ((img.bytes.size() + 255) & ~(size_t)255);
-  if ((e = cudaMemcpyAsync(host, dev + o_dig, dig_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+  if ((e = cudaMemcpyAsync(host, dev + o_dig, all_dig, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
     return fail_cuda(ctx, e);
   if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return fail_cuda(ctx, e);
   ctx->staged_pending = false;
   ctx->ws_pending = false;
   std::memcpy(digits.data(), host, dig_bytes);
+  if (dig64_bytes) std::memcpy(digits64.data(), host + o_dig64, dig64_bytes);
   return ASMV_OK;
 }
 
@@ -815,23 +913,21 @@ int check_eq_call(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   int rc = check_pairs(ref, cands, k, n);
   if (rc != ASMV_OK) return rc;
   for (size_t i = 0; i < n; ++i)
-    if (is_float(ref[i].dtype) &&
-        (ref[i].dtype == ASMV_F64 || ref[i].n_elems > ((uint64_t)1 << 31)))
-      return ASMV_EINVAL;
+    if (is_float(ref[i].dtype) && ref[i].n_elems > ((uint64_t)1 << 31)) return ASMV_EINVAL;
   return ASMV_OK;
 }
 
 // The statistics and the digit vectors of the Eq. 1 sums (the kernels).
 int run_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands, size_t k,
                    size_t n, const asmv_tol *tol, asmv_stream_t stream, std::vector<asmv_stats> &stats,
-                   std::vector<long long> &digits) {
+                   std::vector<long long> &digits, std::vector<long long> &digits64) {
   DeviceScope ds(ctx->device);
   if (!ds.ok) return fail_cuda(ctx, cudaErrorInvalidDevice);
   const cudaStream_t s = (cudaStream_t)stream;
   stats.assign(k * n, asmv_stats());
   int rc;
   if ((rc = run_compare(ctx, ref, cands, k, n, tol, stats.data(), s, false)) != ASMV_OK) return rc;
-  return run_eq(ctx, ref, cands, k, n, s, digits);
+  return run_eq(ctx, ref, cands, k, n, s, digits, digits64);
 }
 
 // Eq. 1 of every (candidate, region) from statistics and digit vectors: the
@@ -839,16 +935,38 @@ int run_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *con
 // vectors of the difference-form dtypes hold sum r d and sum d^2, from which
 // S_rc = S_rr + sum r d and S_cc = S_rr + 2 sum r d + sum d^2, digit by
 // digit; a digit sum that would leave the int64 range is rejected.
+//
+// Binary64 regions take their sums from digits64 (the m-th binary64 region
+// of the table at [m][1 + 2k][kEq64Digits]): each rounded with gradual
+// underflow and overflow to infinity, and the cosine formed from the sums
+// scaled by powers of two (eq_cosine_scaled).
 int eq_combine(const uint32_t *dtypes, size_t k, size_t n, const asmv_stats *stats,
-               const long long *digits, double theta, double tau, asmv_eq *res) {
+               const long long *digits, const long long *digits64, double theta, double tau,
+               asmv_eq *res) {
   const size_t nslots = 1 + 2 * k;
+  std::vector<size_t> m64(n, 0);
+  for (size_t i = 0, m = 0; i < n; ++i)
+    if (dtypes[i] == ASMV_F64) m64[i] = m++;
   for (size_t j = 0; j < k; ++j) {
     for (size_t i = 0; i < n; ++i) {
       const asmv_stats &st = stats[j * n + i];
       asmv_eq &q = res[j * n + i];
       std::memset(&q, 0, sizeof q);
       const bool flt = is_float(dtypes[i]);
-      if (flt) {
+      if (flt && dtypes[i] == ASMV_F64) {
+        if (digits64 == nullptr) return ASMV_EINVAL;
+        const long long *d = digits64 + m64[i] * nslots * kEq64Digits;
+        Magnitude rr, rc, cc;
+        magnitude_of((const int64_t *)d, kEq64Digits, &rr);
+        magnitude_of((const int64_t *)(d + (1 + 2 * j) * kEq64Digits), kEq64Digits, &rc);
+        magnitude_of((const int64_t *)(d + (2 + 2 * j) * kEq64Digits), kEq64Digits, &cc);
+        if (rr.neg || cc.neg) return ASMV_EINVAL;           // sums of squares
+        q.sum_rr = round_magnitude(rr, kEq64Base);
+        q.sum_cc = round_magnitude(cc, kEq64Base);
+        q.sum_rc = round_magnitude(rc, kEq64Base);
+        if (rc.neg) q.sum_rc = -q.sum_rc;
+        q.cos = eq_cosine_scaled(rc, rr, cc, kEq64Base);
+      } else if (flt) {
         const long long *d = digits + i * nslots * kEqDigits;
         const int base = eq_digit_base(dtypes[i]);
         int64_t rc[kEqDigits], cc[kEqDigits];
@@ -903,12 +1021,14 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
   if (!theta_tau_ok(theta, tau)) return ASMV_EINVAL;
   if (n == 0) return ASMV_OK;
   std::vector<asmv_stats> stats;
-  std::vector<long long> digits;
-  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits)) != ASMV_OK) return rc;
+  std::vector<long long> digits, digits64;
+  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits, digits64)) != ASMV_OK)
+    return rc;
   std::vector<uint32_t> dt(n);
   for (size_t i = 0; i < n; ++i) dt[i] = ref[i].dtype;
   std::vector<asmv_eq> res(k * n);
-  if (eq_combine(dt.data(), k, n, stats.data(), digits.data(), theta, tau, res.data()) != ASMV_OK)
+  if (eq_combine(dt.data(), k, n, stats.data(), digits.data(), digits64.data(), theta, tau,
+                 res.data()) != ASMV_OK)
     return ASMV_ECUDA;                                // digits out of range: a device fault
   std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
   std::memcpy(eq_host, res.data(), res.size() * sizeof(asmv_eq));
@@ -921,9 +1041,12 @@ int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_reg
   int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, digits_host);
   if (rc != ASMV_OK) return rc;
   if (n == 0) return ASMV_OK;
+  for (size_t i = 0; i < n; ++i)
+    if (ref[i].dtype == ASMV_F64) return ASMV_EINVAL;
   std::vector<asmv_stats> stats;
-  std::vector<long long> digits;
-  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits)) != ASMV_OK) return rc;
+  std::vector<long long> digits, digits64;
+  if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits, digits64)) != ASMV_OK)
+    return rc;
   std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
   std::memcpy(digits_host, digits.data(), digits.size() * sizeof(int64_t));
   return ASMV_OK;
@@ -938,7 +1061,7 @@ int asmv_eq_from_digits(const uint32_t *dtypes, size_t k, size_t n, const asmv_s
   for (size_t i = 0; i < n; ++i)
     if (dtypes[i] >= (uint32_t)ASMV_NDTYPES || dtypes[i] == ASMV_F64) return ASMV_EINVAL;
   std::vector<asmv_eq> res(k * n);
-  int rc = eq_combine(dtypes, k, n, stats, (const long long *)digits, theta, tau, res.data());
+  int rc = eq_combine(dtypes, k, n, stats, (const long long *)digits, nullptr, theta, tau, res.data());
   if (rc != ASMV_OK) return rc;
   std::memcpy(eq_out, res.data(), res.size() * sizeof(asmv_eq));
   return ASMV_OK;

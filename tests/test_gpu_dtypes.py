@@ -2,7 +2,8 @@
 binary64, int16, int64): the guarded fill byte for byte, the comparison
 field by field (bit patterns over the whole code space, special values, the
 fnuz NaN and top values, int64 differences beyond 2^53), and Eq. 1's exact
-sums for the fp8 formats, all against the oracle on the same bytes."""
+sums for the fp8 formats (binary64: test_gpu_eq64.py), all against the
+oracle on the same bytes."""
 import numpy as np
 import pytest
 
@@ -159,15 +160,6 @@ def test_eq_sums_new_fp8(ctx, oracle):
                                   ORACLE_DTYPE[r.dtype], r.n_elems)
             want = oracle.eq_verdict(st, sums, ORACLE_DTYPE[r.dtype])
             assert_stats_equal(eqs[j][i], want, "%s cand %d" % (r.dtype, j))
-
-
-def test_eq_rejects_binary64(ctx):
-    torch = torch_cuda()
-    buf = torch.zeros(1 << 16, dtype=torch.uint8, device="cuda")
-    reg = [asmv.make_region(buf.data_ptr(), 100, "f64")]
-    with pytest.raises(asmv.AsmvError) as e:
-        ctx.compare_eq(reg, [reg], W.DEFAULT_TOL)
-    assert e.value.status == asmv.EINVAL
 
 
 def test_restore_wide_types(ctx, oracle):
