@@ -250,13 +250,15 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
  * digit vectors are added element-wise over the processes and the
  * statistics merged, and asmv_eq_from_digits gives the verdict of the
  * whole -- the same result as one asmv_compare_eq over the whole regions.
- * Binary64 regions are not taken here (EINVAL): their sums need 136 digits.
  *
  * asmv_compare_eq_digits: the statistics of asmv_compare_batched in
  * stats_host[j*n + i], and the exact sums of region i in
- *   digits_host[(i*(1 + 2k) + slot) * ASMV_EQ_DIGITS + d]   (k*n, n*(1+2k)*20 entries)
+ *   digits_host[(i*(1 + 2k) + slot) * D + d]     (k*n and n*(1+2k)*D entries)
  * as signed 64-bit digits, digit d weighing 2^(32 d + base) with base =
- * asmv_eq_digit_base(dtype of region i).  Slot 0 holds sum r*r; slots
+ * asmv_eq_digit_base(dtype of region i).  D = ASMV_EQ_DIGITS (20) unless
+ * the table holds a binary64 region, whose sums need ASMV_EQ64_DIGITS
+ * (136): then D = 136 for every region, and the digits of the other
+ * regions beyond their first 20 are zero.  Slot 0 holds sum r*r; slots
  * 1 + 2j and 2 + 2j hold candidate j's two further sums (for fp16 and the
  * fp8 formats other than E4M3 these are sum r*d and sum d*d with d = c - r,
  * otherwise sum r*c and sum c*c); every slot is a sum over elements, so
@@ -264,6 +266,7 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
  * asmv_compare_eq (theta and tau are not taken), with digits_host in place
  * of eq_host.  Synchronous. */
 #define ASMV_EQ_DIGITS 20
+#define ASMV_EQ64_DIGITS 136
 int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
                            size_t k, size_t n, const asmv_tol *tol, asmv_stats *stats_host,
                            int64_t *digits_host, asmv_stream_t stream);
@@ -271,15 +274,17 @@ int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_reg
 /* Host only: the Eq. 1 results eq_out[j*n + i] (as asmv_compare_eq) from
  * statistics and digit vectors laid out as asmv_compare_eq_digits returns
  * them (possibly the sums over shards; any signed digit values are
- * accepted), for regions of dtypes[i].  Makes no CUDA call.  EINVAL for a
- * null pointer with k*n > 0, k == 0, an unknown or binary64 dtype, theta
- * or tau as asmv_compare_eq, or digits whose sum is outside the normal
- * double range. */
+ * accepted), for regions of dtypes[i] (D follows from them as above).
+ * Makes no CUDA call.  EINVAL for a null pointer with k*n > 0, k == 0, an
+ * unknown dtype, theta or tau as asmv_compare_eq, digits of a format other
+ * than binary64 whose sum is outside the normal double range (or, with
+ * D = 136, does not fit its first 20 digits), or a negative sum of squares
+ * of a binary64 region. */
 int asmv_eq_from_digits(const uint32_t *dtypes, size_t k, size_t n, const asmv_stats *stats,
                         const int64_t *digits, double theta, double tau, asmv_eq *eq_out);
 
-/* The binary weight of digit 0 of the exact sums of a float dtype other
- * than binary64, in *base.  EINVAL for other dtypes or a null base. */
+/* The binary weight of digit 0 of the exact sums of a float dtype, in
+ * *base (-2148 for binary64).  EINVAL for other dtypes or a null base. */
 int asmv_eq_digit_base(uint32_t dtype, int *base);
 
 /* The integer sum_k digits[k] * 2^(32 k + base_exp) (k < ndigits, each

@@ -33,6 +33,8 @@ OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM = 0, -1, -2, -3, -4
 def dtype_code(dtype) -> int:
     """The ABI code of a dtype name (or a code, returned as is)."""
     return DTYPE_CODE[dtype] if isinstance(dtype, str) else int(dtype)
+
+
 U64_NONE = (1 << 64) - 1
 
 
@@ -94,6 +96,7 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds",
                  "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base")
 EQ_DIGITS = 20                           # signed 64-bit digits per exact Eq. 1 sum
+EQ64_DIGITS = 136                        # ... when the region table holds a binary64 region
 NOALLOC_SCRATCH_BYTES = 1 << 20
 WAIT_ROUNDS = 20000                      # default bound of the compare's device waits
 
@@ -401,22 +404,24 @@ class Context:
     def compare_eq_digits(self, ref: Sequence, cands: Sequence[Sequence], tol, stream=None):
         """asmv_compare_eq_digits: (stats, digits) with stats[j][i] as
         compare_batched and digits[i, slot, d] the unrounded Eq. 1 sums
-        (int64, shape (n, 1 + 2k, EQ_DIGITS)): the per-shard result of a
-        check split across processes (see eq_from_digits)."""
+        (int64, shape (n, 1 + 2k, D), D = EQ_DIGITS, or EQ64_DIGITS when a
+        region is binary64): the per-shard result of a check split across
+        processes (see eq_from_digits)."""
         n, k = len(ref), len(cands)
         ra = region_array(ref)
+        nd = digits_per_slot([ra[i].dtype for i in range(n)])
         cas = [region_array(c) for c in cands]
         ptrs = (ctypes.POINTER(Region) * max(1, k))(*[ctypes.cast(c, ctypes.POINTER(Region))
                                                       for c in cas])
         st = (Stats * max(1, k * n))()
-        dig = np.zeros(max(1, n * (1 + 2 * k) * EQ_DIGITS), np.int64)
+        dig = np.zeros(max(1, n * (1 + 2 * k) * nd), np.int64)
         self._check(self._lib.asmv_compare_eq_digits(
             self._h, ra, ptrs, k, n,
             tol_array(tol) if not isinstance(tol, ctypes.Array) else tol,
             st, dig.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), _stream_handle(stream)))
         flat = stats_dicts(st, k * n)
         return ([flat[j * n:(j + 1) * n] for j in range(k)],
-                dig[:n * (1 + 2 * k) * EQ_DIGITS].reshape(n, 1 + 2 * k, EQ_DIGITS))
+                dig[:n * (1 + 2 * k) * nd].reshape(n, 1 + 2 * k, nd))
 
 
 def stats_array(stats: Sequence[dict]) -> ctypes.Array:
@@ -440,8 +445,9 @@ def eq_from_digits(dtypes: Sequence, stats: Sequence[Sequence[dict]], digits: np
     codes = (ctypes.c_uint32 * max(1, n))(*[dtype_code(d) for d in dtypes])
     st = stats_array([s for row in stats for s in row])
     dig = np.ascontiguousarray(np.asarray(digits, dtype=np.int64).reshape(-1))
-    if dig.size != n * (1 + 2 * k) * EQ_DIGITS:
-        raise ValueError("digits must have shape (n, 1 + 2k, %d)" % EQ_DIGITS)
+    nd = digits_per_slot(dtypes)
+    if dig.size != n * (1 + 2 * k) * nd:
+        raise ValueError("digits must have shape (n, 1 + 2k, %d)" % nd)
     out = (EqResult * max(1, k * n))()
     rc = lib().asmv_eq_from_digits(codes, k, n, st, dig.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
                                    float(theta), float(tau), out)
@@ -449,6 +455,12 @@ def eq_from_digits(dtypes: Sequence, stats: Sequence[Sequence[dict]], digits: np
         raise AsmvError(rc, strerror(rc))
     eqs = [{f: getattr(out[x], f) for f in EQ_FIELDS} for x in range(k * n)]
     return [eqs[j * n:(j + 1) * n] for j in range(k)]
+
+
+def digits_per_slot(dtypes: Sequence) -> int:
+    """Digits per exact sum in the digit-vector calls for a table of these
+    dtypes: EQ64_DIGITS if any region is binary64, else EQ_DIGITS."""
+    return EQ64_DIGITS if any(dtype_code(d) == F64 for d in dtypes) else EQ_DIGITS
 
 
 def eq_digit_base(dtype) -> int:

@@ -30,6 +30,7 @@ static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout"
 static_assert(sizeof(CopyRegion) == 48, "copy region layout");
 static_assert(kWaitRounds == ASMV_WAIT_ROUNDS, "default wait bound");
 static_assert(kEqDigits == ASMV_EQ_DIGITS, "Eq. 1 digits");
+static_assert(kEq64Digits == ASMV_EQ64_DIGITS, "Eq. 1 digits of binary64");
 static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
               "plan layouts");
 
@@ -1041,14 +1042,31 @@ int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_reg
   int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, digits_host);
   if (rc != ASMV_OK) return rc;
   if (n == 0) return ASMV_OK;
-  for (size_t i = 0; i < n; ++i)
-    if (ref[i].dtype == ASMV_F64) return ASMV_EINVAL;
   std::vector<asmv_stats> stats;
   std::vector<long long> digits, digits64;
   if ((rc = run_compare_eq(ctx, ref, cands, k, n, tol, stream, stats, digits, digits64)) != ASMV_OK)
     return rc;
   std::memcpy(stats_host, stats.data(), stats.size() * sizeof(asmv_stats));
-  std::memcpy(digits_host, digits.data(), digits.size() * sizeof(int64_t));
+  if (digits64.empty()) {
+    std::memcpy(digits_host, digits.data(), digits.size() * sizeof(int64_t));
+    return ASMV_OK;
+  }
+  // a table with binary64 regions: every slot takes kEq64Digits digits
+  const size_t nslots = 1 + 2 * k;
+  size_t m = 0;
+  for (size_t i = 0; i < n; ++i) {
+    int64_t *dst = digits_host + i * nslots * kEq64Digits;
+    if (ref[i].dtype == ASMV_F64) {
+      std::memcpy(dst, digits64.data() + m * nslots * kEq64Digits, nslots * kEq64Digits * sizeof(int64_t));
+      ++m;
+      continue;
+    }
+    for (size_t sl = 0; sl < nslots; ++sl) {
+      std::memcpy(dst + sl * kEq64Digits, digits.data() + (i * nslots + sl) * kEqDigits,
+                  kEqDigits * sizeof(int64_t));
+      std::memset(dst + sl * kEq64Digits + kEqDigits, 0, (kEq64Digits - kEqDigits) * sizeof(int64_t));
+    }
+  }
   return ASMV_OK;
 }
 
@@ -1058,19 +1076,50 @@ int asmv_eq_from_digits(const uint32_t *dtypes, size_t k, size_t n, const asmv_s
   if (n == 0) return ASMV_OK;
   if (dtypes == nullptr || stats == nullptr || digits == nullptr || eq_out == nullptr) return ASMV_EINVAL;
   if (k > (size_t)0x7FFFFFFF / n) return ASMV_EINVAL;
-  for (size_t i = 0; i < n; ++i)
-    if (dtypes[i] >= (uint32_t)ASMV_NDTYPES || dtypes[i] == ASMV_F64) return ASMV_EINVAL;
+  size_t n64 = 0;
+  for (size_t i = 0; i < n; ++i) {
+    if (dtypes[i] >= (uint32_t)ASMV_NDTYPES) return ASMV_EINVAL;
+    n64 += dtypes[i] == ASMV_F64;
+  }
   std::vector<asmv_eq> res(k * n);
-  int rc = eq_combine(dtypes, k, n, stats, (const long long *)digits, nullptr, theta, tau, res.data());
+  int rc;
+  if (n64 == 0) {
+    rc = eq_combine(dtypes, k, n, stats, (const long long *)digits, nullptr, theta, tau, res.data());
+  } else {
+    // kEq64Digits per slot: split into the two layouts eq_combine reads
+    const size_t nslots = 1 + 2 * k;
+    std::vector<long long> d20(n * nslots * kEqDigits, 0), d64(n64 * nslots * kEq64Digits);
+    for (size_t i = 0, m = 0; i < n; ++i) {
+      const int64_t *src = digits + i * nslots * kEq64Digits;
+      if (dtypes[i] == ASMV_F64) {
+        std::memcpy(d64.data() + m * nslots * kEq64Digits, src, nslots * kEq64Digits * sizeof(int64_t));
+        ++m;
+        continue;
+      }
+      // the digits past this format's 20 (all -1 words for a carried negative
+      // sum) fold into its top digit, which must stay in int64
+      for (size_t sl = 0; sl < nslots; ++sl) {
+        const int64_t *x = src + sl * kEq64Digits;
+        long long *y = d20.data() + (i * nslots + sl) * kEqDigits;
+        __int128 top = 0;
+        for (int d = kEq64Digits - 1; d >= kEqDigits - 1; --d) {
+          top = top * ((__int128)1 << 32) + x[d];
+          if (top > INT64_MAX || top < INT64_MIN) return ASMV_EINVAL;
+        }
+        std::memcpy(y, x, (kEqDigits - 1) * sizeof(int64_t));
+        y[kEqDigits - 1] = (long long)top;
+      }
+    }
+    rc = eq_combine(dtypes, k, n, stats, d20.data(), d64.data(), theta, tau, res.data());
+  }
   if (rc != ASMV_OK) return rc;
   std::memcpy(eq_out, res.data(), res.size() * sizeof(asmv_eq));
   return ASMV_OK;
 }
 
 int asmv_eq_digit_base(uint32_t dtype, int *base) {
-  if (base == nullptr || dtype >= (uint32_t)ASMV_NDTYPES || !is_float(dtype) || dtype == ASMV_F64)
-    return ASMV_EINVAL;
-  *base = eq_digit_base(dtype);
+  if (base == nullptr || dtype >= (uint32_t)ASMV_NDTYPES || !is_float(dtype)) return ASMV_EINVAL;
+  *base = dtype == ASMV_F64 ? kEq64Base : eq_digit_base(dtype);
   return ASMV_OK;
 }
 

@@ -135,12 +135,14 @@ def allreduce_stats(per_region: Sequence[Dict], group=None) -> List[Dict]:
     return out
 
 
-def normalize_digits(digits, ndigits: int = 20):
-    """Carry every digit vector along its last axis so that each digit but
-    the top one lies in [0, 2^32) (the integer it represents is unchanged):
-    a sum over many processes then keeps every digit far inside int64."""
+def normalize_digits(digits, ndigits: int = None):
+    """Carry every digit vector along its last axis (ndigits digits, by
+    default the length of that axis) so that each digit but the top one lies
+    in [0, 2^32) (the integer it represents is unchanged): a sum over many
+    processes then keeps every digit far inside int64."""
     import numpy as np
     d = np.asarray(digits, dtype=np.int64)
+    ndigits = d.shape[-1] if ndigits is None else ndigits
     flat = d.reshape(-1, ndigits)
     out = np.zeros_like(flat)
     for r in range(flat.shape[0]):

@@ -28,7 +28,7 @@ def _workload():
     from oracle import oracle as O
     regs = []
     for i, (dt, n) in enumerate([("f32", 100003), ("bf16", 7), ("f16", 65536), ("f8e4m3", 999),
-                                 ("i32", 4097), ("i8", 1), ("u8", 123457)]):
+                                 ("i32", 4097), ("i8", 1), ("u8", 123457), ("f64", 5001)]):
         dist_ = "normal" if dt in W.FLOAT_DTYPES else "raw"
         regs.append(W.Region("r%d" % i, dt, n, dist_, 0.0, 1.0, 64 + i, 128, 0xA5, i))
     size = W.layout(regs)
@@ -40,14 +40,19 @@ def _workload():
     cand_t = torch.from_numpy(ref.copy())
     rng = np.random.default_rng(5)
     for r in regs:
-        W.perturb_sparse(cand_t, r, rng, rate=0.01)
+        if r.dtype == "f64":              # low-bit flips at 1 % of the values
+            v = cand_t[r.payload_offset:r.payload_offset + r.payload_bytes].numpy().view(np.uint64)
+            v[rng.random(v.size) < 0.01] ^= np.uint64(3)
+        else:
+            W.perturb_sparse(cand_t, r, rng, rate=0.01)
         if r.guard_hi:
             W.corrupt_guard(cand_t, r, rng, "hi")
     W.corrupt_guard(cand_t, regs[2], rng, "lo")
     return regs, ref, cand_t.numpy()
 
 
-TOL = {"f32": (1e-5, 1e-5), "bf16": (1e-2, 1.6e-2), "f16": (1e-5, 1e-3), "f8e4m3": (1e-5, 0.125)}
+TOL = {"f32": (1e-5, 1e-5), "bf16": (1e-2, 1.6e-2), "f16": (1e-5, 1e-3), "f8e4m3": (1e-5, 0.125),
+       "f64": (1e-9, 1e-9)}
 
 
 def _region_stats(O, ref, cand, r, shift_ref_alloc, s):
@@ -128,15 +133,17 @@ def _eq_worker(rank, world, port, out):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
         from oracle import oracle as O
+        from paper_2608_20711_gb300 import asmv
         from tests.test_eq_digits import full_stats, shard_digits
         regs, ref, cand = _workload()
         flt = [r for r in regs if r.dtype in W.FLOAT_DTYPES]
+        nd = asmv.digits_per_slot([r.dtype for r in flt])
         digs, parts = [], []
         for r in flt:
             a, b = D.slice_bounds(r.n_elems, W.DTYPE_SIZE[r.dtype], rank, world)
             off = r.payload_offset
             rp, cp = ref[off:off + r.payload_bytes], cand[off:off + r.payload_bytes]
-            digs.append(shard_digits(O, rp, [cp], r.dtype, a, b))
+            digs.append(shard_digits(O, rp, [cp], r.dtype, a, b, nd=nd))
             t = TOL[r.dtype]
             parts.append(D.to_region_coordinates(full_stats(O, rp, cp, r.dtype, a, b, t), a, 0))
         merged_digits = D.allreduce_digits(np.stack(digs))
