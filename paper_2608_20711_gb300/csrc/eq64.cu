@@ -10,20 +10,24 @@
 // t = E - kEq64Base, the product is the five 32-bit words of
 // M << (t mod 32) placed at digits q .. q+4, q = t div 32.
 //
-// Reduction.  A lane handles two values (one 16-byte chunk) per step; the
-// products of a warp that share q add their words with one redux per 16-bit
-// half (64 halves sum below 2^22) and five lanes add the recombined words to
-// the CTA's shared digits; a warp repeats this once per distinct q among its
-// products, which is one or two for values of similar magnitude.  The CTA
-// adds its shared digits to the region's global digits when it leaves the
-// region.  Every element adds less than 2^32 to any one digit and a region
-// holds at most 2^31 elements, so no digit, shared or global, leaves the
-// int64 range; the host carries and rounds.
+// Reduction.  The tile is passed over once for S_rr and once per candidate
+// (S_rc and S_cc together; the reference comes from L1 after the first
+// pass).  In a pass every lane keeps a window of six 64-bit digits
+// qa .. qa+5 per sum, qa the lowest q among the warp's first products; a
+// product starting at qa or qa + 1 is added to the window with one select
+// and one 64-bit add per digit, and any other product (rare for values of
+// one scale) goes to the CTA's shared digits with five atomics.  At the end
+// of the pass the warp sums each window digit with three reduxes (two 16-bit
+// pieces and the signed rest) and six lanes add the results to the shared
+// digits.  The CTA adds its shared digits to the region's global digits when
+// it leaves the region.  Every element adds less than 2^32 to any one digit
+// and a region holds at most 2^31 elements, so no digit, shared or global,
+// leaves the int64 range; the host carries and rounds.
 //
 // Work split: a persistent grid over 16 KiB tiles of the reference payloads
 // (2048 values); CTA b takes the contiguous tile range [T b / G,
-// T (b+1) / G); within a tile, thread t reads the 16-byte chunks t, t + 256,
-// ... of the reference and of each candidate in turn.
+// T (b+1) / G); within a pass, thread t reads the 16-byte chunks t, t + 256,
+// ... of the tile.
 #include <cuda_runtime.h>
 #include "device.cuh"
 #include "eq64.h"
@@ -71,54 +75,94 @@ __device__ __forceinline__ uint32_t product_words(const F64Parts &a, const F64Pa
   return t >> 5;
 }
 
-// Add the products a0 b0 and a1 b1 (each with sign (-1)^neg when SIGNED,
-// and only where ok0 / ok1 hold and both factors are non-zero) to the
-// digits acc.  All 32 lanes of the warp call this together.  Each round
-// takes the lowest digit index qq still pending in the warp: every lane
-// adds the 16-bit halves of its products placed at qq (at most two, so a
-// lane's half sums stay below 2^17 and a warp's below 2^22), one redux per
-// half sums them over the warp, and lanes 0..4 add the five recombined
-// words to digits qq .. qq+4.
-template <bool SIGNED>
-__device__ __forceinline__ void warp_add_pair(long long *acc, bool ok0, uint32_t neg0, const F64Parts &a0,
-                                              const F64Parts &b0, bool ok1, uint32_t neg1,
-                                              const F64Parts &a1, const F64Parts &b1) {
-  const uint32_t lane = threadIdx.x & 31u;
-  uint32_t w0[5] = {0u, 0u, 0u, 0u, 0u}, w1[5] = {0u, 0u, 0u, 0u, 0u};
-  uint32_t q0 = 0xFFFFFFFFu, q1 = 0xFFFFFFFFu;                      // 0xFFFFFFFF: nothing pending
-  if (ok0 && a0.m != 0ull && b0.m != 0ull) q0 = product_words(a0, b0, w0);
-  if (ok1 && a1.m != 0ull && b1.m != 0ull) q1 = product_words(a1, b1, w1);
-  while (__any_sync(kFull, (q0 & q1) != 0xFFFFFFFFu)) {
-    const uint32_t qq = __reduce_min_sync(kFull, min(q0, q1));
-    const bool m0 = q0 == qq, m1 = q1 == qq;
-    if (m0) q0 = 0xFFFFFFFFu;
-    if (m1) q1 = 0xFFFFFFFFu;
-    long long word = 0;
+constexpr uint32_t kNoAnchor = 0xFFFFFFFFu;
+
+// One product: its words, its digit index q (kNoAnchor when the product is
+// zero or skipped) and its sign.
+struct Prod {
+  uint32_t w[5];
+  uint32_t q;
+  uint32_t neg;
+};
+
+__device__ __forceinline__ Prod make_prod(bool ok, uint32_t neg, const F64Parts &a, const F64Parts &b) {
+  Prod P;
+  P.neg = neg;
+  P.q = kNoAnchor;
 #pragma unroll
-    for (int k = 0; k < 5; ++k) {
-      int lo = 0, hi = 0;
-      if (m0) {
-        const int l = (int)(w0[k] & 0xFFFFu), h = (int)(w0[k] >> 16);
-        lo += (SIGNED && neg0) ? -l : l;
-        hi += (SIGNED && neg0) ? -h : h;
-      }
-      if (m1) {
-        const int l = (int)(w1[k] & 0xFFFFu), h = (int)(w1[k] >> 16);
-        lo += (SIGNED && neg1) ? -l : l;
-        hi += (SIGNED && neg1) ? -h : h;
-      }
-      const int slo = (int)__reduce_add_sync(kFull, (uint32_t)lo);
-      const int shi = (int)__reduce_add_sync(kFull, (uint32_t)hi);
-      if (lane == (uint32_t)k) word = (long long)slo + ((long long)shi << 16);
+  for (int k = 0; k < 5; ++k) P.w[k] = 0u;
+  if (ok && a.m != 0ull && b.m != 0ull) P.q = product_words(a, b, P.w);
+  return P;
+}
+
+// A lane's window on one sum: digits qa .. qa+5, each a signed 64-bit sum
+// of at most eight words below 2^32 (|d| < 2^35).  qa is the same in every
+// lane.
+struct Win {
+  long long d[6];
+  uint32_t qa;
+};
+
+__device__ __forceinline__ void win_reset(Win &W) {
+#pragma unroll
+  for (int j = 0; j < 6; ++j) W.d[j] = 0;
+  W.qa = kNoAnchor;
+}
+
+// Anchor a window still without one at the lowest digit index among the
+// warp's products p0, p1 (all 32 lanes call this together).
+__device__ __forceinline__ void win_anchor(Win &W, const Prod &p0, const Prod &p1) {
+  if (W.qa == kNoAnchor) W.qa = __reduce_min_sync(kFull, min(p0.q, p1.q));
+}
+
+// Add one product: into the window when it starts at digit qa or qa + 1,
+// else (rare for values of one scale) straight to the shared digits acc.
+template <bool SIGNED>
+__device__ __forceinline__ void win_add(Win &W, const Prod &P, long long *acc) {
+  if (P.q == kNoAnchor) return;
+  const uint32_t o = P.q - W.qa;                  // wraps for q < qa: out of the window
+  const bool neg = SIGNED && P.neg;
+  if (o <= 1u) {
+#pragma unroll
+    for (int i = 0; i < 6; ++i) {
+      const uint32_t a = i < 5 ? P.w[i] : 0u, b = i >= 1 ? P.w[i - 1] : 0u;
+      const long long x = (long long)(o == 0u ? a : b);
+      W.d[i] += neg ? -x : x;
     }
-    if (lane < 5u && word != 0)
-      atomicAdd(reinterpret_cast<unsigned long long *>(acc + qq + lane), (unsigned long long)word);
+  } else {
+#pragma unroll
+    for (int k = 0; k < 5; ++k)
+      if (P.w[k] != 0u)
+        atomicAdd(reinterpret_cast<unsigned long long *>(acc + P.q + k),
+                  neg ? (unsigned long long)(-(long long)P.w[k]) : (unsigned long long)P.w[k]);
   }
 }
 
-__device__ __forceinline__ uint4 load16(uint64_t addr, uint32_t n, uint32_t vec) {
+// Sum the window over the warp and add its six digits to acc; all 32
+// lanes call this together.  A digit (|d| < 2^35) is cut into two 16-bit
+// pieces and the signed rest, whose warp sums fit in 32 bits.
+__device__ __forceinline__ void win_flush(Win &W, long long *acc) {
+  if (W.qa == kNoAnchor) return;                  // warp-uniform
+  const uint32_t lane = threadIdx.x & 31u;
+  long long word = 0;
+#pragma unroll
+  for (int i = 0; i < 6; ++i) {
+    const long long v = W.d[i];
+    const uint32_t s0 = __reduce_add_sync(kFull, (uint32_t)v & 0xFFFFu);
+    const uint32_t s1 = __reduce_add_sync(kFull, (uint32_t)(v >> 16) & 0xFFFFu);
+    const int s2 = (int)__reduce_add_sync(kFull, (uint32_t)(int)(v >> 32));
+    if (lane == (uint32_t)i)
+      word = (long long)s0 + ((long long)s1 << 16) + ((long long)s2 << 32);
+  }
+  if (lane < 6u && word != 0)
+    atomicAdd(reinterpret_cast<unsigned long long *>(acc + W.qa + lane), (unsigned long long)word);
+}
+
+// 16 bytes (n of them; the rest zero), through L1 when `cached`.
+__device__ __forceinline__ uint4 load16(uint64_t addr, uint32_t n, uint32_t vec, bool cached) {
   if (n == 0u) return make_uint4(0u, 0u, 0u, 0u);
-  return (vec && n == 16u) ? ldg16(addr) : load_bytes(addr, n);
+  if (!vec || n != 16u) return load_bytes(addr, n);
+  return cached ? __ldg(reinterpret_cast<const uint4 *>(addr)) : ldg16(addr);
 }
 
 __device__ __forceinline__ uint64_t lo64(const uint4 &v) { return (uint64_t)v.y << 32 | v.x; }
@@ -157,22 +201,51 @@ __global__ void __launch_bounds__(kThreads) eq64_kernel(Eq64Params p) {
     }
     const uint64_t a = (t - R.tile0) * kEq64TileBytes;
     const uint32_t nb = (uint32_t)umin64(kEq64TileBytes, R.bytes - a);
+    // one pass over the tile per sum (S_rr), then per candidate (S_rc and
+    // S_cc together); the reference tile comes from L1 after the first pass
+    if (p.do_rr) {
+      Win W;
+      win_reset(W);
 #pragma unroll 1
-    for (uint32_t c0 = 0; 16u * c0 < nb; c0 += kThreads) {       // the same trip count for every thread
-      const uint32_t off = 16u * (c0 + threadIdx.x);
-      const uint32_t n = off < nb ? min(16u, nb - off) : 0u;    // bytes past the payload read as zero
-      const uint4 rv = load16(R.ref + a + off, n, R.vec);
-      const F64Parts r0 = split_f64(lo64(rv)), r1 = split_f64(hi64(rv));
-      if (p.do_rr) warp_add_pair<false>(sdig, r0.fin, 0u, r0, r0, r1.fin, 0u, r1, r1);
-#pragma unroll 1
-      for (uint32_t j = 0; j < p.K; ++j) {
-        const uint4 cv = load16(p.cands[(size_t)j * p.nregions + i] + a + off, n, R.vec);
-        const F64Parts c0 = split_f64(lo64(cv)), c1 = split_f64(hi64(cv));
-        long long *rc = sdig + (1 + 2 * j) * kEq64Digits, *cc = rc + kEq64Digits;
-        warp_add_pair<true>(rc, r0.fin && c0.fin, r0.neg ^ c0.neg, r0, c0,
-                            r1.fin && c1.fin, r1.neg ^ c1.neg, r1, c1);
-        warp_add_pair<false>(cc, c0.fin, 0u, c0, c0, c1.fin, 0u, c1, c1);
+      for (uint32_t c0 = 0; 16u * c0 < nb; c0 += kThreads) {     // the same trip count for every thread
+        const uint32_t off = 16u * (c0 + threadIdx.x);
+        const uint32_t n = off < nb ? min(16u, nb - off) : 0u;  // bytes past the payload read as zero
+        const uint4 rv = load16(R.ref + a + off, n, R.vec, true);
+        const F64Parts r0 = split_f64(lo64(rv)), r1 = split_f64(hi64(rv));
+        const Prod p0 = make_prod(r0.fin, 0u, r0, r0), p1 = make_prod(r1.fin, 0u, r1, r1);
+        win_anchor(W, p0, p1);
+        win_add<false>(W, p0, sdig);
+        win_add<false>(W, p1, sdig);
       }
+      win_flush(W, sdig);
+    }
+#pragma unroll 1
+    for (uint32_t j = 0; j < p.K; ++j) {
+      const uint64_t cb = p.cands[(size_t)j * p.nregions + i] + a;
+      long long *rc = sdig + (1 + 2 * j) * kEq64Digits, *cc = rc + kEq64Digits;
+      Win Wrc, Wcc;
+      win_reset(Wrc);
+      win_reset(Wcc);
+#pragma unroll 1
+      for (uint32_t c0 = 0; 16u * c0 < nb; c0 += kThreads) {
+        const uint32_t off = 16u * (c0 + threadIdx.x);
+        const uint32_t n = off < nb ? min(16u, nb - off) : 0u;
+        const uint4 rv = load16(R.ref + a + off, n, R.vec, true);
+        const uint4 cv = load16(cb + off, n, R.vec, false);
+        const F64Parts r0 = split_f64(lo64(rv)), r1 = split_f64(hi64(rv));
+        const F64Parts c0v = split_f64(lo64(cv)), c1v = split_f64(hi64(cv));
+        const Prod x0 = make_prod(r0.fin && c0v.fin, r0.neg ^ c0v.neg, r0, c0v);
+        const Prod x1 = make_prod(r1.fin && c1v.fin, r1.neg ^ c1v.neg, r1, c1v);
+        win_anchor(Wrc, x0, x1);
+        win_add<true>(Wrc, x0, rc);
+        win_add<true>(Wrc, x1, rc);
+        const Prod y0 = make_prod(c0v.fin, 0u, c0v, c0v), y1 = make_prod(c1v.fin, 0u, c1v, c1v);
+        win_anchor(Wcc, y0, y1);
+        win_add<false>(Wcc, y0, cc);
+        win_add<false>(Wcc, y1, cc);
+      }
+      win_flush(Wrc, rc);
+      win_flush(Wcc, cc);
     }
   }
   if (cur != 0xFFFFFFFFu) cta_flush64(p, cur, sdig);
