@@ -55,7 +55,8 @@
 //
 // Roofline: HBM reads of reference + candidate payloads (reference once per
 // launch of up to 8 candidates); the screen costs about 10 fp32 operations
-// per differing element, so dense small differences are also ALU-heavy.
+// per differing element (its three thresholds on packed f32x2 for the 16-
+// and 8-bit formats), so dense small differences are also ALU-heavy.
 #include <float.h>
 #include <math_constants.h>
 #include <atomic>
@@ -308,6 +309,31 @@ __device__ __forceinline__ uint32_t screen(float r, float s, float Tp, const Tol
   return bad ? 1u : 0u;
 }
 
+__device__ __forceinline__ float2 ffma2_rd(float2 a, float2 b, float2 c) {
+  unsigned long long d;
+  asm("fma.rm.f32x2 %0, %1, %2, %3;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<unsigned long long *>(&a)), "l"(*reinterpret_cast<unsigned long long *>(&b)),
+        "l"(*reinterpret_cast<unsigned long long *>(&c)));
+  return *reinterpret_cast<float2 *>(&d);
+}
+
+// screen() of the two elements of a pair, their three bounds formed by
+// packed fp32 multiply-adds (each lane rounded exactly as the scalar one).
+// Returns the definite-mismatch bits (element 0 in bit 0).
+__device__ __forceinline__ uint32_t screen2(float2 r, float2 s, float Tp, const TolF &t, bool &rare,
+                                           float &cm) {
+  const float2 ar = make_float2(fabsf(r.x), fabsf(r.y));
+  const float2 lo = __ffma2_rn(make_float2(t.rlo, t.rlo), ar, make_float2(t.alo, t.alo));
+  const float2 hi = __ffma2_rn(make_float2(t.rhi, t.rhi), ar, make_float2(t.ahi, t.ahi));
+  const float2 y = ffma2_rd(make_float2(Tp, Tp), ar, make_float2(0x1p-149f, 0x1p-149f));
+  const float a0 = fabsf(s.x), a1 = fabsf(s.y);
+  const bool ok0 = a0 < lo.x, bad0 = a0 > hi.x, ok1 = a1 < lo.y, bad1 = a1 > hi.y;
+  rare |= (!(ok0 | bad0)) | (a0 >= y.x) | (!(ok1 | bad1)) | (a1 >= y.y);
+  cm = fmaxf(cm, fmaxf(a0, a1));
+  return (bad0 ? 1u : 0u) | (bad1 ? 2u : 0u);
+}
+
 // One 16-byte chunk whose first element has index e0.
 //  - Equal chunks cost one comparison.
 //  - 16- and 8-bit floats subtract in their own format (one packed
@@ -347,9 +373,9 @@ __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e
                                         *reinterpret_cast<const __nv_bfloat162 *>(&rw));
       acc = __hfma2(s2, zero, acc);
       const uint32_t sw = *reinterpret_cast<const uint32_t *>(&s2);
-      bad |= screen(__uint_as_float(rw << 16), __uint_as_float(sw << 16), Tp, t, rare, cm) << (2 * w);
-      bad |= screen(__uint_as_float(rw & 0xFFFF0000u), __uint_as_float(sw & 0xFFFF0000u), Tp, t, rare,
-                    cm) << (2 * w + 1);
+      bad |= screen2(make_float2(__uint_as_float(rw << 16), __uint_as_float(rw & 0xFFFF0000u)),
+                     make_float2(__uint_as_float(sw << 16), __uint_as_float(sw & 0xFFFF0000u)), Tp, t,
+                     rare, cm) << (2 * w);
     }
     const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
     rare |= (aw & 0x7FFF7FFFu) != 0u;
@@ -369,10 +395,7 @@ __device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e
       const __half2 s2 = __hsub2(*reinterpret_cast<const __half2 *>(&cw),
                                  *reinterpret_cast<const __half2 *>(&rw));
       acc = __hfma2(s2, zero, acc);
-      const float2 rf = f16x2_to_f32(rw);
-      const float2 sf = __half22float2(s2);
-      bad |= screen(rf.x, sf.x, Tp, t, rare, cm) << (2 * w);
-      bad |= screen(rf.y, sf.y, Tp, t, rare, cm) << (2 * w + 1);
+      bad |= screen2(f16x2_to_f32(rw), __half22float2(s2), Tp, t, rare, cm) << (2 * w);
     }
     const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
     rare |= (aw & 0x7FFF7FFFu) != 0u;
