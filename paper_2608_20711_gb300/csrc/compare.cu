@@ -28,18 +28,18 @@
 //      elements update an fp32 running maximum m32 with fmaxf, exactly.
 //      Every other element goes to the exact path, which keeps the fp64
 //      maximum of RN64(D).  max_abs = max(m32, that maximum).
-//  (4) max_rel: a thread keeps its exact maximum Rmax and T <= Rmax(1-2^-19)
-//      in fp32.  An element can exceed Rmax only if as > T*|r| (the
-//      relative error of as/|r| against d/|r| is below 2^-23).  The screen
-//      flags as >= y, y = RD32(Tp*|r| + 2^-149) (one fma rounded down),
-//      Tp = min(T, 1/2 -).  as lies on the fp32 grid, whose spacing is at
-//      least 2^-149: if as > Tp*|r| then either as >= Tp*|r| + 2^-149 >= y,
-//      or Tp*|r| + 2^-149 lies in (as, as + 2^-149) and rounds down to as;
-//      as = 0 (relative error 0) is never flagged, since y >= 2^-149.
-//      Flagged elements get the exact RN64(d/|r|) (one fma decides
-//      as > T*|r| exactly in sign).  Since y < |r|/2 for normal r, and a
-//      subnormal r makes every nonzero inexact difference exceed y, every
-//      element whose c - r may be inexact is flagged as well.
+//  (4) max_rel: a thread keeps its exact maximum Rmax and T = RD32(Rmax).
+//      An element with as < |r|/2 is plain (as = D = d, see (3)), and it
+//      can raise the maximum only if RN64(D/|r|) > Rmax, hence only if
+//      D/|r| > Rmax >= T, i.e. as > T*|r| (RN64 is monotone and Rmax is a
+//      double).  The screen flags as > y, y = RD32(Tp*|r|) (one fma rounded
+//      down), Tp = min(T, 1/2 -): as > Tp*|r| >= y.  An element whose
+//      relative error equals Rmax (as = T*|r| exactly) is not flagged and
+//      cannot change the maximum; as = 0 is never flagged.  Flagged
+//      elements get the exact RN64(d/|r|).  Since y <= Tp*|r| < |r|/2,
+//      every element with as >= |r|/2 -- every element whose c - r may be
+//      inexact -- is flagged as well, and r = 0 makes y = 0, so every
+//      nonzero difference from a zero reference is flagged.
 // The maxima are order-independent (max of exact values), counts are sums
 // and first_mismatch a minimum, so any grid gives bit-identical results.
 //
@@ -83,7 +83,7 @@ __device__ __forceinline__ unsigned long long dbits(double x) {
 }
 
 __device__ __forceinline__ float tfloor(double d) {
-  return __fmul_rd(__double2float_rd(d), 0x1.ffffcp-1f);    // <= d (1 - 2^-19)
+  return __double2float_rd(d);                               // <= d
 }
 
 __device__ __forceinline__ void rel_update(Hot &h, double d, double r64) {
@@ -301,10 +301,10 @@ __device__ __forceinline__ uint32_t screen(float r, float s, float Tp, const Tol
   const float as = fabsf(s), ar = fabsf(r);
   const float lo = __fmaf_rn(t.rlo, ar, t.alo);
   const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
-  const float y = __fmaf_rd(Tp, ar, 0x1p-149f);
+  const float y = __fmul_rd(Tp, ar);
   const bool ok = as < lo;
   const bool bad = as > hi;
-  rare |= (!(ok | bad)) | (as >= y);
+  rare |= (!(ok | bad)) | (as > y);
   cm = fmaxf(cm, as);
   return bad ? 1u : 0u;
 }
@@ -326,10 +326,10 @@ __device__ __forceinline__ uint32_t screen2(float2 r, float2 s, float Tp, const 
   const float2 ar = make_float2(fabsf(r.x), fabsf(r.y));
   const float2 lo = __ffma2_rn(make_float2(t.rlo, t.rlo), ar, make_float2(t.alo, t.alo));
   const float2 hi = __ffma2_rn(make_float2(t.rhi, t.rhi), ar, make_float2(t.ahi, t.ahi));
-  const float2 y = ffma2_rd(make_float2(Tp, Tp), ar, make_float2(0x1p-149f, 0x1p-149f));
+  const float2 y = ffma2_rd(make_float2(Tp, Tp), ar, make_float2(0.0f, 0.0f));   // RD32(Tp*|r|)
   const float a0 = fabsf(s.x), a1 = fabsf(s.y);
   const bool ok0 = a0 < lo.x, bad0 = a0 > hi.x, ok1 = a1 < lo.y, bad1 = a1 > hi.y;
-  rare |= (!(ok0 | bad0)) | (a0 >= y.x) | (!(ok1 | bad1)) | (a1 >= y.y);
+  rare |= (!(ok0 | bad0)) | (a0 > y.x) | (!(ok1 | bad1)) | (a1 > y.y);
   cm = fmaxf(cm, fmaxf(a0, a1));
   return (bad0 ? 1u : 0u) | (bad1 ? 2u : 0u);
 }
