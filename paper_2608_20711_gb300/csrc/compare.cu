@@ -93,6 +93,15 @@ __device__ __forceinline__ void rel_update(Hot &h, double d, double r64) {
   if (b > h.drel) { h.drel = b; h.T = tfloor(rel); }
 }
 
+// rel_update for the binary64 and integer paths, where every differing
+// element comes here: the exact RN64(d/|r|) enters the maximum only if it
+// can exceed it, and a negative RN64(d - T|r|) (one fma; negative only when
+// the exact value is) proves d/|r| < T <= Rmax, so the division is skipped.
+__device__ __forceinline__ void rel_update_guarded(Hot &h, double d, double r64) {
+  if (__fma_rn(-(double)h.T, fabs(r64), d) < 0.0) return;
+  rel_update(h, d, r64);
+}
+
 // Exact fp64 evaluation of one float pair; returns the mismatch bit.
 __device__ __forceinline__ uint32_t exact_float(float r, float c, Hot &h, const TolF &t) {
   const bool rn = isnan(r), cn = isnan(c), ri = isinf(r), ci = isinf(c);
@@ -120,7 +129,7 @@ __device__ __forceinline__ uint32_t exact_double(double r64, double c64, Hot &h,
   const double d = fabs(__dsub_rn(c64, r64));
   const double bound = __dadd_rn(t.atol, __dmul_rn(t.rtol, fabs(r64)));
   h.dabs = umax64(h.dabs, dbits(d));
-  rel_update(h, d, r64);
+  rel_update_guarded(h, d, r64);
   return d > bound ? 1u : 0u;
 }
 
@@ -131,7 +140,7 @@ __device__ __forceinline__ void exact_int64(long long r, long long c, Hot &h) {
                                           : (unsigned long long)r - (unsigned long long)c;
   const double d = __ull2double_rn(dlo);               // |c - r| < 2^64 fits the unsigned difference
   h.dabs = umax64(h.dabs, dbits(d));
-  rel_update(h, d, __ll2double_rn(r));
+  rel_update_guarded(h, d, __ll2double_rn(r));
 }
 
 // Exact evaluation of one differing integer pair (always a mismatch).
@@ -139,7 +148,7 @@ __device__ __forceinline__ void exact_int(int64_t r, int64_t c, Hot &h) {
   const int64_t dd = c - r;
   const double d = (double)(dd < 0 ? -dd : dd);     // exact: |d| < 2^33
   h.dabs = umax64(h.dabs, dbits(d));
-  rel_update(h, d, (double)r);
+  rel_update_guarded(h, d, (double)r);
 }
 
 __device__ __forceinline__ uint32_t word_of(const uint4 &v, int w) {
@@ -222,7 +231,7 @@ __device__ __forceinline__ uint32_t settle_float(float r, float c, Hot &h, const
   const bool plain = as < __fmul_rn(0.5f, ar);          // c - r exact (Sterbenz)
   if ((ok | bad) && plain) {
     h.m32 = fmaxf(h.m32, as);
-    if (__fmaf_rn(-h.T, ar, as) > 0.0f) rel_update(h, (double)as, (double)r);
+    if (!(__fmaf_rn(-h.T, ar, as) < 0.0f)) rel_update(h, (double)as, (double)r);
     return bad ? 1u : 0u;
   }
   return exact_float(r, c, h, t);
