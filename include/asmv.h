@@ -292,7 +292,9 @@ int asmv_eq_digit_base(uint32_t dtype, int *base);
  * the conversion asmv_compare_eq applies to its exact sums.  Host only,
  * makes no CUDA call.  EINVAL for a null pointer, ndigits outside
  * [1, 64], or a result outside the normal double range (which the sums of
- * asmv_compare_eq never reach). */
+ * the formats other than binary64 never reach; asmv_compare_eq rounds the
+ * 136-digit binary64 sums itself, with gradual underflow and overflow to
+ * +-Inf). */
 int asmv_exact_to_double(const int64_t *digits, int ndigits, int base_exp, double *out);
 
 /* ---------------------------------------------------------------------
