@@ -33,3 +33,11 @@ def test_committed_profiles_name_every_kernel():
     for k in bench.KERNEL_SOURCES:
         path = os.path.join(root, "profiles", "%s_batched_gemm_fp16.md" % k)
         assert os.path.exists(path), path
+
+
+def test_committed_profiles_match_the_kernels_as_built():
+    """Every committed ncu summary was taken on its kernel's current code,
+    so the bench reports its traffic figure rather than null."""
+    for k in bench.KERNEL_SOURCES:
+        traffic, path = bench.kernel_traffic(k, "batched_gemm_fp16")
+        assert traffic is not None and traffic > 0, (k, path)
