@@ -10,11 +10,14 @@ GEMM input buffers, then one fp16 [32768, 32768] reference checked against
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
                        [--workload NAME] [--no-e2e] [--no-cpu] [--no-eq]
 
-Beside the step, the line carries `eq1`: Eq. 1 as a whole (the exact sums
-of the cosine term over the same reference and candidates), its kernel
-timed alone with CUDA events; `eq1_f64`: the same for binary64 outputs of
-the reference's size; and `restore`: the Tier 2 restore of the step's input
-regions from a captured snapshot, timed the same way.
+Beside the step, the line carries `snapshot_4096`: the 4096-region replay
+snapshot's fill and check, each kernel timed alone with CUDA events;
+`eq1`: Eq. 1 as a whole (the exact sums of the cosine term over the same
+reference and candidates); `eq1_f64`: the same for binary64 outputs of the
+reference's size; and `restore`: the Tier 2 restore of the step's input
+regions from a captured snapshot, timed the same way.  `--impl reference`
+times the CPU oracle alone on host-built samples of the same workload (no
+GPU library is loaded).
 For N > 1 launch under torchrun; every rank runs its own replica (weak
 scaling, no data-path collective) and rank 0 prints one JSON line.
 """
@@ -36,6 +39,9 @@ sys.path.insert(0, ROOT)
 METRIC = "verify GB/s (ref+cand bytes compared per s) and fill GB/s, % of GB300 HBM peak"
 UNIT = "GB/s"
 FALLBACK_HBM_GBS = 6800.0
+# bounded CPU samples: the cpu_baseline leg's check bytes, and one reference-arm step's
+CPU_SAMPLE_VERIFY_BYTES = 2 << 30
+REF_STEP_VERIFY_BYTES = 1 << 30
 
 
 # ------------------------------------------------------------------ helpers
@@ -120,7 +126,8 @@ def kernel_traffic(kernel, workload):
 
 
 # the source files each kernel is compiled from
-KERNEL_SOURCES = {"fill": ("fill.cu", "fill_math.cuh", "device.cuh", "ln_table.h", "plan.h"),
+KERNEL_SOURCES = {"fill": ("fill.cu", "fill_math.cuh", "fill_tables.h", "device.cuh", "ln_table.h",
+                           "plan.h"),
                   "compare": ("compare.cu", "device.cuh", "plan.h"),
                   "eqsum": ("eqsum.cu", "device.cuh", "plan.h"),
                   "copy": ("copy.cu", "device.cuh", "plan.h"),
@@ -145,40 +152,66 @@ def source_hash(kernel):
     return d.hexdigest()[:16]
 
 
-# Algorithmic operations of the fill per 16-byte chunk, counted from the
-# operation sequences the fill's specification states (include/asmv.h); one
-# op is one 32-bit integer or fp32 operation: a 32x32->64 product, a
-# three-input XOR, an IEEE add/mul/fma/sqrt, a conversion, a shift or mask.
-PHILOX_BLOCK_OPS = 40          # 10 rounds x (2 wide products + 2 three-input XORs)
-BOX_MULLER_PAIR_OPS = 54       # word prep 3, ln 20, rho 2, sincos 23, z 2, mean+std*z 4
-UNIFORM_ELEM_OPS = 5           # shift, int->float, scale, multiply, add
-INT_RANGE_ELEM_OPS = 2         # wide product, add
-# GB300: 152 SMs x 128 fp32/int32 lanes x 2070 MHz (maximum SM clock)
-ALU_PEAK_TOPS = 152 * 128 * 2.070e9 / 1e12
-
-
-def fill_ops_per_chunk(dtype, dist):
-    size = {"f32": 4, "bf16": 2, "f16": 2, "f8e4m3": 1, "i32": 4, "i8": 1, "u8": 1}[dtype]
-    elems = 16 // size
-    blocks = max(1, elems // 4) if dist != "raw" else 1
-    packs = elems // 2 if size < 4 else 0          # packed conversions to 16/8-bit
-    if dist == "raw":
-        return PHILOX_BLOCK_OPS
-    if dist == "none":
-        return 0
-    if dist == "int_range":
-        return blocks * PHILOX_BLOCK_OPS + elems * INT_RANGE_ELEM_OPS
-    if dist == "uniform":
-        return blocks * PHILOX_BLOCK_OPS + elems * UNIFORM_ELEM_OPS + packs
-    return blocks * PHILOX_BLOCK_OPS + (elems // 2) * BOX_MULLER_PAIR_OPS + packs
-
-
-def fill_algorithmic_ops(regions):
-    return sum(((r.payload_bytes + 15) // 16) * fill_ops_per_chunk(r.dtype, r.dist)
-               for r in regions)
-
-
 # ------------------------------------------------------------------ workload
+def fill_specs_of(wl):
+    """The regions a step fills: the input buffers, or the outputs themselves."""
+    return wl.input_regions if wl.input_regions else wl.regions
+
+
+def step_bytes(wl):
+    """(fill bytes, physical verify bytes, logical verify bytes) of one step:
+    the fill writes payload + guards; the check reads the reference once and
+    every candidate once, guards included (logical: reference per candidate)."""
+    fill = sum(r.alloc_bytes if r.dist != "none" else r.guard_lo + r.guard_hi
+               for r in fill_specs_of(wl))
+    payload = sum(r.payload_bytes for r in wl.regions)
+    guards = sum(r.guard_lo + r.guard_hi for r in wl.regions)
+    k = wl.n_cands
+    return fill, payload * (1 + k) + guards * (1 + k), 2 * payload * k
+
+
+def step_config(wl, world):
+    fill, vp, vl = step_bytes(wl)
+    return {"workload": wl.name, "description": wl.description, "fill_bytes": fill,
+            "verify_bytes_physical": vp, "verify_bytes_logical": vl, "candidates": wl.n_cands,
+            "l2": "inputs larger than L2 (129 MB); no flush",
+            "parallelism": "replica per GPU" if world > 1 else "1 GPU"}
+
+
+def make_candidates(wl, ref):
+    """The workload's candidate outputs: copies of the reference arena (a
+    torch uint8 tensor, on any device) perturbed by the workload's recipe."""
+    W = _workloads()
+    rng = np.random.default_rng(wl.seed + 77)
+    recipe = wl.name.split("_8kx16k")[0].split("_4kx16k")[0]   # size variants share the recipe
+    cands = []
+    for j in range(wl.n_cands):
+        c = ref.clone()
+        if recipe == "batched_gemm_fp16":
+            W.perturb_uniform_ulps(c, wl.regions[0], seed=wl.seed * 100 + j,
+                                   magnitude=wl.ulp_magnitudes[j])
+        elif recipe == "fp32_1m":
+            W.perturb_fp32_single(c, wl)
+        elif recipe == "attention_bf16":
+            for r in wl.regions:
+                W.perturb_ulp_noise(c, r, seed=wl.seed * 10 + r.region_id)
+        elif recipe == "int_exact":
+            for r in wl.regions:
+                W.flip_bit(c, r, rng)
+        elif recipe == "snapshot_4096":
+            for r in wl.regions:
+                W.perturb_sparse(c, r, rng, rate=1e-6)
+            for k in rng.choice(len(wl.regions), 3, replace=False):
+                W.corrupt_guard(c, wl.regions[int(k)], rng, "hi")
+        cands.append(c)
+    return cands
+
+
+def _workloads():
+    from paper_2608_20711_gb300 import workloads as W
+    return W
+
+
 class Setup:
     """Device buffers and region tables of one workload replica."""
 
@@ -205,37 +238,10 @@ class Setup:
             self.fill_regs = self.ref_regs
             self.fill_specs = wl.regions
         # candidates (input construction, outside the timed region)
-        rng = np.random.default_rng(wl.seed + 77)
-        self.cands = []
-        ncand = wl.n_cands
-        recipe = wl.name               # the recipe, shared by the size variants
-        for j in range(ncand):
-            c = self.ref.clone()
-            if recipe == "batched_gemm_fp16":
-                W.perturb_uniform_ulps(c, wl.regions[0], seed=wl.seed * 100 + j,
-                                       magnitude=wl.ulp_magnitudes[j])
-            elif recipe == "fp32_1m":
-                W.perturb_fp32_single(c, wl)
-            elif recipe == "attention_bf16":
-                for r in wl.regions:
-                    W.perturb_ulp_noise(c, r, seed=wl.seed * 10 + r.region_id)
-            elif recipe == "int_exact":
-                for r in wl.regions:
-                    W.flip_bit(c, r, rng)
-            elif recipe == "snapshot_4096":
-                for r in wl.regions:
-                    W.perturb_sparse(c, r, rng, rate=1e-6)
-                for k in rng.choice(len(wl.regions), 3, replace=False):
-                    W.corrupt_guard(c, wl.regions[int(k)], rng, "hi")
-            self.cands.append(c)
+        self.cands = make_candidates(wl, self.ref)
         self.cand_regs = [asmv.regions_in_arena(wl.regions, c.data_ptr()) for c in self.cands]
         torch.cuda.synchronize(dev)
-        self.fill_bytes = sum(r.alloc_bytes if r.dist != "none" else r.guard_lo + r.guard_hi
-                              for r in self.fill_specs)
-        ref_payload = sum(r.payload_bytes for r in wl.regions)
-        guards = sum(r.guard_lo + r.guard_hi for r in wl.regions)
-        self.verify_physical = ref_payload * (1 + ncand) + guards * (1 + ncand)
-        self.verify_logical = 2 * ref_payload * ncand
+        self.fill_bytes, self.verify_physical, self.verify_logical = step_bytes(wl)
         self.tol = wl.tol
 
     def step(self):
@@ -269,59 +275,92 @@ def _timed_until(budget_s, fn, n0, nmax):
     return n, total_t, total_w
 
 
-def cpu_oracle_sample(setup, budget_s=12.0, threads=None):
-    """The oracle as it stands, on the host cores (all of them unless
-    `threads` is given), over a bounded sample of the same workload: element
-    prefixes of the fill regions (one of each dtype/distribution kind) and
-    of the reference/candidate payloads.  The two measured rates are
-    combined over the step's byte mix."""
+class OracleSample:
+    """A bounded sample of one step of a workload, built and checked on the
+    host by the CPU oracle alone (no GPU library is loaded): every region of
+    the workload scaled down by the same factor (at least one element each),
+    the fill regions scaled so that the sample's fill and verify bytes keep
+    the full step's ratio.  The reference arena comes from the oracle's fill,
+    the candidates from the workload's recipe on host tensors; run() times the
+    oracle's fill of the fill sample plus its check of every candidate."""
+
+    def __init__(self, name, verify_bytes, threads):
+        import copy
+        import torch
+        from oracle import oracle as O
+        W = _workloads()
+        self.O = O
+        self.threads = int(threads)
+        wl = W.WORKLOADS[name]()
+        fill_full, verify_full, _ = step_bytes(wl)
+        f = min(1.0, verify_bytes / verify_full)
+        sample = copy.deepcopy(wl)
+        for r in sample.regions:
+            r.n_elems = max(1, int(r.n_elems * f))
+        sample.arena_bytes = W.layout(sample.regions)
+        if wl.input_regions:              # the same factor keeps the fill : verify ratio
+            for r in sample.input_regions:
+                r.n_elems = max(1, int(r.n_elems * f))
+            sample.input_arena_bytes = W.layout(sample.input_regions)
+        self.wl = sample
+        self.ref = torch.zeros(sample.arena_bytes, dtype=torch.uint8)
+        host = self.ref.numpy()
+        for r in sample.regions:
+            O.fill_region(host[r.offset:r.offset + r.alloc_bytes], r.n_elems, O.CODE_OF_DTYPE[r.dtype],
+                          O.CODE_OF_DIST[r.dist], r.guard_lo, r.guard_hi, r.region_id, r.canary,
+                          r.p0, r.p1, sample.seed, threads=self.threads)
+        self.cands = [c.numpy() for c in make_candidates(sample, self.ref)]
+        self.fill_specs = fill_specs_of(sample)
+        self.fill_arena = np.zeros(W.layout(self.fill_specs) + 256, np.uint8)
+        self.fill_bytes, self.verify_bytes, _ = step_bytes(sample)
+        self.kinds = len({(r.dtype, r.dist) for r in self.fill_specs})
+
+    def run(self):
+        """(seconds of fill, seconds of check, mismatches found)."""
+        O, wl, th = self.O, self.wl, self.threads
+        t0 = time.perf_counter()
+        for r in self.fill_specs:
+            O.fill_region(self.fill_arena[r.offset:r.offset + r.alloc_bytes], r.n_elems,
+                          O.CODE_OF_DTYPE[r.dtype], O.CODE_OF_DIST[r.dist], r.guard_lo, r.guard_hi,
+                          r.region_id, r.canary, r.p0, r.p1, wl.seed, threads=th)
+        t1 = time.perf_counter()
+        ref = self.ref.numpy()
+        mism = 0
+        for c in self.cands:
+            for r in wl.regions:
+                t = wl.tol.get(r.dtype, _workloads().Tolerance(0.0, 0.0))
+                a = ref[r.offset:r.offset + r.alloc_bytes]
+                b = c[r.offset:r.offset + r.alloc_bytes]
+                st = O.compare_region(a, r.guard_lo, r.guard_hi, r.canary, b, r.guard_lo, r.guard_hi,
+                                      r.canary, r.n_elems, O.CODE_OF_DTYPE[r.dtype], t.atol, t.rtol,
+                                      threads=th if r.n_elems >= (1 << 16) else 1)
+                mism += int(st["mismatches"])
+        t2 = time.perf_counter()
+        return t1 - t0, t2 - t1, mism
+
+    def describe(self, seconds):
+        return ("oracle on host-built inputs: fill of %.1f MB (%d region kinds) and check of "
+                "%.1f MB (reference + %d candidates, %d regions), %d threads, %.2f s"
+                % (self.fill_bytes / 1e6, self.kinds, self.verify_bytes / 1e6, len(self.cands),
+                   len(self.wl.regions), self.threads, seconds))
+
+
+def cpu_oracle_sample(name, verify_bytes, threads=None, repeats=1):
+    """The oracle as it stands on the host cores over a bounded sample of the
+    workload (OracleSample): rate = sample bytes / measured seconds."""
     from oracle import oracle as O
-    ORACLE_DTYPE, ORACLE_DIST = O.CODE_OF_DTYPE, O.CODE_OF_DIST
-    W = setup.W
     threads = O.host_threads() if threads is None else int(threads)
-    kinds = {}
-    for r in setup.fill_specs:
-        kinds.setdefault((r.dtype, r.dist), r)
-    cap_bytes = 256 << 20
-    bufs = {k: np.zeros(min(r.payload_bytes, cap_bytes), np.uint8) for k, r in kinds.items()}
-
-    def fill(n_bytes):
-        done = 0
-        for (dt, dist), r in kinds.items():
-            sz = W.DTYPE_SIZE[dt]
-            n = min(n_bytes // sz, bufs[(dt, dist)].size // sz)
-            O.fill_region(bufs[(dt, dist)], n, ORACLE_DTYPE[dt], ORACLE_DIST[dist], 0, 0,
-                          r.region_id, r.canary, r.p0, r.p1, setup.wl.seed, threads=threads)
-            done += n * sz
-        return done
-
-    _, t_fill, fill_done = _timed_until(budget_s / 2, fill, 1 << 16, cap_bytes)
-    # reference/candidate payload prefixes of the first region
-    r = setup.wl.regions[0]
-    nb = min(r.payload_bytes, cap_bytes // max(1, len(setup.cands)))
-    a = setup.ref[r.payload_offset:r.payload_offset + nb].cpu().numpy()
-    cs = [c[r.payload_offset:r.payload_offset + nb].cpu().numpy() for c in setup.cands]
-    t = setup.tol.get(r.dtype, W.Tolerance(0.0, 0.0))
-    sz = W.DTYPE_SIZE[r.dtype]
-
-    def compare(n_bytes):
-        n = min(n_bytes, nb) // sz
-        for c in cs:
-            O.compare_payload(a, c, ORACLE_DTYPE[r.dtype], n, t.atol, t.rtol, threads=threads)
-        return n * sz * (1 + len(cs))
-
-    _, t_cmp, cmp_done = _timed_until(budget_s / 2, compare, 1 << 16, nb)
-    fill_rate = fill_done / t_fill
-    cmp_rate = cmp_done / t_cmp
-    step_s = setup.fill_bytes / fill_rate + setup.verify_physical / cmp_rate
-    value = (setup.fill_bytes + setup.verify_physical) / step_s / 1e9
-    sample = ("oracle fill of %.1f MB over %d region kinds and compare of %.1f MB of "
-              "reference + %d candidate payload prefixes, %d threads; rates combined over the "
-              "step's fill/verify byte mix" % (fill_done / 1e6, len(kinds), cmp_done / 1e6,
-                                               len(cs), threads))
-    return {"value": round(value, 4), "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": sample, "fill_gbs": round(fill_rate / 1e9, 4),
-            "verify_gbs": round(cmp_rate / 1e9, 4), "seconds": round(t_fill + t_cmp, 2)}
+    smp = OracleSample(name, verify_bytes, threads)
+    tf = tc = 0.0
+    for _ in range(repeats):
+        a, b, _ = smp.run()
+        tf, tc = tf + a, tc + b
+    nb = (smp.fill_bytes + smp.verify_bytes) * repeats
+    return {"value": round(nb / (tf + tc) / 1e9, 4), "unit": UNIT, "cores": threads,
+            "kind": "oracle", "sample": smp.describe(tf + tc),
+            "fill_gbs": round(smp.fill_bytes * repeats / tf / 1e9, 4),
+            "verify_gbs": round(smp.verify_bytes * repeats / tc / 1e9, 4),
+            "seconds": round(tf + tc, 2)}
 
 
 # ------------------------------------------------------------------ runs
@@ -394,61 +433,42 @@ def run_mine(args):
     f_ms, c_ms = float(np.mean(fill_ms)), float(np.mean(cmp_ms))
     fill_gbs = setup.fill_bytes / (f_ms / 1e3) / 1e9
     verify_gbs = setup.verify_physical / (c_ms / 1e3) / 1e9
-    fill_ops = fill_algorithmic_ops(setup.fill_specs)
-    fill_alu_ms = fill_ops / (ALU_PEAK_TOPS * 1e12) * 1e3
-    fill_hbm_ms = setup.fill_bytes / (peak * 1e9) * 1e3
-    if c_ms >= f_ms:
-        traffic, _ = kernel_traffic("compare", args.workload)
-        achieved = setup.verify_physical / (c_ms / 1e3) / 1e9
-        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                    "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": "compare",
-                    "peak_kind": peak_kind + " (copy bandwidth, burst)",
-                    "algorithmic_bytes_per_launch": setup.verify_physical,
-                    "avg_launch_ms": round(c_ms, 4)}
-    else:
-        traffic, _ = kernel_traffic("fill", args.workload)
-        # the fill's roof is the ALU when its operations take longer than its bytes
-        if fill_alu_ms >= fill_hbm_ms:
-            achieved = fill_ops / (f_ms / 1e3) / 1e12
-            roofline = {"bound": "alu", "achieved": round(achieved, 3), "peak": round(ALU_PEAK_TOPS, 3),
-                        "unit": "Top/s", "frac": round(achieved / ALU_PEAK_TOPS, 4),
-                        "traffic": traffic, "kernel": "fill",
-                        "peak_kind": "derived: 152 SMs x 128 lanes x 2070 MHz",
-                        "algorithmic_ops_per_launch": fill_ops, "avg_launch_ms": round(f_ms, 4),
-                        "hbm_gbs": round(fill_gbs, 1), "hbm_frac": round(fill_gbs / peak, 4)}
-        else:
-            achieved = setup.fill_bytes / (f_ms / 1e3) / 1e9
-            roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                        "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": "fill",
-                        "peak_kind": peak_kind + " (copy bandwidth, burst)",
-                        "algorithmic_bytes_per_launch": setup.fill_bytes,
-                        "avg_launch_ms": round(f_ms, 4)}
+    # the roofline of the step's dominant kernel: HBM, algorithmic bytes per launch over the
+    # kernel's CUDA-event time, against the measured copy bandwidth
+    kern = "compare" if c_ms >= f_ms else "fill"
+    nbytes, ms = (setup.verify_physical, c_ms) if kern == "compare" else (setup.fill_bytes, f_ms)
+    achieved = nbytes / (ms / 1e3) / 1e9
+    traffic, _ = kernel_traffic(kern, args.workload)
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": traffic, "kernel": kern + "_kernel",
+                "peak_kind": peak_kind + " (copy bandwidth, burst)",
+                "algorithmic_bytes_per_launch": nbytes, "avg_launch_ms": round(ms, 4),
+                "other_kernel": {"kernel": ("fill" if kern == "compare" else "compare") + "_kernel",
+                                 "frac": round((fill_gbs if kern == "compare" else verify_gbs) / peak, 4)}}
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(elapsed / args.steps * 1e3, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "scaling": "weak", "vs_baseline": None, "dtype": dtype_label(setup.wl),
         "data": "synthetic (seeded Philox fill; seeded candidate perturbations)",
-        "config": {"workload": args.workload, "description": setup.wl.description,
-                   "fill_bytes": setup.fill_bytes, "verify_bytes_physical": setup.verify_physical,
-                   "verify_bytes_logical": setup.verify_logical, "candidates": len(setup.cands),
-                   "l2": "inputs larger than L2 (129 MB); no flush",
-                   "parallelism": "replica per GPU" if world > 1 else "1 GPU"},
+        "config": step_config(setup.wl, world),
         "fill_gbs": round(fill_gbs, 1), "verify_gbs": round(verify_gbs, 1),
         "fill_frac": round(fill_gbs / peak, 4), "verify_frac": round(verify_gbs / peak, 4),
         "clocks": clk.summary(), "gpu_launches": launches, "roofline": roofline,
         "e2e": e2e,
     }
+    if args.snapshot and args.workload != "snapshot_4096":
+        line["snapshot_4096"] = run_snapshot(args, device, peak)
     if args.eq:
         line["eq1"] = run_eq1(setup, args, peak)
         line["eq1_f64"] = run_eq1_f64(setup, args, peak)
     if args.restore:
         line["restore"] = run_restore(setup, args, peak)
     if rank == 0 and world == 1 and args.cpu:
-        line["cpu_baseline"] = cpu_oracle_sample(setup)
-        one = cpu_oracle_sample(setup, budget_s=4.0, threads=1)
+        line["cpu_baseline"] = cpu_oracle_sample(args.workload, CPU_SAMPLE_VERIFY_BYTES)
+        one = cpu_oracle_sample(args.workload, CPU_SAMPLE_VERIFY_BYTES // 16, threads=1)
         line["cpu_baseline"]["single_thread"] = {k: one[k] for k in ("value", "fill_gbs", "verify_gbs",
-                                                                      "seconds")}
+                                                                      "seconds", "sample")}
     if rank == 0:
         mism = sum(int(s["mismatches"]) for cs in stats for s in cs)
         line["check"] = {"total_mismatches": mism}
@@ -456,6 +476,48 @@ def run_mine(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def dtype_label(wl):
+    """What the path computes: the stored formats of the payloads it fills
+    and checks, and the exact fp64 statistics."""
+    fmts = sorted({r.dtype for r in fill_specs_of(wl)} | {r.dtype for r in wl.regions})
+    return "/".join(fmts) + " payloads; statistics exact in fp64"
+
+
+def run_snapshot(args, device, peak):
+    """The 4096-region replay snapshot: its fill and its check of one
+    candidate, each kernel timed alone with CUDA events around its launches
+    (the same protocol as the step's kernels)."""
+    import torch
+    snap = Setup("snapshot_4096", device)
+    ctx = snap.ctx
+    ctx.fill(snap.fill_regs, seed=snap.wl.seed)
+    ctx.compare(snap.ref_regs, snap.cand_regs[0], snap.tol)
+    ctx.set_timing(True)
+    fill_ms, cmp_ms = [], []
+    for _ in range(max(5, args.steps)):
+        ctx.fill(snap.fill_regs, seed=snap.wl.seed)
+        fill_ms.append(ctx.kernel_ms())
+        st = ctx.compare(snap.ref_regs, snap.cand_regs[0], snap.tol)
+        cmp_ms.append(ctx.kernel_ms())
+    ctx.set_timing(False)
+    f_ms, c_ms = float(np.mean(fill_ms)), float(np.mean(cmp_ms))
+    fill_gbs = snap.fill_bytes / (f_ms / 1e3) / 1e9
+    verify_gbs = snap.verify_physical / (c_ms / 1e3) / 1e9
+    out = {"regions": len(snap.wl.regions), "fill_bytes": snap.fill_bytes,
+           "verify_bytes_physical": snap.verify_physical,
+           "fill_avg_launch_ms": round(f_ms, 4), "verify_avg_launch_ms": round(c_ms, 4),
+           "fill_gbs": round(fill_gbs, 1), "verify_gbs": round(verify_gbs, 1),
+           "fill_frac": round(fill_gbs / peak, 4), "verify_frac": round(verify_gbs / peak, 4),
+           "fill_traffic": kernel_traffic("fill", "snapshot_4096")[0],
+           "verify_traffic": kernel_traffic("compare", "snapshot_4096")[0],
+           "mismatches": int(sum(s["mismatches"] for s in st)),
+           "bad_guard_bytes": int(sum(s["guard_bad_bytes"] for s in st))}
+    ctx.close()
+    del snap
+    torch.cuda.empty_cache()
+    return out
 
 
 def run_eq1(setup, args, peak):
@@ -607,32 +669,36 @@ def run_e2e(setup, args, device, world, barrier):
 
 
 def run_reference(args):
-    """The oracle (plain CPU program) on the same workload: each step is a
-    bounded sample, extrapolated to the step's byte mix."""
-    world, rank, local = dist_env()
+    """The oracle (the plain CPU program) on the same workload, metric and
+    config: every step is one OracleSample of the workload run on the host
+    cores, with inputs the oracle built on the host (no GPU library is
+    loaded); value = sample bytes / measured seconds."""
+    world, rank, _ = dist_env()
     if rank != 0:
         return
-    import torch
-    device = torch.device("cuda", local)
-    torch.cuda.set_device(device)
-    setup = Setup(args.workload, device)
+    from oracle import oracle as O
+    W = _workloads()
+    wl = W.WORKLOADS[args.workload]()
+    threads = O.host_threads()
+    smp = OracleSample(args.workload, REF_STEP_VERIFY_BYTES, threads)
     for _ in range(args.warmup):
-        pass
-    vals, secs = [], []
+        smp.run()
+    secs = []
     for _ in range(args.steps):
-        r = cpu_oracle_sample(setup, budget_s=max(2.0, 60.0 / max(1, args.steps)))
-        vals.append(r["value"])
-        secs.append(r["seconds"])
-    step_bytes = setup.fill_bytes + setup.verify_physical
-    value = float(np.median(vals))
-    line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
-            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(step_bytes / (value * 1e9) * 1e3, 3), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": args.workload},
-            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": r["cores"],
-                             "kind": "oracle", "sample": r["sample"]},
-            "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+        tf, tc, _ = smp.run()
+        secs.append(tf + tc)
+    total = float(np.sum(secs))
+    nb = (smp.fill_bytes + smp.verify_bytes) * args.steps
+    value = nb / total / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": dtype_label(wl),
+            "data": "synthetic (the oracle's seeded fill and the workload's candidate recipe, on the host)",
+            "config": step_config(wl, world),
+            "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": threads,
+                             "kind": "oracle", "sample": smp.describe(total / args.steps) + " per step"},
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -648,13 +714,16 @@ def main():
     ap.add_argument("--no-cpu", dest="cpu", action="store_false")
     ap.add_argument("--no-eq", dest="eq", action="store_false")
     ap.add_argument("--no-restore", dest="restore", action="store_false")
+    ap.add_argument("--no-snapshot", dest="snapshot", action="store_false")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
-    import __graft_entry__
-    __graft_entry__.build()
     if args.impl == "reference":
+        from oracle import build as oracle_build      # the oracle only: no GPU library
+        oracle_build.build()
         run_reference(args)
     else:
+        import __graft_entry__
+        __graft_entry__.build()
         run_mine(args)
 
 

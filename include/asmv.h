@@ -72,19 +72,39 @@ typedef enum {
  *   RAW       payload byte j is byte (j mod 16) of block (j div 16); the
  *             block's four 32-bit words in order, each little-endian.
  *             Any dtype.
- *   UNIFORM   float dtypes: word w = word (i mod 4) of block (i div 4),
- *             f = (w >> 8) * 2^-24, v = p0 + f*(p1 - p0) in fp32 (p0, p1 and
- *             p1 - p0 rounded to fp32 first; multiply then add), then
- *             round-to-nearest-even to the dtype (every fp8 format saturates
- *             at its largest finite value; fnuz formats give +0 for a zero
- *             result; binary64 is the exact widening of the fp32 value).
- *   NORMAL    float dtypes: Box-Muller on words (0,1) and (2,3) of block
- *             (i div 4): u1 = ((w0 >> 8) + 1) 2^-24, u2 = (w1 >> 8) 2^-24,
- *             z0 = sqrt(-2 ln u1) cos(2 pi u2), z1 = ... sin(2 pi u2);
+ *   UNIFORM   float dtypes: a fraction f, v = p0 + f*(p1 - p0) in fp32
+ *             (p0, p1 and p1 - p0 rounded to fp32 first; multiply then add),
+ *             then round-to-nearest-even to the dtype (every fp8 format
+ *             saturates at its largest finite value; fnuz formats give +0 for
+ *             a zero result; binary64 is the exact widening of the fp32
+ *             value).  fp32 and binary64: w = word (i mod 4) of block
+ *             (i div 4), f = (w >> 8) * 2^-24.  16-bit formats: h = half
+ *             (i mod 2) (low half first) of word (i mod 8) div 2 of block
+ *             (i div 8), f = h * 2^-16.  8-bit formats: b = byte (i mod 4) of
+ *             word (i mod 16) div 4 of block (i div 16), f = b * 2^-8.
+ *   NORMAL    fp32 and binary64: Box-Muller on words (0,1) and (2,3) of
+ *             block (i div 4): u1 = ((w0 >> 8) + 1) 2^-24, u2 = (w1 >> 8)
+ *             2^-24, z0 = sqrt(-2 ln u1) cos(2 pi u2), z1 = ... sin(2 pi u2);
  *             element 4b+2p+t is z_t of pair p; v = p0 + p1*z in fp32, then
  *             RNE to the dtype.  ln and sincos are fixed fp32 series
  *             evaluations, so results are bit-reproducible.
- *   INT_RANGE integer dtypes: w as for UNIFORM, v = lo + ((w*(hi-lo)) >> 32)
+ *             16-bit formats: element i is v_(i mod 2) of the pair drawn from
+ *             word (i mod 8) div 2 of block (i div 8): radius from the low
+ *             half k, u = (k + 1/2) 2^-16, rho = sqrt(-2 ln u) as a chord over
+ *             one of 512 cells (within 2^-13); angle from the high half a,
+ *             theta = 2 pi (a + 1/2) / 65536, as a table angle
+ *             2 pi (j + 1/2) / 256 (j = a div 256) turned to first order;
+ *             v0 = p1 rho cos theta + p0, v1 = p1 rho sin theta + p0 (one fma
+ *             each after rs = rho p1).  8-bit formats: element i is
+ *             v_(i mod 2) of the pair drawn from half (i mod 4) div 2 of word
+ *             (i mod 16) div 4 of block (i div 16): radius index = its low
+ *             byte k, rho = sqrt(-2 ln((k + 1/2) / 256)); angle index = its
+ *             high byte j, theta = 2 pi (j + 1/2) / 256.  Every constant is
+ *             the correctly rounded fp32 value of its closed form and every
+ *             step one IEEE fp32 operation in a fixed order, so the bytes are
+ *             reproducible on any IEEE machine.
+ *   INT_RANGE integer dtypes: w = word (i mod 4) of block (i div 4),
+ *             v = lo + ((w*(hi-lo)) >> 32)
  *             with lo = p0, hi = p1 (integers; 1 <= hi - lo <= 2^32 and
  *             [lo, hi) inside the dtype's range; for int64 |p0|, |p1| <= 2^53).
  *   NONE      the payload is left untouched; only guard bands are written. */

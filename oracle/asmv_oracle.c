@@ -49,6 +49,14 @@
  *      the fp32 value.  For binary64, d = RN64(|c - r|) is one rounded
  *      subtraction.  For int64, |c - r| is formed exactly and rounded once
  *      to fp64, and rel = RN64(that / RN64(|r|)).
+ *   R12 The 16-bit and 8-bit float formats draw as many Philox bits per
+ *      element as they store: one Philox block per 16-byte chunk of payload.
+ *      UNIFORM takes a 16-bit (8-bit) fraction per element.  NORMAL is
+ *      Box-Muller on one pair per 32 bits (16-bit formats: a 16-bit radius
+ *      index and a 16-bit angle index) or per 16 bits (8-bit formats: 8 + 8),
+ *      with radius and angle taken from tables whose entries are the
+ *      correctly rounded fp32 values of their closed forms (see "narrow
+ *      formats" below).  fp32 and binary64 keep R3.
  *
  * Parity pins live in tests/test_oracle_*.py.  The stats of the large
  * perturbed workloads (attention outputs, the 4096-region snapshot, the
@@ -312,7 +320,10 @@ uint8_t oracle_f32_to_f8e4m3(float f) {
  * fp32 Box-Muller pieces.  Every step below is one IEEE fp32 operation
  * (fmaf where written).
  *
- * ln(u), u = k 2^-24: u = m 2^e with m in [1, 2) and j = round(128 (m-1));
+ * ln(u), u = k 2^-24, is P. T. P. Tang's table-driven logarithm ("Table-
+ * driven implementation of the logarithm function in IEEE floating-point
+ * arithmetic", ACM TOMS 16, 1990) with this library's table and series:
+ * u = m 2^e with m in [1, 2) and j = round(128 (m-1));
  * with inv_j = round(32768/(128+j))/256 (eight significant bits) the
  * reduction r = m*inv_j - 1 is exact in one fma and |r| < 2^-7; then
  *   ln u = e ln2 + (-ln inv_j) + log1p(r),
@@ -428,15 +439,135 @@ void oracle_boxmuller(uint32_t w0, uint32_t w1, float *z0, float *z1) {
 }
 
 /* ======================================================================
+ * Narrow formats (reading R12): Box-Muller for the 16-bit and 8-bit floats.
+ *
+ * 16-bit formats, one pair per 32-bit word w:
+ *   radius  k = w mod 2^16, u = (k + 1/2) 2^-16.  With d = 1 when u > 1/2,
+ *           x = u (d = 0) or x = 1 - u (d = 1) is K 2^-17 for the odd
+ *           K = 2t + 1, t = (k mod 2^15) xor (d ? 2^15 - 1 : 0).  The fp32
+ *           value F = K 2^(16 d) is exact; write F = 2^E m with m in [1, 2)
+ *           and take cell c = 16 E + floor(16 (m - 1)), 0 <= c < 512.  Then
+ *             rho = fma(F, A_c, B_c)
+ *           where, for the cell's mantissa interval [m0, m0 + 1/16) and
+ *           g(m) = sqrt(-2 ln y(m)), y(m) = m 2^(e-17) (d = 0) or
+ *           1 - m 2^(e-17) (d = 1), e = E - 16 d, the secant slope is
+ *           S = 16 (g(m0 + 1/16) - g(m0)), A_c = RN32(S 2^-E) and
+ *           B_c = RN32(g(m0) - S m0): the chord of rho over the cell.
+ *   angle   a = w div 2^16, theta = 2 pi (a + 1/2) / 65536.  With
+ *           j = a div 256, n = a mod 256, phi_j = 2 pi (j + 1/2) / 256 and
+ *           (S_j, C_j) = (RN32(sin phi_j), RN32(cos phi_j)):
+ *             delta = fma(n - 128, c16, c16 / 2),  c16 = RN32(2 pi / 65536)
+ *             sin ~ fma(C_j, delta, S_j),  cos ~ fma(-S_j, delta, C_j)
+ *           (the first-order rotation of phi_j by delta = theta - phi_j).
+ *   values  rs = RN32(rho * std); v0 = fma(rs, cos, mean),
+ *           v1 = fma(rs, sin, mean).
+ * 8-bit formats, one pair per 16-bit half h of a word (low half first):
+ *   rho = R8[h mod 256] = RN32(sqrt(-2 ln((k + 1/2) / 256))) and the angle
+ *   table entry j = h div 256 itself, (sin, cos) = (S_j, C_j); the values
+ *   as above.
+ * ====================================================================== */
+static float N16_A[512], N16_B[512], T_SIN[256], T_COS[256], R8_RHO[256];
+static float C16_STEP;
+static int narrow_ready = 0;
+
+static long double nr_g(long double m, int e, int d) {
+  long double y = ldexpl(m, e - 17);
+  if (d) y = 1.0L - y;
+  return sqrtl(-2.0L * logl(y));
+}
+
+static void init_narrow(void) {
+  if (narrow_ready) return;
+  long double pi = acosl(-1.0L);
+  for (int E = 0; E < 32; ++E) {
+    int d = E >= 16, e = E - 16 * d;
+    for (int i = 0; i < 16; ++i) {
+      long double m0 = 1.0L + i / 16.0L, m1 = m0 + 1.0L / 16.0L;
+      long double g0 = nr_g(m0, e, d), g1 = nr_g(m1, e, d);
+      long double S = 16.0L * (g1 - g0);
+      N16_A[16 * E + i] = (float)ldexpl(S, -E);
+      N16_B[16 * E + i] = (float)(g0 - S * m0);
+    }
+  }
+  for (int j = 0; j < 256; ++j) {
+    long double phi = 2.0L * pi * (j + 0.5L) / 256.0L;
+    T_SIN[j] = (float)sinl(phi);
+    T_COS[j] = (float)cosl(phi);
+    R8_RHO[j] = (float)sqrtl(-2.0L * logl((j + 0.5L) / 256.0L));
+  }
+  C16_STEP = (float)(2.0L * pi / 65536.0L);
+  narrow_ready = 1;
+}
+
+/* out: A[512], B[512], sin[256], cos[256], R8[256], c16 */
+void oracle_narrow_tables(float *out) {
+  init_narrow();
+  for (int c = 0; c < 512; ++c) { out[c] = N16_A[c]; out[512 + c] = N16_B[c]; }
+  for (int j = 0; j < 256; ++j) {
+    out[1024 + j] = T_SIN[j]; out[1280 + j] = T_COS[j]; out[1536 + j] = R8_RHO[j];
+  }
+  out[1792] = C16_STEP;
+}
+
+/* The radius of a 16-bit pair, k in [0, 2^16). */
+float oracle_radius16(uint32_t k) {
+  init_narrow();
+  uint32_t d = (k >> 15) & 1u;
+  uint32_t t = (k & 0x7FFFu) ^ (d ? 0x7FFFu : 0u);
+  float F = (float)(2u * t + 1u) * (d ? 65536.0f : 1.0f);     /* exact */
+  uint32_t b = f32_bits(F);
+  int E = (int)(b >> 23) - 127;
+  int c = 16 * E + (int)((b >> 19) & 15u);
+  return fmaf(F, N16_A[c], N16_B[c]);
+}
+
+/* sin and cos of the angle of a 16-bit pair, a in [0, 2^16). */
+void oracle_angle16(uint32_t a, float *sn, float *cs) {
+  init_narrow();
+  uint32_t j = a >> 8, n = a & 255u;
+  float delta = fmaf((float)n - 128.0f, C16_STEP, C16_STEP * 0.5f);
+  *sn = fmaf(T_COS[j], delta, T_SIN[j]);
+  *cs = fmaf(-T_SIN[j], delta, T_COS[j]);
+}
+
+/* v0, v1 of the pair drawn from word w (16-bit formats). */
+void oracle_normal16(uint32_t w, float mean, float sd, float *v0, float *v1) {
+  float rho = oracle_radius16(w & 0xFFFFu);
+  float sn, cs;
+  oracle_angle16(w >> 16, &sn, &cs);
+  float rs = rho * sd;
+  *v0 = fmaf(rs, cs, mean);
+  *v1 = fmaf(rs, sn, mean);
+}
+
+/* v0, v1 of the pair drawn from the 16-bit half h (8-bit formats). */
+void oracle_normal8(uint32_t h, float mean, float sd, float *v0, float *v1) {
+  init_narrow();
+  float rho = R8_RHO[h & 255u];
+  uint32_t j = (h >> 8) & 255u;
+  float rs = rho * sd;
+  *v0 = fmaf(rs, T_COS[j], mean);
+  *v1 = fmaf(rs, T_SIN[j], mean);
+}
+
+/* ======================================================================
  * Tier 1 fill.
  * Element i of a payload, per distribution:
  *   RAW       payload byte j = byte (j mod 16) of block (j div 16); a block
  *             is its four words in order, each little-endian.
  *   INT_RANGE word (i mod 4) of block (i div 4): lo + ((w * (hi-lo)) >> 32)
- *   UNIFORM   word (i mod 4) of block (i div 4): f = (w >> 8) 2^-24,
- *             v = lo + f*(hi - lo) in fp32, then RNE to the dtype
- *   NORMAL    block i div 4 gives two pairs (words 0,1 and 2,3); element
- *             4b+2j+t is z_t of pair j, v = mean + std*z in fp32, then RNE
+ *   UNIFORM   fp32 / binary64: word (i mod 4) of block (i div 4),
+ *             f = (w >> 8) 2^-24; 16-bit formats: half (i mod 2) of word
+ *             (i mod 8) div 2 of block (i div 8), f = h 2^-16; 8-bit formats:
+ *             byte (i mod 4) of word (i mod 16) div 4 of block (i div 16),
+ *             f = b 2^-8.  v = lo + f*(hi - lo) in fp32, then RNE
+ *   NORMAL    fp32 / binary64: block i div 4 gives two pairs (words 0,1 and
+ *             2,3); element 4b+2j+t is z_t of pair j, v = mean + std*z in
+ *             fp32, then RNE.  16-bit formats: element i is v_(i mod 2) of
+ *             the pair of word (i mod 8) div 2 of block (i div 8); 8-bit
+ *             formats: v_(i mod 2) of the pair of half (i mod 4) div 2 of
+ *             word (i mod 16) div 4 of block (i div 16) (narrow formats
+ *             above)
  *   NONE      payload untouched
  * ====================================================================== */
 static void store_float(uint8_t *p, int dt, uint64_t i, float v) {
@@ -496,10 +627,42 @@ int oracle_fill_payload(uint8_t *payload, int dt, int dist, uint64_t i0,
     float width = hi - lo;
     for (uint64_t i = i0; i < i1; ++i) {
       uint32_t w[4];
-      payload_block(seed, region_id, i / 4, w);
-      float f = (float)(w[i % 4] >> 8) * 0x1p-24f;
+      float f;
+      if (sz == 2) {
+        payload_block(seed, region_id, i / 8, w);
+        f = (float)((w[(i % 8) / 2] >> (16 * (i % 2))) & 0xFFFFu) * 0x1p-16f;
+      } else if (sz == 1) {
+        payload_block(seed, region_id, i / 16, w);
+        f = (float)((w[(i % 16) / 4] >> (8 * (i % 4))) & 0xFFu) * 0x1p-8f;
+      } else {
+        payload_block(seed, region_id, i / 4, w);
+        f = (float)(w[i % 4] >> 8) * 0x1p-24f;
+      }
       float v = lo + f * width;
       store_float(payload, dt, i, v);
+    }
+    return 0;
+  }
+  if (dist == OX_NORMAL && sz == 2) {
+    float mean = (float)p0, sd = (float)p1;
+    for (uint64_t i = i0; i < i1; ++i) {
+      uint32_t w[4];
+      payload_block(seed, region_id, i / 8, w);
+      float v0, v1;
+      oracle_normal16(w[(i % 8) / 2], mean, sd, &v0, &v1);
+      store_float(payload, dt, i, (i % 2 == 0) ? v0 : v1);
+    }
+    return 0;
+  }
+  if (dist == OX_NORMAL && sz == 1) {
+    float mean = (float)p0, sd = (float)p1;
+    for (uint64_t i = i0; i < i1; ++i) {
+      uint32_t w[4];
+      payload_block(seed, region_id, i / 16, w);
+      uint32_t h = (w[(i % 16) / 4] >> (16 * ((i % 4) / 2))) & 0xFFFFu;
+      float v0, v1;
+      oracle_normal8(h, mean, sd, &v0, &v1);
+      store_float(payload, dt, i, (i % 2 == 0) ? v0 : v1);
     }
     return 0;
   }
@@ -841,6 +1004,24 @@ void oracle_sincos_2pi_u24_many(const uint32_t *k, uint64_t n, float *sn,
 void oracle_boxmuller_many(const uint32_t *w0, const uint32_t *w1, uint64_t n,
                            float *z0, float *z1) {
   for (uint64_t i = 0; i < n; ++i) oracle_boxmuller(w0[i], w1[i], z0 + i, z1 + i);
+}
+
+void oracle_radius16_many(const uint32_t *k, uint64_t n, float *out) {
+  for (uint64_t i = 0; i < n; ++i) out[i] = oracle_radius16(k[i]);
+}
+
+void oracle_angle16_many(const uint32_t *a, uint64_t n, float *sn, float *cs) {
+  for (uint64_t i = 0; i < n; ++i) oracle_angle16(a[i], &sn[i], &cs[i]);
+}
+
+void oracle_normal16_many(const uint32_t *w, uint64_t n, float mean, float sd, float *v0,
+                          float *v1) {
+  for (uint64_t i = 0; i < n; ++i) oracle_normal16(w[i], mean, sd, &v0[i], &v1[i]);
+}
+
+void oracle_normal8_many(const uint32_t *h, uint64_t n, float mean, float sd, float *v0,
+                         float *v1) {
+  for (uint64_t i = 0; i < n; ++i) oracle_normal8(h[i], mean, sd, &v0[i], &v1[i]);
 }
 
 void oracle_encode_many(const float *x, uint64_t n, int dt, uint8_t *out) {

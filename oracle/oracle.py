@@ -89,40 +89,43 @@ class use_library:
 
 
 def _load(path):
-    if True:
-        if True:
-            L = ctypes.CDLL(path)
-            c = ctypes
-            L.oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
-            L.oracle_philox_many.argtypes = [_u32p, _u32p, c.c_uint64, _u32p]
-            L.oracle_ln_u24_many.argtypes = [_u32p, c.c_uint64, _f32p]
-            L.oracle_sincos_2pi_u24_many.argtypes = [_u32p, c.c_uint64, _f32p, _f32p]
-            L.oracle_boxmuller_many.argtypes = [_u32p, _u32p, c.c_uint64, _f32p, _f32p]
-            L.oracle_boxmuller_consts.argtypes = [_f32p]
-            L.oracle_ln_table.argtypes = [_f32p]
-            L.oracle_encode_many.argtypes = [_f32p, c.c_uint64, c.c_int, _u8p]
-            L.oracle_decode_many.argtypes = [_u8p, c.c_uint64, c.c_int, _f64p]
-            L.oracle_fill_payload.argtypes = [_u8p, c.c_int, c.c_int, c.c_uint64,
-                                              c.c_uint64, c.c_uint32, c.c_double,
-                                              c.c_double, c.c_uint64]
-            L.oracle_fill_payload.restype = c.c_int
-            L.oracle_fill_guards.argtypes = [_u8p, c.c_uint64, c.c_uint32,
-                                             c.c_uint32, c.c_uint8]
-            L.oracle_guard_check.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
-                                             c.c_uint8, _u64p, _u64p]
-            L.oracle_compare_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
-                                               c.c_uint64, c.c_double, c.c_double,
-                                               c.POINTER(_Stats)]
-            L.oracle_compare_region.argtypes = [
-                _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
-                _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
-                c.c_uint64, c.c_int, c.c_double, c.c_double,
-                c.POINTER(_RegionStats)]
-            L.oracle_eq_sums_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
-                                               c.c_uint64, _i64p]
-            L.oracle_eq64_sums_range.argtypes = [_u8p, _u8p, c.c_uint64, c.c_uint64, _i64p]
-            L.oracle_restore_region.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
-                                                c.c_uint8, _u8p]
+    L = ctypes.CDLL(path)
+    c = ctypes
+    L.oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
+    L.oracle_philox_many.argtypes = [_u32p, _u32p, c.c_uint64, _u32p]
+    L.oracle_ln_u24_many.argtypes = [_u32p, c.c_uint64, _f32p]
+    L.oracle_sincos_2pi_u24_many.argtypes = [_u32p, c.c_uint64, _f32p, _f32p]
+    L.oracle_boxmuller_many.argtypes = [_u32p, _u32p, c.c_uint64, _f32p, _f32p]
+    L.oracle_boxmuller_consts.argtypes = [_f32p]
+    L.oracle_ln_table.argtypes = [_f32p]
+    L.oracle_narrow_tables.argtypes = [_f32p]
+    L.oracle_radius16_many.argtypes = [_u32p, c.c_uint64, _f32p]
+    L.oracle_angle16_many.argtypes = [_u32p, c.c_uint64, _f32p, _f32p]
+    L.oracle_normal16_many.argtypes = [_u32p, c.c_uint64, c.c_float, c.c_float, _f32p, _f32p]
+    L.oracle_normal8_many.argtypes = [_u32p, c.c_uint64, c.c_float, c.c_float, _f32p, _f32p]
+    L.oracle_encode_many.argtypes = [_f32p, c.c_uint64, c.c_int, _u8p]
+    L.oracle_decode_many.argtypes = [_u8p, c.c_uint64, c.c_int, _f64p]
+    L.oracle_fill_payload.argtypes = [_u8p, c.c_int, c.c_int, c.c_uint64,
+                                      c.c_uint64, c.c_uint32, c.c_double,
+                                      c.c_double, c.c_uint64]
+    L.oracle_fill_payload.restype = c.c_int
+    L.oracle_fill_guards.argtypes = [_u8p, c.c_uint64, c.c_uint32,
+                                     c.c_uint32, c.c_uint8]
+    L.oracle_guard_check.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
+                                     c.c_uint8, _u64p, _u64p]
+    L.oracle_compare_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
+                                       c.c_uint64, c.c_double, c.c_double,
+                                       c.POINTER(_Stats)]
+    L.oracle_compare_region.argtypes = [
+        _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
+        _u8p, c.c_uint32, c.c_uint32, c.c_uint8,
+        c.c_uint64, c.c_int, c.c_double, c.c_double,
+        c.POINTER(_RegionStats)]
+    L.oracle_eq_sums_range.argtypes = [_u8p, _u8p, c.c_int, c.c_uint64,
+                                       c.c_uint64, _i64p]
+    L.oracle_eq64_sums_range.argtypes = [_u8p, _u8p, c.c_uint64, c.c_uint64, _i64p]
+    L.oracle_restore_region.argtypes = [_u8p, c.c_uint64, c.c_uint32, c.c_uint32,
+                                        c.c_uint8, _u8p]
     return L
 
 
@@ -186,6 +189,53 @@ def ln_table():
     out = np.empty(129 * 3, np.float32)
     lib().oracle_ln_table(_ptr(out, _f32p))
     return out.reshape(129, 3)
+
+
+def narrow_tables():
+    """The tables of the 16-bit and 8-bit NORMAL fill: A (512), B (512) of
+    the radius chords, sin and cos (256 each) of the angles 2 pi (j + 1/2)
+    / 256, the 8-bit radii (256) and the angle step RN32(2 pi / 65536)."""
+    out = np.empty(1793, np.float32)
+    lib().oracle_narrow_tables(_ptr(out, _f32p))
+    return {"A": out[:512].copy(), "B": out[512:1024].copy(), "sin": out[1024:1280].copy(),
+            "cos": out[1280:1536].copy(), "r8": out[1536:1792].copy(), "c16": out[1792]}
+
+
+def radius16(k):
+    k = np.ascontiguousarray(k, dtype=np.uint32)
+    out = np.empty(k.shape, np.float32)
+    lib().oracle_radius16_many(_ptr(k, _u32p), k.size, _ptr(out, _f32p))
+    return out
+
+
+def angle16(a):
+    """(sin, cos) of the angle 2 pi (a + 1/2) / 65536 as the 16-bit fill
+    forms it."""
+    a = np.ascontiguousarray(a, dtype=np.uint32)
+    sn = np.empty(a.shape, np.float32)
+    cs = np.empty(a.shape, np.float32)
+    lib().oracle_angle16_many(_ptr(a, _u32p), a.size, _ptr(sn, _f32p), _ptr(cs, _f32p))
+    return sn, cs
+
+
+def normal16(w, mean=0.0, sd=1.0):
+    """The pair (v0, v1) the 16-bit NORMAL fill draws from 32-bit words w."""
+    w = np.ascontiguousarray(w, dtype=np.uint32)
+    v0 = np.empty(w.shape, np.float32)
+    v1 = np.empty(w.shape, np.float32)
+    lib().oracle_normal16_many(_ptr(w, _u32p), w.size, float(mean), float(sd),
+                               _ptr(v0, _f32p), _ptr(v1, _f32p))
+    return v0, v1
+
+
+def normal8(h, mean=0.0, sd=1.0):
+    """The pair (v0, v1) the 8-bit NORMAL fill draws from 16-bit halves h."""
+    h = np.ascontiguousarray(h, dtype=np.uint32)
+    v0 = np.empty(h.shape, np.float32)
+    v1 = np.empty(h.shape, np.float32)
+    lib().oracle_normal8_many(_ptr(h, _u32p), h.size, float(mean), float(sd),
+                              _ptr(v0, _f32p), _ptr(v1, _f32p))
+    return v0, v1
 
 
 def encode(x, dtype):

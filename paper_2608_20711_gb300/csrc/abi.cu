@@ -206,7 +206,7 @@ struct DeviceScope {
 struct asmv_ctx {
   int device = 0;
   int sms = 0;
-  int fill_ctas = 1;
+  int fill_ctas[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // per set of fill tables (kNeed* mask)
   int eq_ctas = 1;
   int eq64_ctas = 1;
   int copy_ctas = 1;
@@ -499,7 +499,14 @@ int asmv_ctx_create(asmv_ctx **out, int device) {
     asmv_ctx_destroy(ctx);
     return ASMV_ECUDA;
   }
-  ctx->fill_ctas = fill_max_ctas_per_sm();
+  for (uint32_t m = 0; m < 8 && e == cudaSuccess; ++m) {
+    ctx->fill_ctas[m] = fill_max_ctas_per_sm(fill_layout(m).bytes);
+    if (ctx->fill_ctas[m] <= 0) e = cudaErrorInvalidConfiguration;
+  }
+  if (e != cudaSuccess) {
+    asmv_ctx_destroy(ctx);
+    return ASMV_ECUDA;
+  }
   ctx->eq_ctas = eq_max_ctas_per_sm();
   ctx->eq64_ctas = eq64_max_ctas_per_sm();
   ctx->copy_ctas = copy_max_ctas_per_sm();
@@ -566,6 +573,7 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   std::vector<FillRegion> fr(n + 1);
   std::vector<GuardSeg> segs;
   uint64_t tile = 0;
+  uint32_t needs = 0;   // the shared-memory tables the launch's NORMAL regions use
   for (size_t i = 0; i < n; ++i) {
     const asmv_region &r = regions[i];
     uint64_t pb, tot;
@@ -589,7 +597,11 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
       f.ilo = (int64_t)r.p0;
       f.ispan = (uint64_t)((int64_t)r.p1 - (int64_t)r.p0);
     }
-    tile += tiles_of(f.bytes);
+    tile += (f.bytes + kFillTileBytes - 1) / kFillTileBytes;
+    if (f.bytes != 0 && f.dist == ASMV_DIST_NORMAL) {
+      const uint32_t sz = (uint32_t)kDtypeSize[r.dtype];
+      needs |= sz == 2 ? kNeedN16 : sz == 1 ? kNeedN8 : kNeedLn;
+    }
     add_region_guards(segs, r, kSegFill, (uint32_t)i);
   }
   std::memset(&fr[n], 0, sizeof(FillRegion));
@@ -609,13 +621,14 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   p.seed = seed;
   p.nregions = (uint32_t)n;
   p.nsegs = (uint32_t)segs.size();
+  p.smem = fill_layout(needs);
   for (uint32_t r = 0; r < 10; ++r) {      // Philox round keys (Weyl sequence from the seed)
     p.key0[r] = (uint32_t)seed + r * 0x9E3779B9u;
     p.key1[r] = (uint32_t)(seed >> 32) + r * 0xBB67AE85u;
   }
   cudaError_t e;
   if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
-  if ((e = (cudaError_t)launch_fill(p, grid_for(ctx, tile, segs.size(), ctx->fill_ctas), s)) !=
+  if ((e = (cudaError_t)launch_fill(p, grid_for(ctx, tile, segs.size(), ctx->fill_ctas[needs]), s)) !=
       cudaSuccess)
     return fail_cuda(ctx, e);
   ctx->launches += 1;

@@ -3,14 +3,21 @@
 // its distribution, and both guard bands receive the region's canary byte.
 //
 // One 16-byte chunk c of a payload always holds the same bytes, whatever
-// the payload's address: RAW chunk c is Philox block c; other distributions
-// map element i to word (i mod 4) of block (i div 4) (NORMAL: Box-Muller on
-// word pairs (0,1) and (2,3)).  Aligned payloads are written with 128-bit
-// stores; unaligned payloads and the short last chunk with byte stores.
+// the payload's address: RAW chunk c is Philox block c; fp32 UNIFORM and
+// NORMAL map element i to word (i mod 4) of block (i div 4) (NORMAL:
+// Box-Muller on word pairs (0,1) and (2,3)), binary64 to half of such a
+// block; the 16-bit and 8-bit float formats take one block per chunk, so
+// that each element draws as many Philox bits as it stores (16-bit: a
+// Box-Muller pair per word, UNIFORM a 16-bit fraction per half word; 8-bit:
+// a pair per half word, UNIFORM an 8-bit fraction per byte).  Aligned
+// payloads are written with 128-bit stores; unaligned payloads and the
+// short last chunk with byte stores.
 //
-// Roofline: HBM writes of payload + guard bytes; Philox (about 80 integer
-// operations per 16-byte block) and Box-Muller for NORMAL also load the
-// ALUs, so 16-bit and 8-bit NORMAL fills are arithmetic-bound.
+// Roofline: HBM writes of payload + guard bytes.  Philox costs 20 wide
+// multiplies per block on the FMA-heavy pipe, so a RAW fill is co-limited by
+// the block rate; NORMAL adds its transform, which makes the fill
+// issue-bound for every NORMAL format.  Each thread computes two chunks at a
+// time so that the two Philox chains overlap.
 #include "fill_math.cuh"
 #include "ln_table.h"
 
@@ -24,7 +31,7 @@ __device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
 
 // v = mean + sd*z for the four normals of a block, two per packed
 // instruction: v[0], v[2] from z0 of the two pairs, v[1], v[3] from z1.
-__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const float4 *tab, float v[4]) {
+__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const uint8_t *tab, float v[4]) {
   float2 z0, z1;
   box_muller2(w, tab, z0, z1);
   const float2 a = __fadd2_rn(f2(mean), __fmul2_rn(f2(sd), z0));
@@ -41,25 +48,45 @@ __device__ __forceinline__ void uniform4(uint4 w, float lo, float width, float v
   v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
 }
 
+// UNIFORM of the narrow formats: v = lo + (k scale) width, k a 16-bit or
+// 8-bit field (k scale is exact).
+__device__ __forceinline__ float uniform_frac(uint32_t k, float scale, float lo, float width) {
+  return __fadd_rn(lo, __fmul_rn(__fmul_rn(__uint2float_rn(k), scale), width));
+}
+
 __device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span) {
   return (uint32_t)(lo + (int64_t)(((uint64_t)w * span) >> 32));
 }
 
-// Round keys of a launch and the ln table (in shared memory).
+// Round keys of a launch and this lane's copies of the shared-memory tables.
 struct Keys {
   const uint32_t *k0, *k1;
-  const float4 *lntab;
+  const uint8_t *sm;
+  const uint8_t *ln;        // ln reduction row 0 (fp32 / binary64 NORMAL)
+  uint32_t offT;            // angle table entry 0
+  uint32_t offR16;          // 16-bit radius chord "entry 1776" (the bias of F' >> 19)
+  uint32_t offR8;           // 8-bit radius entry 0
 };
 
 __device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id, uint64_t b) {
   return philox10_keyed(make_uint4((uint32_t)b, (uint32_t)(b >> 32), region_id, 0u), K.k0, K.k1);
 }
 
-// Four fp32 values of one block, per float distribution.
+// Four fp32 values of one block (fp32 formats), per float distribution.
 template <uint32_t DIST>
 __device__ __forceinline__ void float4_of(uint4 w, const FillRegion &r, const Keys &K, float v[4]) {
-  if (DIST == kNormal) normal4(w, r.f0, r.f1, K.lntab, v);
+  if (DIST == kNormal) normal4(w, r.f0, r.f1, K.ln, v);
   else uniform4(w, r.f0, r.f1, v);
+}
+
+__device__ __forceinline__ uint32_t pack_fp8(uint32_t DT, const float v[4]) {
+  if (DT == kF8) return pack_f8x4(v[0], v[1], v[2], v[3]);
+  if (DT == kF8E5M2) return pack_e5m2x4(v[0], v[1], v[2], v[3]);
+  if (DT == kF8E4FNUZ)
+    return enc_e4m3fnuz(v[0]) | (enc_e4m3fnuz(v[1]) << 8) | (enc_e4m3fnuz(v[2]) << 16) |
+           (enc_e4m3fnuz(v[3]) << 24);
+  return enc_e5m2fnuz(v[0]) | (enc_e5m2fnuz(v[1]) << 8) | (enc_e5m2fnuz(v[2]) << 16) |
+         (enc_e5m2fnuz(v[3]) << 24);
 }
 
 // The 16 bytes of chunk c.
@@ -106,8 +133,8 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     float v0, v1;
     if (DIST == kNormal) {
       float z0, z1;
-      if (c & 1) box_muller(w.z, w.w, K.lntab, z0, z1);
-      else box_muller(w.x, w.y, K.lntab, z0, z1);
+      if (c & 1) box_muller(w.z, w.w, K.ln, z0, z1);
+      else box_muller(w.x, w.y, K.ln, z0, z1);
       v0 = __fadd_rn(r.f0, __fmul_rn(r.f1, z0));
       v1 = __fadd_rn(r.f0, __fmul_rn(r.f1, z1));
     } else {
@@ -123,47 +150,62 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     float4_of<DIST>(payload_block(K, r.region_id, c), r, K, v);
     return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
                       __float_as_uint(v[3]));
-  } else if (DT == kBF16 || DT == kF16) {       // 8 elements: blocks 2c, 2c+1
-    uint32_t out[4];
+  }
+  const uint4 w = payload_block(K, r.region_id, c);   // the narrow formats: block c
+  const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+  uint32_t out[4];
+  if (DT == kBF16 || DT == kF16) {              // 8 elements: a pair (or two fractions) per word
 #pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      float v[4];
-      float4_of<DIST>(payload_block(K, r.region_id, 2 * c + q), r, K, v);
-      if (DT == kBF16) { out[2 * q] = pack_bf16x2(v[0], v[1]); out[2 * q + 1] = pack_bf16x2(v[2], v[3]); }
-      else { out[2 * q] = pack_f16x2(v[0], v[1]); out[2 * q + 1] = pack_f16x2(v[2], v[3]); }
+    for (int q = 0; q < 4; ++q) {
+      float a, b;
+      if (DIST == kNormal) {
+        normal16_pair(ww[q], K.sm, K.offR16, K.offT, r.f0, r.f1, a, b);
+      } else {
+        a = uniform_frac(ww[q] & 0xFFFFu, 0x1p-16f, r.f0, r.f1);
+        b = uniform_frac(ww[q] >> 16, 0x1p-16f, r.f0, r.f1);
+      }
+      out[q] = (DT == kBF16) ? pack_bf16x2(a, b) : pack_f16x2(a, b);
     }
-    return make_uint4(out[0], out[1], out[2], out[3]);
-  } else {                                      // fp8: 16 elements, blocks 4c..4c+3
-    uint32_t out[4];
+  } else {                                      // fp8: 16 elements, four per word
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       float v[4];
-      float4_of<DIST>(payload_block(K, r.region_id, 4 * c + q), r, K, v);
-      if (DT == kF8) out[q] = pack_f8x4(v[0], v[1], v[2], v[3]);
-      else if (DT == kF8E5M2) out[q] = pack_e5m2x4(v[0], v[1], v[2], v[3]);
-      else if (DT == kF8E4FNUZ)
-        out[q] = enc_e4m3fnuz(v[0]) | (enc_e4m3fnuz(v[1]) << 8) | (enc_e4m3fnuz(v[2]) << 16) |
-                 (enc_e4m3fnuz(v[3]) << 24);
-      else
-        out[q] = enc_e5m2fnuz(v[0]) | (enc_e5m2fnuz(v[1]) << 8) | (enc_e5m2fnuz(v[2]) << 16) |
-                 (enc_e5m2fnuz(v[3]) << 24);
+      if (DIST == kNormal) {
+        normal8_word(ww[q], K.sm, K.offR8, K.offT, r.f0, r.f1, v);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) v[e] = uniform_frac((ww[q] >> (8 * e)) & 0xFFu, 0x1p-8f, r.f0, r.f1);
+      }
+      out[q] = pack_fp8(DT, v);
     }
-    return make_uint4(out[0], out[1], out[2], out[3]);
   }
+  return make_uint4(out[0], out[1], out[2], out[3]);
 }
 
+__device__ __forceinline__ void store_chunk(const FillRegion &r, uint64_t c, uint64_t full, uint4 v) {
+  const uint64_t addr = r.payload + 16 * c;
+  if (r.vec && c < full) stg16(addr, v);
+  else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * c));
+}
+
+// Thread t makes chunks t + 2 k kFillThreads and t + (2 k + 1) kFillThreads
+// of the tile together, so that their Philox chains overlap; where a thread
+// has no second chunk it recomputes its first and stores once.
 template <uint32_t DIST, uint32_t DT>
 __device__ void fill_tile(const FillRegion &r, const Keys &K, uint64_t tile_in_region) {
-  const uint64_t c0 = tile_in_region * kTileChunks;
+  const uint64_t c0 = tile_in_region * kFillTileChunks;
   const uint64_t nchunks = (r.bytes + 15) >> 4;
   const uint64_t full = r.bytes >> 4;
-  const uint32_t nloc = (uint32_t)umin64(kTileChunks, nchunks - c0);
-  for (uint32_t i = threadIdx.x; i < nloc; i += kThreads) {
-    const uint64_t c = c0 + i;
-    const uint4 v = make_chunk<DIST, DT>(r, K, c);
-    const uint64_t addr = r.payload + 16 * c;
-    if (r.vec && c < full) stg16(addr, v);
-    else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * c));
+  const uint32_t nloc = (uint32_t)umin64(kFillTileChunks, nchunks - c0);
+#pragma unroll 1
+  for (uint32_t i = threadIdx.x; i < nloc; i += 2 * kFillThreads) {
+    const uint32_t i2 = i + kFillThreads;
+    const bool two = i2 < nloc;
+    const uint64_t ca = c0 + i, cb = c0 + (two ? i2 : i);
+    const uint4 va = make_chunk<DIST, DT>(r, K, ca);
+    const uint4 vb = make_chunk<DIST, DT>(r, K, cb);
+    store_chunk(r, ca, full, va);
+    if (two) store_chunk(r, cb, full, vb);
   }
 }
 
@@ -218,16 +260,33 @@ __device__ __noinline__ uint32_t next_region(const FillRegion *regs, uint32_t n,
   return lo;
 }
 
-__global__ void __launch_bounds__(kThreads, 6) fill_kernel(const FillParams p) {
-  __shared__ float4 lntab[ASMV_LN_TABLE_ROWS];
-  for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS; i += kThreads) lntab[i] = kLnTableInit[i];
+// Copy `entries` table entries of T into shared memory at `off`, `copies`
+// copies of each side by side.
+template <class T>
+__device__ __forceinline__ void load_table(uint8_t *sm, uint32_t off, const T *src, uint32_t entries,
+                                           uint32_t copies) {
+  for (uint32_t i = threadIdx.x; i < entries * copies; i += kFillThreads)
+    *reinterpret_cast<T *>(sm + off + sizeof(T) * i) = src[i / copies];
+}
+
+__global__ void __launch_bounds__(kFillThreads) fill_kernel(const __grid_constant__ FillParams p) {
+  extern __shared__ __align__(16) uint8_t sm[];
+  const FillLayout &L = p.smem;
+  if (L.angle != kNoTable) load_table(sm, L.angle, kAngleTable, 256, kAngleCopies);
+  if (L.rad16 != kNoTable) load_table(sm, L.rad16, kRadius16Table, 512, kRad16Copies);
+  if (L.rad8 != kNoTable) load_table(sm, L.rad8, kRadius8Table, 256, kRad8Copies);
+  if (L.ln != kNoTable) load_table(sm, L.ln, kLnTableInit, ASMV_LN_TABLE_ROWS, kLnCopies);
   __syncthreads();
+  const uint32_t lane = threadIdx.x & 31;
   const uint64_t G = gridDim.x, b = blockIdx.x;
   // Tiles b, b + G, b + 2G, ...: every CTA gets its share of every region,
   // so regions of very different cost per tile (NORMAL against RAW) spread
   // evenly over the SMs.
   if (b < p.ntiles) {
-    const Keys K = {p.key0, p.key1, lntab};
+    const Keys K = {p.key0, p.key1, sm, sm + L.ln + 16u * (lane % kLnCopies),
+                    L.angle + 8u * (lane % kAngleCopies),
+                    L.rad16 + 8u * (lane % kRad16Copies) - 1776u * 8u * kRad16Copies,
+                    L.rad8 + 4u * (lane % kRad8Copies)};
     uint32_t ri = find_region(p.regions, p.nregions, b);
     for (uint64_t t = b; t < p.ntiles; t += G) {
       if (p.regions[ri + 1].tile0 <= t) ri = next_region(p.regions, p.nregions, ri, t);
@@ -236,8 +295,7 @@ __global__ void __launch_bounds__(kThreads, 6) fill_kernel(const FillParams p) {
     }
   }
   // guard bands: one warp per segment
-  const uint32_t lane = threadIdx.x & 31;
-  const uint64_t warp = b * kWarps + (threadIdx.x >> 5), nw = G * kWarps;
+  const uint64_t warp = b * kFillWarps + (threadIdx.x >> 5), nw = G * kFillWarps;
   for (uint64_t s = warp; s < p.nsegs; s += nw) {
     const GuardSeg g = p.segs[s];
     uint8_t *dst = reinterpret_cast<uint8_t *>(g.ptr);
@@ -247,15 +305,22 @@ __global__ void __launch_bounds__(kThreads, 6) fill_kernel(const FillParams p) {
 
 }  // namespace
 
-int fill_max_ctas_per_sm() {
+// CTAs of the fill per SM with `smem_bytes` of tables, on the current device
+// (which also receives the kernel's shared-memory opt-in); 0 on an error.
+int fill_max_ctas_per_sm(uint32_t smem_bytes) {
+  const size_t most = (size_t)kAngleBytes + kRad16Bytes + kRad8Bytes + kLnBytes;
+  if (cudaFuncSetAttribute(fill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)most) !=
+      cudaSuccess)
+    return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fill_kernel, kThreads, 0) != cudaSuccess)
-    return 1;
-  return n > 0 ? n : 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fill_kernel, kFillThreads, smem_bytes) !=
+      cudaSuccess)
+    return 0;
+  return n;
 }
 
 int launch_fill(const FillParams &p, int grid, void *stream) {
-  fill_kernel<<<grid, kThreads, 0, (cudaStream_t)stream>>>(p);
+  fill_kernel<<<grid, kFillThreads, p.smem.bytes, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }
 

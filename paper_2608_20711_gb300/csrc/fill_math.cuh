@@ -7,6 +7,7 @@
 // states, which makes the filled bytes reproducible on any IEEE machine.
 #pragma once
 #include "device.cuh"
+#include "fill_tables.h"
 
 namespace asmv {
 
@@ -36,8 +37,12 @@ __device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, con
 // ln(u), u = k 2^-24: u = m 2^e with m in [1, 2); j = round(128 (m - 1));
 // r = m*inv_j - 1 exactly (fma); ln u = e ln2 + (-ln inv_j) + log1p(r), with
 // ln 2 and -ln inv_j split into a 2^-9-multiple head (exact sum) and an fp32
-// tail, and log1p(r) = r + r^2 (-1/2 + r (1/3 - r/4)) for |r| < 2^-7.  The
-// table lives in shared memory (ln_table.h).
+// tail, and log1p(r) = r + r^2 (-1/2 + r (1/3 - r/4)) for |r| < 2^-7: the
+// table-driven logarithm of P. T. P. Tang ("Table-driven implementation of
+// the logarithm function in IEEE floating-point arithmetic", ACM TOMS 16,
+// 1990), with this library's table and series.  The table lives in shared
+// memory (ln_table.h), kLnCopies copies of each row side by side; `ln` is the
+// address of this lane's copy of row 0.
 // sin/cos(2 pi u): nearest quarter turn removed exactly in integers, then the
 // Taylor series of sin(pi/2 r) and cos(pi/2 r) for r in [-1/2, 1/2); each
 // coefficient is the fp32 rounding of +-(pi/2)^j / j!.
@@ -55,13 +60,17 @@ __device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, con
 #define ASMV_C8 0x1.e1f506p-11f
 #define ASMV_C10 (-0x1.a6d1f2p-16f)
 
-__device__ __forceinline__ float ln_u24(uint32_t k, const float4 *tab) {
+__device__ __forceinline__ float4 ln_row(const uint8_t *ln, uint32_t j) {
+  return *reinterpret_cast<const float4 *>(ln + j * (16u * kLnCopies));
+}
+
+__device__ __forceinline__ float ln_u24(uint32_t k, const uint8_t *tab) {
   const float u = __fmul_rn(__uint2float_rn(k), 0x1p-24f);   // exact
   const uint32_t bits = __float_as_uint(u);
   const int e = (int)(bits >> 23) - 127;
   const uint32_t mb = bits & 0x7FFFFFu;
   const float m = __uint_as_float(mb | 0x3F800000u);
-  const float4 t = tab[(mb + (1u << 15)) >> 16];             // inv, hi, lo
+  const float4 t = ln_row(tab, (mb + (1u << 15)) >> 16);       // inv, hi, lo
   const float r = __fmaf_rn(m, t.x, -1.0f);                  // exact
   const float r2 = __fmul_rn(r, r);
   float p = __fmaf_rn(r, -0.25f, ASMV_THIRD);
@@ -113,7 +122,7 @@ __device__ __forceinline__ float sqrt_radius(float x) {
   return x == 0.0f ? x : y;
 }
 
-__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const float4 *tab, float &z0,
+__device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const uint8_t *tab, float &z0,
                                            float &z1) {
   const float l = ln_u24((w0 >> 8) + 1u, tab);
   const float rho = sqrt_radius(__fmul_rn(-2.0f, l));
@@ -130,13 +139,13 @@ __device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const float
 // z0 = (z0 of pair a, z0 of pair b), z1 likewise.
 __device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
 
-__device__ __forceinline__ void box_muller2(uint4 w, const float4 *tab, float2 &z0, float2 &z1) {
+__device__ __forceinline__ void box_muller2(uint4 w, const uint8_t *tab, float2 &z0, float2 &z1) {
   // ln(k 2^-24), k = (w >> 8) + 1
   const uint32_t ka = (w.x >> 8) + 1u, kb = (w.z >> 8) + 1u;
   const float2 u = __fmul2_rn(make_float2(__uint2float_rn(ka), __uint2float_rn(kb)), f2(0x1p-24f));
   const uint32_t ba = __float_as_uint(u.x), bb = __float_as_uint(u.y);
   const uint32_t ma = ba & 0x7FFFFFu, mb = bb & 0x7FFFFFu;
-  const float4 ta = tab[(ma + (1u << 15)) >> 16], tb = tab[(mb + (1u << 15)) >> 16];
+  const float4 ta = ln_row(tab, (ma + (1u << 15)) >> 16), tb = ln_row(tab, (mb + (1u << 15)) >> 16);
   const float2 m = make_float2(__uint_as_float(ma | 0x3F800000u), __uint_as_float(mb | 0x3F800000u));
   const float2 r = __ffma2_rn(m, make_float2(ta.x, tb.x), f2(-1.0f));
   const float2 r2 = __fmul2_rn(r, r);
@@ -182,6 +191,86 @@ __device__ __forceinline__ void box_muller2(uint4 w, const float4 *tab, float2 &
                                 __uint_as_float(__float_as_uint(cb) ^ (((qb + 1u) & 2u) << 30)));
   z0 = __fmul2_rn(rho, cs);
   z1 = __fmul2_rn(rho, sn);
+}
+
+// ---------------------------------------------------------------- narrow formats
+// Box-Muller for the 16-bit and 8-bit formats: one Philox block per 16-byte
+// chunk, so every element draws as many Philox bits as it stores.
+//
+// 16-bit formats, one pair per 32-bit word w.  Radius from the low half k:
+// u = (k + 1/2) 2^-16; with d = bit 15 of w (u > 1/2), x = u or 1 - u is
+// K 2^-17 for the odd K = 2t + 1, t = (k mod 2^15) xor (d ? 2^15 - 1 : 0);
+// F = K 2^(16 d) is exact in fp32, its exponent and top four mantissa bits
+// pick a chord (A, B) of rho = sqrt(-2 ln u) over a cell of relative width
+// 1/16 (within 2^-13 of the curve), and rho = fma(F, A, B).  The kernel
+// forms F' = F 2^-16 (its scale 2^-16 or 1 is one OR into the bits of
+// 2^-16) and uses A' = A 2^16 from fill_tables.h: F' A' = F A exactly, so
+// rho is the same; the cell of F' is entry (bits(F') >> 19) - 1776.  Angle from the
+// high half a = (j, n): theta = 2 pi (a + 1/2) / 65536 is the table angle
+// phi_j = 2 pi (j + 1/2) / 256 turned by delta = (n - 127.5) 2 pi / 65536,
+// taken to first order: (sin, cos) = (S + C delta, C - S delta), which is a
+// rotation by atan(delta) (within 2^-20.5 rad of delta) scaled by
+// sqrt(1 + delta^2) <= 1 + 2^-13.7.
+//
+// 8-bit formats, one pair per 16-bit half h: rho = R8[h mod 256] =
+// sqrt(-2 ln((k + 1/2) / 256)) and (sin, cos) = table entry h div 256.
+//
+// Values: rs = rho * std, v0 = fma(rs, cos, mean), v1 = fma(rs, sin, mean).
+// The tables come from fill_tables.h; in shared memory each entry has
+// k{Angle,Rad16,Rad8}Copies copies side by side, and every address below is
+// this lane's copy (the `off*` arguments hold the lane's copy of entry 0).
+__device__ __forceinline__ uint32_t mad32(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
+// Bit 15 of w copied into every bit (PTX prmt with the sign-replicating
+// selector 0x9: the sign of byte 1 in each result byte).
+__device__ __forceinline__ uint32_t bit15_mask(uint32_t w) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, 0, 0x9999;" : "=r"(r) : "r"(w));
+  return r;
+}
+
+template <class T>
+__device__ __forceinline__ T lds(const uint8_t *sm, uint32_t off) {
+  return *reinterpret_cast<const T *>(sm + off);
+}
+
+__device__ __forceinline__ void normal16_pair(uint32_t w, const uint8_t *sm, uint32_t offR,
+                                              uint32_t offT, float mean, float sd, float &v0,
+                                              float &v1) {
+  const uint32_t sx = bit15_mask(w);
+  const uint32_t t = (w ^ sx) & 0x7FFFu;
+  const float scl = __uint_as_float((sx & 0x08000000u) | 0x37800000u);       // 2^-16 or 1
+  const float F = __fmul_rn(__fsub_rn(__uint_as_float(mad32(t, 2u, 0x4B000001u)), 8388608.0f), scl);
+  // chord of the cell (exponent, top four mantissa bits of F'): entry (F' >> 19) - 1776
+  const float2 ab = lds<float2>(sm, mad32(__float_as_uint(F) >> 19, 8u * kRad16Copies, offR));
+  const float rho = __fmaf_rn(F, ab.x, ab.y);
+  const float x = __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7442u));   // 2^23 + n
+  const float delta = __fmaf_rn(__fsub_rn(x, 8388736.0f), ASMV_C16, ASMV_C16_HALF);
+  const float2 sc = lds<float2>(sm, mad32(w >> 24, 8u * kAngleCopies, offT));   // (S, C)
+  const float sn = __fmaf_rn(sc.y, delta, sc.x);
+  const float cs = __fmaf_rn(-sc.x, delta, sc.y);
+  const float rs = __fmul_rn(rho, sd);
+  v0 = __fmaf_rn(rs, cs, mean);
+  v1 = __fmaf_rn(rs, sn, mean);
+}
+
+// The two pairs of word w (halves low, then high): v[0..3] = v0, v1 of the
+// low half, v0, v1 of the high half.
+__device__ __forceinline__ void normal8_word(uint32_t w, const uint8_t *sm, uint32_t offR,
+                                             uint32_t offT, float mean, float sd, float v[4]) {
+  const float ra = lds<float>(sm, mad32(__byte_perm(w, 0u, 0x4440u), 4u * kRad8Copies, offR));
+  const float2 ta = lds<float2>(sm, mad32(__byte_perm(w, 0u, 0x4441u), 8u * kAngleCopies, offT));
+  const float rb = lds<float>(sm, mad32(__byte_perm(w, 0u, 0x4442u), 4u * kRad8Copies, offR));
+  const float2 tb = lds<float2>(sm, mad32(w >> 24, 8u * kAngleCopies, offT));
+  const float sa = __fmul_rn(ra, sd), sb = __fmul_rn(rb, sd);
+  v[0] = __fmaf_rn(sa, ta.y, mean);
+  v[1] = __fmaf_rn(sa, ta.x, mean);
+  v[2] = __fmaf_rn(sb, tb.y, mean);
+  v[3] = __fmaf_rn(sb, tb.x, mean);
 }
 
 // ---------------------------------------------------------------- encoders

@@ -2,16 +2,17 @@
 // the kernels (fill.cu, compare.cu).  Internal to the library.
 //
 // Work decomposition.  Every region's payload is cut into tiles of
-// kTileBytes for the fill, and of a per-launch tile size for the compare
-// (the last tile of a region may be short).  Tiles of all
+// kFillTileBytes for the fill, kTileBytes for the Eq. 1 sums and the
+// restore, and of a per-launch tile size for the compare (the last tile of a
+// region may be short).  Tiles of all
 // regions form one index space; region i owns tiles [tile0[i], tile0[i+1]).
 // A launch runs a persistent grid.  In the compare and the Eq. 1 sums CTA b
 // takes the contiguous tile range [T*b/G, T*(b+1)/G), so a CTA crosses few
 // region boundaries and flushes its per-region partial statistics once per
 // boundary; the fill, which keeps no per-region state, takes tiles b, b+G,
 // b+2G, ..., so that regions of very different cost per tile spread evenly
-// over the SMs.  Inside a tile, thread t handles 16-byte chunks t, t+256,
-// ... (coalesced 128-bit accesses).
+// over the SMs.  Inside a tile, thread t handles 16-byte chunks t, t+T, ...
+// for a CTA of T threads (coalesced 128-bit accesses).
 //
 // Guard bands are cut into segments of at most kGuardSegBytes and handled
 // one warp per segment after the payload tiles.
@@ -97,6 +98,41 @@ struct StatsDev {
   unsigned long long guard_bad, guard_first, ref_guard_bad;
 };
 
+// The fill runs CTAs of kFillThreads; each CTA copies into shared memory
+// only the tables its launch needs, every entry replicated so that the lanes
+// of a warp read distinct banks: the angle table (256 x 8 B, 16 copies) and
+// the 16-bit radius chords (512 x 8 B, 8 copies) for 16-bit NORMAL, the
+// angle table and the 8-bit radii (256 x 4 B, 16 copies) for 8-bit NORMAL,
+// the ln reduction table (129 x 16 B, 8 copies) for fp32 and binary64
+// NORMAL.  fill_layout() gives the byte offsets for a set of needs.
+constexpr int kFillThreads = 512;
+constexpr int kFillWarps = kFillThreads / 32;
+// The fill's tiles are 64 KiB (eight chunks per thread, two at a time), so
+// the per-tile work (region lookup, dispatch) is spread over more chunks.
+constexpr int kFillTileChunks = 4096;
+constexpr uint64_t kFillTileBytes = (uint64_t)kChunkBytes * kFillTileChunks;
+enum : uint32_t { kNeedN16 = 1, kNeedN8 = 2, kNeedLn = 4 };
+constexpr uint32_t kAngleCopies = 16, kRad16Copies = 8, kRad8Copies = 16, kLnCopies = 8;
+constexpr uint32_t kNoTable = 0xFFFFFFFFu;
+constexpr uint32_t kAngleBytes = 256 * 8 * kAngleCopies;     // 32 KiB
+constexpr uint32_t kRad16Bytes = 512 * 8 * kRad16Copies;     // 32 KiB
+constexpr uint32_t kRad8Bytes = 256 * 4 * kRad8Copies;       // 16 KiB
+constexpr uint32_t kLnBytes = 129 * 16 * kLnCopies;          // 16.1 KiB
+
+struct FillLayout {
+  uint32_t angle, rad16, rad8, ln;   // byte offsets in shared memory, kNoTable if absent
+  uint32_t bytes;                    // dynamic shared memory of the launch
+};
+
+inline FillLayout fill_layout(uint32_t needs) {
+  FillLayout L = {kNoTable, kNoTable, kNoTable, kNoTable, 0};
+  if (needs & (kNeedN16 | kNeedN8)) { L.angle = L.bytes; L.bytes += kAngleBytes; }
+  if (needs & kNeedN16) { L.rad16 = L.bytes; L.bytes += kRad16Bytes; }
+  if (needs & kNeedN8) { L.rad8 = L.bytes; L.bytes += kRad8Bytes; }
+  if (needs & kNeedLn) { L.ln = L.bytes; L.bytes += kLnBytes; }
+  return L;
+}
+
 struct FillParams {
   const FillRegion *regions;   // nregions + 1 entries (sentinel)
   const GuardSeg *segs;
@@ -104,6 +140,7 @@ struct FillParams {
   uint64_t seed;
   uint32_t nregions;
   uint32_t nsegs;
+  FillLayout smem;             // the tables in shared memory
   // Philox key of each of the 10 rounds: (seed lo, seed hi) advanced by the
   // Weyl increments, precomputed on the host (kernel-parameter operands)
   uint32_t key0[10], key1[10];
@@ -173,7 +210,7 @@ struct CopyParams {
 // Launchers (defined in fill.cu / compare.cu / eqsum.cu / copy.cu).  Return a cudaError_t.
 int launch_fill(const FillParams &p, int grid, void *stream);
 int launch_compare(const CmpParams &p, int grid, void *stream);
-int fill_max_ctas_per_sm();
+int fill_max_ctas_per_sm(uint32_t smem_bytes);
 uint32_t compare_tile_bytes(uint32_t K);
 uint32_t compare_stages(uint32_t K, uint32_t tile_bytes);
 size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes, uint32_t nstages);

@@ -8,12 +8,15 @@
 #include "ln_table.h"
 
 __global__ void check(unsigned long long *bad, unsigned int *first) {
-  __shared__ float4 tab[ASMV_LN_TABLE_ROWS];
-  for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS; i += blockDim.x) tab[i] = kLnTableInit[i];
+  // the ln table as the fill keeps it: kLnCopies copies of each row side by side
+  __shared__ float4 tab[ASMV_LN_TABLE_ROWS * asmv::kLnCopies];
+  for (int i = threadIdx.x; i < ASMV_LN_TABLE_ROWS * (int)asmv::kLnCopies; i += blockDim.x)
+    tab[i] = kLnTableInit[i / asmv::kLnCopies];
   __syncthreads();
   const unsigned int k = blockIdx.x * blockDim.x + threadIdx.x + 1u;   // 1 .. 2^24
   if (k > (1u << 24)) return;
-  const float x = __fmul_rn(-2.0f, asmv::ln_u24(k, tab));
+  const uint8_t *row0 = reinterpret_cast<const uint8_t *>(tab) + 16u * (threadIdx.x % asmv::kLnCopies);
+  const float x = __fmul_rn(-2.0f, asmv::ln_u24(k, row0));
   if (__float_as_uint(__fsqrt_rn(x)) != __float_as_uint(asmv::sqrt_radius(x))) {
     atomicAdd(bad, 1ull);
     atomicMin(first, k);

@@ -121,22 +121,38 @@ def test_encode_f64_is_exact_widening(oracle):
 
 @pytest.mark.parametrize("name", ["F8E5M2", "F8E4M3FNUZ", "F8E5M2FNUZ", "F64"])
 def test_fill_float_mappings(oracle, torch_philox, name):
+    """binary64 takes word (i mod 4) of block i div 4 (UNIFORM) and the pairs
+    of words (0, 1), (2, 3) (NORMAL); the 8-bit formats take byte (i mod 4)
+    of word (i mod 16) div 4 of block i div 16 (UNIFORM, f = b 2^-8) and the
+    8 + 8 pair of half (i mod 4) div 2 of that word (NORMAL)."""
     code = getattr(oracle, name)
     n = 4099
     size = oracle.DTYPE_SIZE[code]
+    per = 16 // size if size == 1 else 4
     p = np.zeros(n * size, np.uint8)
     oracle.fill_payload(p, code, oracle.UNIFORM, 0, n, 5, -3.0, 5.0, 21)
-    w = torch_philox(21, 5, np.arange((n + 3) // 4)).reshape(-1)[:n]
-    v = np.float32(-3.0) + ((w >> 8).astype(np.float32) * np.float32(2.0 ** -24)) * np.float32(8.0)
+    w = torch_philox(21, 5, np.arange((n + per - 1) // per)).reshape(-1)
+    if size == 1:
+        f = np.stack([(w >> (8 * q)) & 0xFF for q in range(4)], axis=1).reshape(-1)[:n]
+        f = f.astype(np.float32) * np.float32(2.0 ** -8)
+    else:
+        f = (w[:n] >> 8).astype(np.float32) * np.float32(2.0 ** -24)
+    v = np.float32(-3.0) + f * np.float32(8.0)
     want = oracle.encode(v, code)
     np.testing.assert_array_equal(p, want)
     q = np.zeros(n * size, np.uint8)
     oracle.fill_payload(q, code, oracle.NORMAL, 0, n, 6, 0.5, 2.0, 22)
-    w = torch_philox(22, 6, np.arange((n + 3) // 4))
-    z0a, z1a = oracle.boxmuller(w[:, 0], w[:, 1])
-    z0b, z1b = oracle.boxmuller(w[:, 2], w[:, 3])
-    z = np.stack([z0a, z1a, z0b, z1b], axis=1).reshape(-1)[:n]
-    np.testing.assert_array_equal(q, oracle.encode(np.float32(0.5) + np.float32(2.0) * z, code))
+    w = torch_philox(22, 6, np.arange((n + per - 1) // per))
+    if size == 1:
+        h = np.stack([w & 0xFFFF, w >> 16], axis=2).reshape(-1)
+        v0, v1 = oracle.normal8(h, 0.5, 2.0)
+        vz = np.stack([v0, v1], axis=1).reshape(-1)[:n]
+    else:
+        z0a, z1a = oracle.boxmuller(w[:, 0], w[:, 1])
+        z0b, z1b = oracle.boxmuller(w[:, 2], w[:, 3])
+        z = np.stack([z0a, z1a, z0b, z1b], axis=1).reshape(-1)[:n]
+        vz = np.float32(0.5) + np.float32(2.0) * z
+    np.testing.assert_array_equal(q, oracle.encode(vz, code))
     if name != "F64":
         tdt = FP8[name][0]
         inr = np.abs(v) <= FP8[name][1]

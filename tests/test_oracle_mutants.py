@@ -21,9 +21,11 @@ from oracle import oracle as O
 PIN_MODULES = ("tests.test_oracle_codecs", "tests.test_oracle_philox",
                "tests.test_oracle_fill", "tests.test_oracle_compare",
                "tests.test_oracle_eq", "tests.test_oracle_dtypes", "tests.test_oracle_restore",
-               "tests.test_oracle_boxmuller", "tests.test_oracle_eq64")
+               "tests.test_oracle_boxmuller", "tests.test_oracle_eq64",
+               "tests.test_oracle_narrow")
 # pins that take seconds run last, in this order
-EXPENSIVE = ("test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
+EXPENSIVE = ("test_normal16_is_standard_normal", "test_narrow_tables_are_correctly_rounded",
+             "test_boxmuller_is_standard_normal", "test_sincos_2pi_u24_all_inputs",
              "test_ln_u24_all_inputs")
 
 # (name, text in the oracle source, replacement): each text occurs once
@@ -62,13 +64,44 @@ MUTANTS = [
     ("u1_offset_dropped", "oracle_ln_u24((w0 >> 8) + 1u)", "oracle_ln_u24(w0 >> 8)"),
     ("cos_sin_outputs_swapped", "*z0 = rho * cs;\n  *z1 = rho * sn;",
      "*z0 = rho * sn;\n  *z1 = rho * cs;"),
+    # the 16-bit and 8-bit formats (reading R12)
+    ("n16_mirror_dropped", "uint32_t t = (k & 0x7FFFu) ^ (d ? 0x7FFFu : 0u);",
+     "uint32_t t = k & 0x7FFFu;"),
+    ("n16_mirror_scale_dropped", "(float)(2u * t + 1u) * (d ? 65536.0f : 1.0f);",
+     "(float)(2u * t + 1u) * 1.0f;"),
+    ("n16_cell_bits", "(int)((b >> 19) & 15u)", "(int)((b >> 20) & 15u)"),
+    ("n16_chord_width", "long double m0 = 1.0L + i / 16.0L, m1 = m0 + 1.0L / 16.0L;",
+     "long double m0 = 1.0L + i / 16.0L, m1 = m0 + 1.0L / 32.0L;"),
+    ("n16_u_scale", "long double y = ldexpl(m, e - 17);", "long double y = ldexpl(m, e - 16);"),
+    ("angle16_half_step_dropped", "fmaf((float)n - 128.0f, C16_STEP, C16_STEP * 0.5f)",
+     "fmaf((float)n - 128.0f, C16_STEP, 0.0f)"),
+    ("angle16_rotation_sign", "*cs = fmaf(-T_SIN[j], delta, T_COS[j]);",
+     "*cs = fmaf(T_SIN[j], delta, T_COS[j]);"),
+    ("angle_table_not_midpoint", "long double phi = 2.0L * pi * (j + 0.5L) / 256.0L;",
+     "long double phi = 2.0L * pi * j / 256.0L;"),
+    ("n16_radius_from_high_half", "float rho = oracle_radius16(w & 0xFFFFu);",
+     "float rho = oracle_radius16(w >> 16);"),
+    ("n16_outputs_swapped", "*v0 = fmaf(rs, cs, mean);\n  *v1 = fmaf(rs, sn, mean);",
+     "*v0 = fmaf(rs, sn, mean);\n  *v1 = fmaf(rs, cs, mean);"),
+    ("n16_std_dropped", "float rs = rho * sd;\n  *v0 = fmaf(rs, cs, mean);",
+     "float rs = rho;\n  *v0 = fmaf(rs, cs, mean);"),
+    ("n8_bytes_swapped", "float rho = R8_RHO[h & 255u];\n  uint32_t j = (h >> 8) & 255u;",
+     "float rho = R8_RHO[(h >> 8) & 255u];\n  uint32_t j = h & 255u;"),
+    ("r8_quantile_not_midpoint", "logl((j + 0.5L) / 256.0L)", "logl((j + 1.0L) / 256.0L)"),
+    ("n8_half_index", "(w[(i % 16) / 4] >> (16 * ((i % 4) / 2))) & 0xFFFFu",
+     "(w[(i % 16) / 4] >> (16 * (i % 2))) & 0xFFFFu"),
+    ("n16_word_index", "oracle_normal16(w[(i % 8) / 2], mean, sd, &v0, &v1);",
+     "oracle_normal16(w[(i % 8) % 4], mean, sd, &v0, &v1);"),
+    ("uniform16_scale", "& 0xFFFFu) * 0x1p-16f;", "& 0xFFFFu) * 0x1p-15f;"),
+    ("uniform8_byte_order", "(w[(i % 16) / 4] >> (8 * (i % 4))) & 0xFFu",
+     "(w[(i % 16) / 4] >> (8 * (3 - i % 4))) & 0xFFu"),
     # Tier-1 fill
     ("raw_big_endian", "(uint8_t)(word >> (8 * (j % 4)))", "(uint8_t)(word >> (8 * (3 - j % 4)))"),
     ("int_range_modulo", "uint64_t off = ((uint64_t)w[i % 4] * span) >> 32;",
      "uint64_t off = (uint64_t)w[i % 4] % span;"),
     ("uniform_sign", "float v = lo + f * width;", "float v = lo - f * width;"),
-    ("uniform_fraction_bits", "float f = (float)(w[i % 4] >> 8) * 0x1p-24f;",
-     "float f = (float)(w[i % 4] >> 9) * 0x1p-23f;"),
+    ("uniform_fraction_bits", "f = (float)(w[i % 4] >> 8) * 0x1p-24f;",
+     "f = (float)(w[i % 4] >> 9) * 0x1p-23f;"),
     ("normal_pair_index", "unsigned pair = (unsigned)((i % 4) / 2);",
      "unsigned pair = (unsigned)((i % 4) % 2);"),
     ("normal_affine_order", "float v = mean + sd * z;", "float v = sd + mean * z;"),
