@@ -40,23 +40,62 @@
 //      every element with as >= |r|/2 -- every element whose c - r may be
 //      inexact -- is flagged as well, and r = 0 makes y = 0, so every
 //      nonzero difference from a zero reference is flagged.
+//  The 16-bit and 8-bit formats are screened in their own format instead
+//  (fp16, each fp8 format through its exact fp16 value, bf16), two
+//  elements per packed instruction.  With s = RN(c - r) in the format,
+//  a = |s|, and per reference element (formed once for all candidates)
+//  lo = max(RZ(lo32), 0), hi = RZ(hi32), where lo32 and hi32 are the fp32
+//  bounds of (1) and (2) and RZ rounds them to the format toward zero,
+//  and y = max(RN(T'*|r| - tiny), 0), tiny the format's least subnormal:
+//  (5) The bracket: where c - r is exact (see (6)), a = D is a value of the
+//      format.  a <= lo gives D <= lo32 < B (proof (1); lo = 0 gives D = 0),
+//      a match.  a > hi gives a > hi32, since a and hi are values of the
+//      format and RZ rounds the non-negative hi32 down, hence D > B (proof
+//      (2)), a mismatch.  So the band left to the exact path, lo < a <= hi,
+//      holds a value of the format only where one lies within the 2^-21
+//      margins of the fp32 bounds.
+//  (6) y <= T|r| and y < |r|/2: T' = RD(Tp (1 - m)) with Tp = min(T, 1/2-),
+//      m = 2^-9 (fp16) or 2^-7 (bf16), which covers the rounding of the
+//      multiply-add (2^-11, resp. 2^-9, relatively; tiny/2 absolutely);
+//      so y <= T'|r| (1 + 2^-11) < Tp|r| or, subnormal, y <= T'|r| - tiny/2;
+//      the max with 0 keeps y >= 0.  An element with a <= y is therefore
+//      exact (if c - r were inexact, |c - r| >= |r| / 2 by Sterbenz's lemma
+//      and exact subnormal arithmetic, so a >= RN(|r|/2) > y) and cannot
+//      raise max_rel (a/|r| <= T <= Rmax, and RN64 is monotone).
+//  (7) Elements with a > y (compared unordered, so a NaN difference counts)
+//      and ambiguous elements (lo < a <= hi) send the chunk to the exact
+//      path.  |r| is replaced by NaN where r is not finite (|r|*0 + |r|),
+//      which makes y = 0 there (and hi infinite or NaN, never exceeded), so
+//      every non-finite value on either side is flagged: y is finite
+//      wherever r is, and an infinite or NaN difference is not below it.  Otherwise d = a, a match iff
+//      a <= lo, a mismatch iff a > hi, and max_abs takes the running
+//      maximum of a in the format (exact).  The fp32 screen takes the same
+//      NaN |r|, with which neither (1) nor (2) can hold.
 // The maxima are order-independent (max of exact values), counts are sums
 // and first_mismatch a minimum, so any grid gives bit-identical results.
 //
-// Work split: one CTA of 17 warps per SM.  The last warp streams each tile
+// Work split: one CTA of 16 warps per SM.  The last warp streams each tile
 // of the reference and of the K <= 8 candidates into shared memory with
-// bulk copies (two or four stages, as fit, mbarrier-completed; the kernel
-// is instantiated per depth); the 16 checking warps are
-// divided among the candidates, so device memory sees the reference once
-// per tile.  Chunks the screen cannot settle are queued per warp and
-// drained lane-parallel.  Each lane keeps its statistics in registers and
-// a warp merges them into the global entries with atomics when its CTA
-// moves to the next region.
+// bulk copies (two to four stages, as fit, mbarrier-completed).  Each of the
+// 15 checking warps takes whole rows of 32 chunks of the tile and checks
+// every candidate against them: a lane reads its reference chunk once,
+// forms its per-element bounds once, and screens the K candidate chunks at
+// the same position, so neither device memory nor the screen's reference
+// work is paid per candidate.  Chunks the screen cannot settle are queued
+// per warp with their candidate and drained lane-parallel; their statistics
+// go to the warp's per-candidate entries in shared memory.  A lane keeps
+// the screen's counts and maxima per candidate in registers, and the warp
+// merges them into the global entries when its CTA moves to the next
+// region.  Sixteen warps in all, four per SM sub-partition, leave each
+// thread 128 registers (a seventeenth would put five warps on one
+// sub-partition and cap every thread at 96, which spilled in the candidate
+// loop): 5088 GB/s against 4864 with 16 checking warps, and 2788 with 8
+// (fp16 [32768,32768] x 8 candidates).
 //
 // Roofline: HBM reads of reference + candidate payloads (reference once per
-// launch of up to 8 candidates); the screen costs about 10 fp32 operations
-// per differing element (its three thresholds on packed f32x2 for the 16-
-// and 8-bit formats), so dense small differences are also ALU-heavy.
+// launch of up to 8 candidates).  The packed screen is about 12 instructions
+// per pair of candidate elements plus 3 per reference pair shared by the
+// candidates.
 #include <float.h>
 #include <math_constants.h>
 #include <atomic>
@@ -200,22 +239,48 @@ template <uint32_t DT> __device__ __forceinline__ constexpr bool is_int_dt() {
   return DT == kI32 || DT == kI8 || DT == kU8 || DT == kI16 || DT == kI64;
 }
 
-// Chunks the screen cannot settle are queued per warp in shared memory and
-// re-examined element by element once per tile, lane-parallel, instead of
-// diverging inside the screen.
-// 32 entries per warp: with 64 the 4096-region snapshot ran 4 % slower
-// (the queues' shared memory comes out of L1), with 16 no faster.
+// ---------------------------------------------------------------- queue
+// Chunks the screen cannot settle are queued per warp in shared memory with
+// their candidate, as copies, and re-examined element by element,
+// lane-parallel, once the queue is half full after a row and when the
+// warp's run over a region ends, instead of diverging inside the screen.
 constexpr uint32_t kQueue = 32;           // chunk entries per warp
 
 struct QEntry {
   uint4 R, C;                             // the raw 16-byte chunks
   unsigned long long e0;                  // element index of the chunk's first element
+  uint32_t k, pad_;                       // the candidate
 };
 
 struct Queue {
   QEntry e[kQueue];
   uint32_t count;
 };
+
+// A warp's statistics of one candidate that do not live in its lanes'
+// registers: everything the exact path finds, and the first mismatch the
+// screen finds.  In shared memory, merged with shared-memory atomics.
+struct ExactStats {
+  unsigned long long first, dabs, drel;
+  uint32_t cnt, nonfin, m32;              // m32: bits of a non-negative float
+  uint32_t th;                            // the screen's relative-error threshold (rel_threshold of drel)
+};
+
+// Shared memory of a compare CTA: [barriers][queues][exact statistics]
+// [stages].  Declared once here so that every function that takes a part
+// of it addresses it as shared memory.
+extern __shared__ __align__(128) unsigned char cmp_smem[];
+constexpr uint32_t kQueueOff = 128;
+constexpr uint32_t kExactOff = kQueueOff + kConsumerWarps * sizeof(Queue);
+constexpr uint32_t kStageOff = (kExactOff + kConsumerWarps * kMaxCands * sizeof(ExactStats) + 127) / 128 * 128;
+static_assert(kStages * 2 * sizeof(uint64_t) <= kQueueOff, "barriers overlap the queues");
+
+__device__ __forceinline__ Queue *queue_of(uint32_t warp) {
+  return reinterpret_cast<Queue *>(cmp_smem + kQueueOff) + warp;
+}
+__device__ __forceinline__ ExactStats *exact_of(uint32_t warp) {
+  return reinterpret_cast<ExactStats *>(cmp_smem + kExactOff) + warp * kMaxCands;
+}
 
 // 0.5 (1 - 2^-20): below this fraction of |r|, c - r is exact in fp32.
 #define ASMV_HALF_LESS 0x1.fffff8p-2f
@@ -266,189 +331,239 @@ __device__ __forceinline__ void settle_chunk(const QEntry &e, Hot &h, const TolF
   }
 }
 
-// Drain the warp's queue: lanes take chunks in turn; then every lane
-// adopts the warp's largest exact relative error (only the overall maximum
-// matters, so a shared threshold is as valid as a per-lane one).
-template <uint32_t DT>
-__device__ __noinline__ Hot drain(Queue *q, Hot h, const TolF t) {
-  __syncwarp();
-  const uint32_t n = min(q->count, kQueue);
-  for (uint32_t j = threadIdx.x & 31; j < n; j += 32) settle_chunk<DT>(q->e[j], h, t);
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) q->count = 0;
-  unsigned long long rb = h.drel;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) rb = umax64(rb, __shfl_xor_sync(0xFFFFFFFFu, rb, o));
-  if (rb > h.drel) { h.drel = rb; h.T = tfloor(__longlong_as_double((long long)rb)); }
-  __syncwarp();
-  return h;
-}
-
-// A chunk that found the queue full is settled in its own lane.
-template <uint32_t DT>
-__device__ __noinline__ Hot settle_overflow(const QEntry e, Hot h, const TolF t) {
-  settle_chunk<DT>(e, h, t);
-  return h;
-}
-
-// Queue one chunk.
-template <uint32_t DT>
-__device__ __forceinline__ void push_chunk(const uint4 &R, const uint4 &C, unsigned long long e0,
-                                           Queue *q, Hot &h, const TolF &t) {
-  const uint32_t slot = atomicAdd(&q->count, 1u);
-  QEntry e;
-  e.R = R; e.C = C; e.e0 = e0;
-  if (slot < kQueue) q->e[slot] = e;
-  else h = settle_overflow<DT>(e, h, t);
-}
-
-// Screen of one element whose difference s is exact when it matters.
-// Returns the definite-mismatch bit; sets `rare` when the element needs the
-// exact path; accumulates the chunk's largest |s|.
-__device__ __forceinline__ uint32_t screen(float r, float s, float Tp, const TolF &t, bool &rare,
-                                          float &cm) {
-  const float as = fabsf(s), ar = fabsf(r);
-  const float lo = __fmaf_rn(t.rlo, ar, t.alo);
-  const float hi = __fmaf_rn(t.rhi, ar, t.ahi);
-  const float y = __fmul_rd(Tp, ar);
-  const bool ok = as < lo;
-  const bool bad = as > hi;
-  rare |= (!(ok | bad)) | (as > y);
-  cm = fmaxf(cm, as);
-  return bad ? 1u : 0u;
-}
-
-__device__ __forceinline__ float2 ffma2_rd(float2 a, float2 b, float2 c) {
-  unsigned long long d;
-  asm("fma.rm.f32x2 %0, %1, %2, %3;"
-      : "=l"(d)
-      : "l"(*reinterpret_cast<unsigned long long *>(&a)), "l"(*reinterpret_cast<unsigned long long *>(&b)),
-        "l"(*reinterpret_cast<unsigned long long *>(&c)));
-  return *reinterpret_cast<float2 *>(&d);
-}
-
-// screen() of the two elements of a pair, their three bounds formed by
-// packed fp32 multiply-adds (each lane rounded exactly as the scalar one).
-// Returns the definite-mismatch bits (element 0 in bit 0).
-__device__ __forceinline__ uint32_t screen2(float2 r, float2 s, float Tp, const TolF &t, bool &rare,
-                                           float &cm) {
-  const float2 ar = make_float2(fabsf(r.x), fabsf(r.y));
-  const float2 lo = __ffma2_rn(make_float2(t.rlo, t.rlo), ar, make_float2(t.alo, t.alo));
-  const float2 hi = __ffma2_rn(make_float2(t.rhi, t.rhi), ar, make_float2(t.ahi, t.ahi));
-  const float2 y = ffma2_rd(make_float2(Tp, Tp), ar, make_float2(0.0f, 0.0f));   // RD32(Tp*|r|)
-  const float a0 = fabsf(s.x), a1 = fabsf(s.y);
-  const bool ok0 = a0 < lo.x, bad0 = a0 > hi.x, ok1 = a1 < lo.y, bad1 = a1 > hi.y;
-  rare |= (!(ok0 | bad0)) | (a0 > y.x) | (!(ok1 | bad1)) | (a1 > y.y);
-  cm = fmaxf(cm, fmaxf(a0, a1));
-  return (bad0 ? 1u : 0u) | (bad1 ? 2u : 0u);
-}
-
-// One 16-byte chunk whose first element has index e0.
-//  - Equal chunks cost one comparison.
-//  - 16- and 8-bit floats subtract in their own format (one packed
-//    instruction per pair): the result is exact whenever |c-r| < |r|/2
-//    (Sterbenz), and every other element fails |s| < Tp*|r| <= |r|/2.
-//  - A packed s*0 accumulation turns any NaN or Inf into a NaN sentinel.
-//  - A chunk with any element the screen cannot settle is queued whole.
-template <uint32_t DT>
-__device__ __forceinline__ void chunk(const uint4 &R, const uint4 &C, uint64_t e0, Hot &h,
-                                      const TolF &t, Queue *q) {
-  if (R.x == C.x && R.y == C.y && R.z == C.z && R.w == C.w) return;
-  if (is_int_dt<DT>() || DT == kF64) {
-    push_chunk<DT>(R, C, e0, q, h, t);          // integer and binary64 differences are evaluated exactly
-    return;
-  }
-  const float Tp = fminf(h.T, ASMV_HALF_LESS);
-  bool rare = false;
-  float cm = 0.0f;
-  uint32_t bad = 0;
-  if (DT == kF32) {
-    float acc = 0.0f;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-      const float r = __uint_as_float(word_of(R, w)), c = __uint_as_float(word_of(C, w));
-      const float s = __fsub_rn(c, r);
-      acc = __fmaf_rn(s, 0.0f, acc);
-      bad |= screen(r, s, Tp, t, rare, cm) << w;
-    }
-    rare |= !(acc == 0.0f);
-  } else if (DT == kBF16) {
-    __nv_bfloat162 acc = __float2bfloat162_rn(0.0f);
-    const __nv_bfloat162 zero = acc;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-      const uint32_t rw = word_of(R, w), cw = word_of(C, w);
-      const __nv_bfloat162 s2 = __hsub2(*reinterpret_cast<const __nv_bfloat162 *>(&cw),
-                                        *reinterpret_cast<const __nv_bfloat162 *>(&rw));
-      acc = __hfma2(s2, zero, acc);
-      const uint32_t sw = *reinterpret_cast<const uint32_t *>(&s2);
-      bad |= screen2(make_float2(__uint_as_float(rw << 16), __uint_as_float(rw & 0xFFFF0000u)),
-                     make_float2(__uint_as_float(sw << 16), __uint_as_float(sw & 0xFFFF0000u)), Tp, t,
-                     rare, cm) << (2 * w);
-    }
-    const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
-    rare |= (aw & 0x7FFF7FFFu) != 0u;
-  } else {
-    // fp16, and fp8 widened to fp16 (exact)
-    __half2 acc = __float2half2_rn(0.0f);
-    const __half2 zero = acc;
-    constexpr int WORDS = (DT == kF16) ? 4 : 8;        // half2 pairs per chunk
-#pragma unroll
-    for (int w = 0; w < WORDS; ++w) {
-      uint32_t rw, cw;
-      if (DT == kF16) { rw = word_of(R, w); cw = word_of(C, w); }
-      else {
-        rw = fp8x2_to_half2_bits<DT>(word_of(R, w >> 1) >> (16 * (w & 1)));
-        cw = fp8x2_to_half2_bits<DT>(word_of(C, w >> 1) >> (16 * (w & 1)));
-      }
-      const __half2 s2 = __hsub2(*reinterpret_cast<const __half2 *>(&cw),
-                                 *reinterpret_cast<const __half2 *>(&rw));
-      acc = __hfma2(s2, zero, acc);
-      bad |= screen2(f16x2_to_f32(rw), __half22float2(s2), Tp, t, rare, cm) << (2 * w);
-    }
-    const uint32_t aw = *reinterpret_cast<const uint32_t *>(&acc);
-    rare |= (aw & 0x7FFF7FFFu) != 0u;
-  }
-  if (rare) {
-    push_chunk<DT>(R, C, e0, q, h, t);
-    return;
-  }
-  h.m32 = fmaxf(h.m32, cm);
-  if (bad) {
-    h.cnt += __popc(bad);
-    h.first = umin64(h.first, e0 + (uint64_t)(__ffs(bad) - 1));
-  }
-}
-
 __device__ __forceinline__ void reset_hot(Hot &h) {
   h.cnt = 0; h.nonfin = 0; h.first = ~0ull;
   h.m32 = 0.0f; h.T = 0.0f; h.dabs = 0; h.drel = 0;
 }
 
-// Merge a warp's statistics for region `ri`, candidate k into the global
-// entry with order-independent atomics; then reset.
-__device__ __forceinline__ void flush(Hot &h, const CmpParams &p, uint32_t k, uint32_t ri) {
-  unsigned long long cnt = h.cnt, nonfin = h.nonfin;
-  unsigned long long first = h.first;
-  unsigned long long ab = umax64(h.dabs, dbits((double)h.m32));
-  unsigned long long rb = h.drel;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
-    nonfin += __shfl_xor_sync(0xFFFFFFFFu, nonfin, o);
-    first = umin64(first, __shfl_xor_sync(0xFFFFFFFFu, first, o));
-    ab = umax64(ab, __shfl_xor_sync(0xFFFFFFFFu, ab, o));
-    rb = umax64(rb, __shfl_xor_sync(0xFFFFFFFFu, rb, o));
-  }
-  if ((threadIdx.x & 31) == 0) {
-    StatsDev *st = p.stats + (size_t)k * p.nregions + ri;
-    if (cnt) atomicAdd(&st->mismatches, cnt);
-    if (nonfin) atomicAdd(&st->nonfinite, nonfin);
-    if (first != ~0ull) atomicMin(&st->first, first);
-    if (ab) atomicMax(&st->abs_bits, ab);
-    if (rb) atomicMax(&st->rel_bits, rb);
-  }
+
+// Settle one queued chunk exactly and merge its statistics into the warp's
+// entry of its candidate.  The exact path's relative-error threshold is the
+// entry's current maximum (any value not above the maximum is valid).
+template <uint32_t DT>
+__device__ __forceinline__ void settle_into(const QEntry &e, ExactStats *ex, const TolF &t) {
+  ExactStats &x = ex[e.k];
+  Hot h;
   reset_hot(h);
+  h.T = tfloor(__longlong_as_double((long long)x.drel));
+  settle_chunk<DT>(e, h, t);
+  if (h.cnt) atomicAdd(&x.cnt, h.cnt);
+  if (h.nonfin) atomicAdd(&x.nonfin, h.nonfin);
+  if (h.first != ~0ull) atomicMin(&x.first, h.first);
+  if (h.m32 > 0.0f) atomicMax(&x.m32, __float_as_uint(h.m32));
+  if (h.dabs) atomicMax(&x.dabs, h.dabs);
+  if (h.drel) atomicMax(&x.drel, h.drel);
+}
+
+template <uint32_t DT> __device__ __forceinline__ uint32_t rel_threshold(unsigned long long drel);
+
+// Drain the warp's queue: lanes take chunks in turn; then the screen's
+// thresholds of the K candidates follow their new maxima.
+template <uint32_t DT>
+__device__ __forceinline__ void drain(uint32_t warp, uint32_t K, const TolF *tp) {
+  Queue *q = queue_of(warp);
+  ExactStats *ex = exact_of(warp);
+  const TolF t = *tp;
+  __syncwarp();
+  const uint32_t n = min(q->count, kQueue), lane = threadIdx.x & 31;
+  for (uint32_t j = lane; j < n; j += 32) settle_into<DT>(q->e[j], ex, t);
+  __syncwarp();
+  if (lane == 0) q->count = 0;
+  if (lane < K) ex[lane].th = rel_threshold<DT>(ex[lane].drel);
+  __syncwarp();
+}
+
+// Queue a chunk of candidate k; false if the queue is full (the caller
+// drains it and tries again).
+__device__ __forceinline__ bool try_push(const uint4 &R, const uint4 &C, unsigned long long e0, uint32_t k,
+                                         Queue *q) {
+  const uint32_t slot = atomicAdd(&q->count, 1u);
+  if (slot >= kQueue) return false;
+  QEntry e;
+  e.R = R; e.C = C; e.e0 = e0; e.k = k; e.pad_ = 0u;
+  q->e[slot] = e;
+  return true;
+}
+
+// ---------------------------------------------------------------- screens
+// Which screen a dtype takes: packed in the stored format (fp16, the fp8
+// formats through fp16, bf16), scalar fp32, or none (integers, opaque
+// bytes and binary64 chunks that differ always take the exact path).
+template <uint32_t DT> __device__ __forceinline__ constexpr bool packed_dt() {
+  return DT == kF16 || DT == kBF16 || is_fp8(DT);
+}
+template <uint32_t DT> __device__ __forceinline__ constexpr int pairs_of() {
+  return is_fp8(DT) ? 8 : 4;               // packed words per chunk
+}
+
+// One packed word in the screen's format (fp16 for fp16 and fp8, bf16).
+template <uint32_t DT> struct P2 { using T = __half2; };
+template <> struct P2<kBF16> { using T = __nv_bfloat162; };
+
+template <class T> __device__ __forceinline__ T as2(uint32_t w) { return *reinterpret_cast<const T *>(&w); }
+template <class T> __device__ __forceinline__ uint32_t bits2(T v) { return *reinterpret_cast<const uint32_t *>(&v); }
+
+// Packed word p of a chunk in the screen's format: fp16 and bf16 words as
+// stored, fp8 bytes 2p, 2p+1 widened to their exact fp16 values.
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t word2(const uint4 &v, int p) {
+  if (is_fp8(DT)) return fp8x2_to_half2_bits<DT>(word_of(v, p >> 1) >> (16 * (p & 1)));
+  return word_of(v, p);
+}
+
+// The screen's per-candidate threshold from the warp's exact maximum of the
+// relative error: Tp = min(RD32(max), 1/2-) as a float (fp32 screen), or
+// T' = RD(Tp (1 - m)) in the packed format, in both halves (see (6)).
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t rel_threshold(unsigned long long drel) {
+  const float Tp = fminf(tfloor(__longlong_as_double((long long)drel)), ASMV_HALF_LESS);
+  if (DT == kBF16) {
+    const uint32_t h = __bfloat16_as_ushort(__float2bfloat16_rd(__fmul_rd(Tp, 1.0f - 0x1p-7f)));
+    return h | (h << 16);
+  }
+  if (packed_dt<DT>()) {
+    const uint32_t h = __half_as_ushort(__float2half_rd(__fmul_rd(Tp, 1.0f - 0x1p-9f)));
+    return h | (h << 16);
+  }
+  return __float_as_uint(Tp);
+}
+
+// A lane's screen statistics of one candidate (its threshold is warp-wide,
+// in ExactStats::th).
+struct Cand {
+  uint32_t cnt;        // mismatches the screen settled
+  uint32_t cm;         // running maximum of |c - r| over settled elements: packed bits, or float bits
+};
+
+// Two non-negative floats rounded toward zero (= down) to the screen's
+// format; x in the low half.
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t rz_pack(float2 v) {
+  uint32_t d;
+  if (DT == kBF16) asm("cvt.rz.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(v.y), "f"(v.x));
+  else asm("cvt.rz.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(v.y), "f"(v.x));
+  return d;
+}
+
+// A packed word of the screen's format as two exact floats.
+template <uint32_t DT>
+__device__ __forceinline__ float2 widen2(uint32_t w) {
+  if (DT == kBF16) return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+  return f16x2_to_f32(w);
+}
+
+// The reference side of a chunk, formed once for all candidates.
+template <uint32_t DT> struct RefPrep {
+  static constexpr int NP = pairs_of<DT>();
+  uint32_t r[NP], ar[NP], lo[NP], hi[NP];  // packed: r, |r|, lo, hi; fp32: floats (NP = 4)
+};
+
+// The fp32 bounds' constants, held in registers by the checking loop.
+struct Bounds {
+  float rlo, alo, rhi, ahi;
+};
+
+template <uint32_t DT>
+__device__ __forceinline__ void prepare(const uint4 &R, const Bounds &b, RefPrep<DT> &P) {
+  if (packed_dt<DT>()) {
+    using T2 = typename P2<DT>::T;
+    const T2 zero = as2<T2>(0u);
+#pragma unroll
+    for (int p = 0; p < RefPrep<DT>::NP; ++p) {
+      P.r[p] = word2<DT>(R, p);
+      // |r|, or NaN where r is not finite (|r| * 0 + |r|), so that y = 0 there
+      const T2 ar0 = __habs2(as2<T2>(P.r[p]));
+      P.ar[p] = bits2(__hfma2(ar0, zero, ar0));
+      const float2 f = widen2<DT>(bits2(ar0));
+      const float2 lo = make_float2(__fmaf_rn(b.rlo, f.x, b.alo), __fmaf_rn(b.rlo, f.y, b.alo));
+      const float2 hi = make_float2(__fmaf_rn(b.rhi, f.x, b.ahi), __fmaf_rn(b.rhi, f.y, b.ahi));
+      P.lo[p] = bits2(__hmax2(as2<T2>(rz_pack<DT>(lo)), zero));
+      P.hi[p] = rz_pack<DT>(hi);
+    }
+  } else {
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float r = __uint_as_float(word_of(R, w)), ar = __fmaf_rn(fabsf(r), 0.0f, fabsf(r));
+      P.r[w] = __float_as_uint(r);
+      P.ar[w] = __float_as_uint(ar);
+      P.lo[w] = __float_as_uint(__fmaf_rn(b.rlo, ar, b.alo));
+      P.hi[w] = __float_as_uint(__fmaf_rn(b.rhi, ar, b.ahi));
+    }
+  }
+}
+
+// Screen one candidate chunk C against the prepared reference chunk.
+// Returns true when the chunk needs the exact path; otherwise `bad` holds
+// its definite mismatches (packed screens: bit p for element 2p, bit 16 + p
+// for element 2p + 1; fp32: bit w for element w) and the lane's running
+// maximum of |c - r| takes the chunk's.
+template <uint32_t DT>
+__device__ __forceinline__ bool screen_chunk(const RefPrep<DT> &P, const uint4 &C, uint32_t thr, Cand &cd,
+                                             uint32_t &bad) {
+  uint32_t rare = 0, b = 0;
+  if (packed_dt<DT>()) {
+    using T2 = typename P2<DT>::T;
+    const T2 zero = as2<T2>(0u);
+    const T2 negtiny = as2<T2>(0x80018001u);               // -(least subnormal), both halves
+    const T2 th = as2<T2>(thr);
+    T2 cmc = zero;
+#pragma unroll
+    for (int p = 0; p < RefPrep<DT>::NP; ++p) {
+      const T2 s = __hsub2(as2<T2>(word2<DT>(C, p)), as2<T2>(P.r[p]));
+      const T2 a = __habs2(s);
+      const T2 y = __hmax2(__hfma2(th, as2<T2>(P.ar[p]), negtiny), zero);
+      const uint32_t mlo = __hgt2_mask(a, as2<T2>(P.lo[p]));
+      const uint32_t mhi = __hgt2_mask(a, as2<T2>(P.hi[p]));
+      const uint32_t my = __hgtu2_mask(a, y);              // unordered: NaN is flagged
+      rare |= my | (mlo & ~mhi);
+      b |= mhi & (0x00010001u << p);
+      cmc = __hmax2(cmc, a);
+    }
+    if (rare) return true;
+    cd.cm = bits2(__hmax2(as2<T2>(cd.cm), cmc));
+  } else {
+    const float Tp = __uint_as_float(thr);
+    float cmc = 0.0f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float s = __fsub_rn(__uint_as_float(word_of(C, w)), __uint_as_float(P.r[w]));
+      const float as = fabsf(s), ar = __uint_as_float(P.ar[w]);
+      const bool ok = as < __uint_as_float(P.lo[w]);
+      const bool bd = as > __uint_as_float(P.hi[w]);
+      rare |= (uint32_t)((!(ok | bd)) | (as > __fmul_rd(Tp, ar)));
+      b |= (bd ? 1u : 0u) << w;
+      cmc = fmaxf(cmc, as);
+    }
+    if (rare) return true;
+    cd.cm = __float_as_uint(fmaxf(__uint_as_float(cd.cm), cmc));
+  }
+  bad = b;
+  return false;
+}
+
+// The lowest element of a chunk's mismatch bits (see screen_chunk).
+template <uint32_t DT>
+__device__ __forceinline__ uint32_t first_of(uint32_t bad) {
+  if (packed_dt<DT>()) {
+    const uint32_t ev = __ffs(bad & 0xFFFFu), od = __ffs(bad >> 16);      // 1-based, 0 if none
+    const uint32_t e = ev ? 2u * (ev - 1u) : 64u, o = od ? 2u * (od - 1u) + 1u : 64u;
+    return min(e, o);
+  }
+  return __ffs(bad) - 1u;
+}
+
+// The value of a lane's running maximum (packed: the larger half).
+template <uint32_t DT>
+__device__ __forceinline__ float cm_value(uint32_t cm) {
+  if (DT == kBF16) {
+    const float2 f = __bfloat1622float2(as2<__nv_bfloat162>(cm));
+    return fmaxf(f.x, f.y);
+  }
+  if (packed_dt<DT>()) {
+    const float2 f = __half22float2(as2<__half2>(cm));
+    return fmaxf(f.x, f.y);
+  }
+  return __uint_as_float(cm);
 }
 
 __device__ __forceinline__ uint4 load_chunk(uint64_t base, uint64_t c, uint64_t full, uint64_t bytes,
@@ -516,107 +631,174 @@ struct Cursor {
   uint32_t ok;         // every wait succeeded
 };
 
-// The last rows of a short tile: lanes past its end are predicated off and
-// chunks beyond the staged part come from global memory.
-template <uint32_t DT>
-__device__ __noinline__ Hot tail_rows(const CmpRegion r, uint64_t cbase, const TileInfo ti,
-                                      const uint4 *sref, const uint4 *scand, uint32_t row,
-                                      uint32_t stride, Hot h, const TolF tol, Queue *q) {
+// One lane's chunk i of a tile against every candidate.  STAGED: the
+// reference and every candidate chunk are in the stage (the common case);
+// otherwise (the short last chunk of a region, or a region not 16-byte
+// aligned) they are read from device memory.  Chunks the screen cannot
+// settle are queued; bit k of `retry` is set where the queue was full.
+template <uint32_t DT, int KMAX, bool STAGED>
+__device__ __forceinline__ void check_chunk(const CmpParams &p, uint32_t ri, const CmpRegion &r,
+                                            const uint4 *stage, uint32_t tbc, uint64_t c, uint32_t K,
+                                            const Bounds &bnd, Queue *q, ExactStats *ex,
+                                            Cand (&cs)[KMAX], uint32_t &found, uint32_t &retry) {
   constexpr int E = Fmt<DT>::E;
-  const uint32_t lane = threadIdx.x & 31;
-  const uint64_t c0 = ti.off >> 4, full_chunks = r.bytes >> 4;
-  for (; row < ti.nloc; row += stride) {
-    const uint32_t i = row + lane;
-    if (i < ti.nloc) {
-      uint4 R, C;
-      if (i < ti.nsm) { R = sref[i]; C = scand[i]; }
-      else {
-        R = load_chunk(r.ref, c0 + i, full_chunks, r.bytes, false);
-        C = load_chunk(cbase, c0 + i, full_chunks, r.bytes, false);
+  const uint64_t full_chunks = r.bytes >> 4;
+  const uint4 R = STAGED ? stage[0] : load_chunk(r.ref, c, full_chunks, r.bytes, false);
+  RefPrep<DT> P;
+  if (!is_int_dt<DT>() && DT != kF64) prepare<DT>(R, bnd, P);
+#pragma unroll
+  for (int k = 0; k < KMAX; ++k) {
+    if (k >= (int)K) break;
+    const uint4 C = STAGED ? stage[(1 + k) * tbc]
+                           : load_chunk(p.cands[(size_t)k * p.nregions + ri], c, full_chunks, r.bytes, false);
+    if (((R.x ^ C.x) | (R.y ^ C.y) | (R.z ^ C.z) | (R.w ^ C.w)) == 0u) continue;
+    uint32_t bad = 0;
+    if (is_int_dt<DT>() || DT == kF64 || screen_chunk<DT>(P, C, ex[k].th, cs[k], bad)) {
+      if (!try_push(R, C, c * E, (uint32_t)k, q)) retry |= 1u << k;
+    } else if (bad) {
+      cs[k].cnt += __popc(bad);
+      if (!((found >> k) & 1u)) {
+        found |= 1u << k;
+        atomicMin(&ex[k].first, c * E + first_of<DT>(bad));
       }
-      chunk<DT>(R, C, (c0 + i) * E, h, tol, q);
     }
-    __syncwarp();
-    if (q->count >= kQueue / 2) h = drain<DT>(q, h, tol);
   }
-  return h;
 }
 
-// A warp's share of the tiles [t, t_end) of one region for its candidate:
-// for every tile, wait for its stage, check chunks part*32 + lane + j*32*W
-// (staged chunks from shared memory, the rest from global), release the
-// stage.  One call per run of tiles keeps the per-tile cost to the waits.
-// NST is the launch's pipeline depth (stage u % NST, phase (u / NST) & 1).
-template <uint32_t DT, uint32_t NST>
-__device__ __noinline__ Hot run(const CmpRegion r, uint64_t cbase, uint64_t t, uint64_t t_end,
-                                const unsigned char *bufs, uint32_t stage_bytes, uint32_t cand_off,
-                                uint64_t *full, uint64_t *empty, uint32_t tile_bytes, uint32_t part,
-                                uint32_t W, bool active, Hot h, const TolF tol, Queue *q,
-                                Cursor *cur) {
+// Chunks that found the queue full (bit k of `retry`: candidate k): drain
+// the queue and queue them again, re-read from the stage (`staged`) or from
+// device memory; every round queues at least min(32, what is left).
+// Warp-wide.
+template <uint32_t DT>
+__device__ __forceinline__ void requeue(const CmpParams &p, uint32_t ri, const uint4 *stage, uint32_t tbc,
+                                     uint64_t c, bool staged, uint32_t retry, uint32_t warp, uint32_t K,
+                                     const TolF *tol) {
   constexpr int E = Fmt<DT>::E;
-  constexpr int U = 2;
-  const uint32_t stride = 32 * W;
-  const uint32_t lane = threadIdx.x & 31;
+  Queue *q = queue_of(warp);
+  const CmpRegion r = p.regions[ri];
+  const uint64_t full_chunks = r.bytes >> 4;
+  while (__any_sync(0xFFFFFFFFu, retry)) {
+    drain<DT>(warp, K, tol);
+    while (retry) {
+      const uint32_t k = __ffs(retry) - 1;
+      const uint4 R = staged ? stage[0] : load_chunk(r.ref, c, full_chunks, r.bytes, false);
+      const uint4 C = staged ? stage[(size_t)(1 + k) * tbc]
+                             : load_chunk(p.cands[(size_t)k * p.nregions + ri], c, full_chunks, r.bytes, false);
+      if (!try_push(R, C, c * E, k, q)) break;
+      retry &= retry - 1;
+    }
+    __syncwarp();
+  }
+}
+
+// A warp's share of the tiles [t, t_end) of region ri, every candidate:
+// for every tile, wait for its stage, check rows warp, warp + 15, ... of 32
+// chunks, release the stage; then merge the region's statistics.  NST is
+// the launch's pipeline depth (stage u % NST, phase (u / NST) & 1), KMAX
+// the most candidates the instance checks.
+template <uint32_t DT, uint32_t NST, int KMAX>
+__device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, uint64_t t_end,
+                                 uint32_t warp, Cursor *cur) {
+  constexpr int E = Fmt<DT>::E;
+  const CmpRegion r = p.regions[ri];
+  const uint32_t K = p.K, TB = p.tile_bytes, lane = threadIdx.x & 31;
+  const uint32_t stage_bytes = (1 + K) * TB, tbc = TB >> 4;
+  uint64_t *full = reinterpret_cast<uint64_t *>(cmp_smem);
+  uint64_t *empty = full + kStages;
+  Queue *q = queue_of(warp);
+  ExactStats *ex = exact_of(warp);
+  const TolF *tol = &p.tol[is_int_dt<DT>() ? 0 : DT];
+  Bounds bnd;
+  bnd.rlo = tol->rlo; bnd.alo = tol->alo; bnd.rhi = tol->rhi; bnd.ahi = tol->ahi;
+  if (lane < K) {
+    ExactStats &x = ex[lane];
+    x.first = ~0ull; x.dabs = 0; x.drel = 0; x.cnt = 0; x.nonfin = 0; x.m32 = 0;
+    x.th = rel_threshold<DT>(0ull);
+  }
+  __syncwarp();
+  Cand cs[KMAX];
+#pragma unroll
+  for (int k = 0; k < KMAX; ++k) {
+    cs[k].cnt = 0u; cs[k].cm = 0u;
+  }
+  uint32_t found = 0;                      // bit k: this lane's first mismatch for k is recorded
   uint32_t u = cur->u;
   for (; t < t_end; ++t, ++u) {
     const uint32_t s = u % NST;
     if (!mbar_wait(smem_addr(&full[s]), (u / NST) & 1u, kWaitRounds)) { cur->ok = 0; break; }
-    if (active) {
-      const TileInfo ti = tile_info(r, t, tile_bytes);
-      const uint4 *sref = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes);
-      const uint4 *scand = reinterpret_cast<const uint4 *>(bufs + (size_t)s * stage_bytes + cand_off);
-      const uint64_t c0 = ti.off >> 4;
-      // Rows of U*32*W chunks; every loop bound below is the same for all
-      // lanes of the warp, so the warp-wide __syncwarp and drain are reached
-      // by every lane.  Whole rows come from shared memory; the last rows of
-      // a short tile go through the predicated tail.
-      uint32_t row = part * 32;
-      for (; row + (U - 1) * stride + 31 < ti.nsm; row += U * stride) {
-        uint4 R[U], C[U];
-#pragma unroll
-        for (int k = 0; k < U; ++k) {
-          R[k] = sref[row + lane + k * stride];
-          C[k] = scand[row + lane + k * stride];
-        }
-#pragma unroll
-        for (int k = 0; k < U; ++k) chunk<DT>(R[k], C[k], (c0 + row + lane + k * stride) * E, h, tol, q);
-        __syncwarp();
-        if (q->count >= kQueue / 2) h = drain<DT>(q, h, tol);
+    const TileInfo ti = tile_info(r, t, TB);
+    const uint4 *stage = reinterpret_cast<const uint4 *>(cmp_smem + kStageOff + (size_t)s * stage_bytes);
+    const uint64_t c0 = ti.off >> 4;
+    const bool all_staged = ti.nsm == ti.nloc;
+    // every bound below is the same for all lanes of the warp, so the
+    // warp-wide __syncwarp and drain are reached by every lane
+    for (uint32_t row = warp * 32; row < ti.nloc; row += 32 * kConsumerWarps) {
+      const uint32_t i = row + lane;
+      uint32_t retry = 0;                  // bit k: candidate k's chunk found the queue full
+      if (i < ti.nloc) {
+        if (all_staged)
+          check_chunk<DT, KMAX, true>(p, ri, r, stage + i, tbc, c0 + i, K, bnd, q, ex, cs, found, retry);
+        else
+          check_chunk<DT, KMAX, false>(p, ri, r, stage + i, tbc, c0 + i, K, bnd, q, ex, cs, found, retry);
       }
-      if (row < ti.nloc) h = tail_rows<DT>(r, cbase, ti, sref, scand, row, stride, h, tol, q);
       __syncwarp();
-      if (q->count) h = drain<DT>(q, h, tol);
+      if (__any_sync(0xFFFFFFFFu, retry))
+        requeue<DT>(p, ri, stage + i, tbc, c0 + i, i < ti.nsm, retry, warp, K, tol);
+      if (q->count >= kQueue / 2) drain<DT>(warp, K, tol);
     }
+    // queued entries are copies, so the stage is released at once
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
   }
   cur->u = u;
-  return h;
+  if (!cur->ok) return;
+  __syncwarp();
+  if (q->count) drain<DT>(warp, K, tol);
+  // merge the region's statistics of every candidate into its global entry
+#pragma unroll
+  for (int k = 0; k < KMAX; ++k) {
+    if (k >= (int)K) break;
+    unsigned long long cnt = cs[k].cnt;
+    float m = cm_value<DT>(cs[k].cm);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
+      m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    }
+    if (lane == 0) {
+      const ExactStats &x = ex[k];
+      StatsDev *st = p.stats + (size_t)k * p.nregions + ri;
+      cnt += x.cnt;
+      const unsigned long long ab =
+          umax64(x.dabs, umax64(dbits((double)m), dbits((double)__uint_as_float(x.m32))));
+      if (cnt) atomicAdd(&st->mismatches, cnt);
+      if (x.nonfin) atomicAdd(&st->nonfinite, (unsigned long long)x.nonfin);
+      if (x.first != ~0ull) atomicMin(&st->first, x.first);
+      if (ab) atomicMax(&st->abs_bits, ab);
+      if (x.drel) atomicMax(&st->rel_bits, x.drel);
+    }
+  }
+  __syncwarp();
 }
 
-template <uint32_t NST>
-__device__ __forceinline__ Hot run_dispatch(const CmpParams &p, const CmpRegion &r, uint64_t cbase,
-                                            uint64_t t, uint64_t t_end, const unsigned char *bufs,
-                                            uint32_t stage_bytes, uint32_t cand_off, uint64_t *full,
-                                            uint64_t *empty, uint32_t part, uint32_t W, bool active,
-                                            Hot h, Queue *q, Cursor *cur) {
-  const uint32_t TB = p.tile_bytes;
-#define ASMV_RUN(DT, TOL) run<DT, NST>(r, cbase, t, t_end, bufs, stage_bytes, cand_off, full, empty, TB, \
-                                  part, W, active, h, TOL, q, cur)
-  switch (r.dtype) {
-    case kF32: return ASMV_RUN(kF32, p.tol[kF32]);
-    case kBF16: return ASMV_RUN(kBF16, p.tol[kBF16]);
-    case kF16: return ASMV_RUN(kF16, p.tol[kF16]);
-    case kF8: return ASMV_RUN(kF8, p.tol[kF8]);
-    case kI32: return ASMV_RUN(kI32, p.tol[0]);
-    case kI8: return ASMV_RUN(kI8, p.tol[0]);
-    case kF8E5M2: return ASMV_RUN(kF8E5M2, p.tol[kF8E5M2]);
-    case kF8E4FNUZ: return ASMV_RUN(kF8E4FNUZ, p.tol[kF8E4FNUZ]);
-    case kF8E5FNUZ: return ASMV_RUN(kF8E5FNUZ, p.tol[kF8E5FNUZ]);
-    case kF64: return ASMV_RUN(kF64, p.tol[kF64]);
-    case kI16: return ASMV_RUN(kI16, p.tol[0]);
-    case kI64: return ASMV_RUN(kI64, p.tol[0]);
-    default: return ASMV_RUN(kU8, p.tol[0]);
+template <uint32_t NST, int KMAX>
+__device__ __forceinline__ void run_dispatch(const CmpParams &p, uint32_t ri, uint64_t t, uint64_t t_end,
+                                             uint32_t warp, Cursor *cur) {
+#define ASMV_RUN(DT) run<DT, NST, KMAX>(p, ri, t, t_end, warp, cur)
+  switch (p.regions[ri].dtype) {
+    case kF32: ASMV_RUN(kF32); break;
+    case kBF16: ASMV_RUN(kBF16); break;
+    case kF16: ASMV_RUN(kF16); break;
+    case kF8: ASMV_RUN(kF8); break;
+    case kI32: ASMV_RUN(kI32); break;
+    case kI8: ASMV_RUN(kI8); break;
+    case kF8E5M2: ASMV_RUN(kF8E5M2); break;
+    case kF8E4FNUZ: ASMV_RUN(kF8E4FNUZ); break;
+    case kF8E5FNUZ: ASMV_RUN(kF8E5FNUZ); break;
+    case kF64: ASMV_RUN(kF64); break;
+    case kI16: ASMV_RUN(kI16); break;
+    case kI64: ASMV_RUN(kI64); break;
+    default: ASMV_RUN(kU8); break;
   }
 #undef ASMV_RUN
 }
@@ -654,18 +836,16 @@ __device__ void guard_phase(const CmpParams &p, uint32_t warp, uint32_t nwarps) 
 // holds the reference tile and the K candidate tiles (tile_bytes each);
 // full[s] completes when its bulk copies land, empty[s] when every
 // consumer warp has finished with it.
-template <uint32_t NST>
-__global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams p) {
-  extern __shared__ __align__(128) unsigned char smem[];
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem);
+template <uint32_t NST, int KMAX>
+__global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_constant__ CmpParams p) {
+  uint64_t *full = reinterpret_cast<uint64_t *>(cmp_smem);
   uint64_t *empty = full + kStages;
-  constexpr uint32_t nst = NST;                              // pipeline depth, 2 or 4
-  Queue *queues = reinterpret_cast<Queue *>(smem + 128);
-  unsigned char *bufs = smem + 128 + kConsumerWarps * sizeof(Queue);
+  constexpr uint32_t nst = NST;                              // pipeline depth, 2 to 4
+  unsigned char *bufs = cmp_smem + kStageOff;
   const uint32_t K = p.K, TB = p.tile_bytes;
   const uint32_t stage_bytes = (1 + K) * TB;
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x < kConsumerWarps) queues[threadIdx.x].count = 0;
+  if (threadIdx.x < kConsumerWarps) queue_of(threadIdx.x)->count = 0;
   if (threadIdx.x == 0) {
     for (uint32_t s = 0; s < nst; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
@@ -711,11 +891,6 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
     }
   } else if (t0 < t1) {
     // consumers: one call per run of tiles of the same region
-    const uint32_t W = kConsumerWarps / K;                  // warps per candidate
-    const bool active = warp < W * K;
-    const uint32_t k = warp % K, part = warp / K;
-    Hot h;
-    reset_hot(h);
     Cursor cur;
     cur.u = 0;
     cur.ok = 1;
@@ -724,12 +899,8 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
     while (t < t1 && cur.ok) {
       while (p.regions[ri + 1].tile0 <= t) ++ri;
       const uint64_t t_end = umin64(t1, p.regions[ri + 1].tile0);
-      const CmpRegion r = p.regions[ri];
-      const uint64_t cbase = p.cands[(size_t)k * p.nregions + ri];
-      h = run_dispatch<NST>(p, r, cbase, t, t_end, bufs, stage_bytes, (1 + k) * TB, full, empty,
-                            part, W, active, h, &queues[warp], &cur);
+      run_dispatch<NST, KMAX>(p, ri, t, t_end, warp, &cur);
       t = t_end;
-      if (active && cur.ok) flush(h, p, k, ri);
     }
     if (!cur.ok && lane == 0) atomicOr(p.err, 1u);
   }
@@ -739,28 +910,21 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const CmpParams
 }  // namespace
 
 size_t compare_smem_bytes(uint32_t K, uint32_t tile_bytes, uint32_t nstages) {
-  return 128 + kConsumerWarps * sizeof(Queue) + (size_t)nstages * (1 + K) * tile_bytes;
+  return kStageOff + (size_t)nstages * (1 + K) * tile_bytes;
 }
 
-// Tiles of a launch group of up to K candidates: 16 KiB for one candidate,
-// 8 KiB otherwise, over as many stages as fit (compare_stages).  Larger
-// tiles mean fewer per-tile waits and less bookkeeping per chunk.  On a
-// 1 GiB fp16 reference (GB/s of reference + candidates read):
-//   K            2     3     4     5     6     7     8
-//   before    3051  2911  2582  2265  2654  2768  3051   (4 KiB tiles from K = 4, 4 stages)
-//   now       3137  2960  3302  3053  3118  3194  3530   (stages: 4 4 4 3 2 2 2)
-// and with one candidate, 4 stages of 16 KiB beat 2 stages by a fifth.
-// Tiles of whole warp rows (no tail rows) were measured too: better at
-// K = 2, worse at K = 3 and 5.
+// Tiles of a launch group of up to K candidates: two rows of 32 chunks per
+// checking warp for one candidate (15 KiB), one row otherwise (7.5 KiB),
+// over as many stages as fit (compare_stages).  Whole rows per warp keep
+// the warps of a stage equally loaded.
+static_assert(kConsumerWarps == 15, "tile sizes are whole rows of the checking warps");
 uint32_t compare_tile_bytes(uint32_t K) {
-  return K <= 1 ? 16384u : 8192u;
+  return K <= 1 ? 15360u : 7680u;
 }
 
 // The deepest pipeline (4, 3, else 2 stages) within kCmpSmemBudget of shared
 // memory.  The budget stays below the 227 KiB a CTA may take: the rest of
-// the SM's 256 KiB is L1, which holds the checking warps' spilled registers
-// (about 100 bytes a thread), and deeper pipelines that squeezed it were
-// slower (K = 5 at 4 stages and 217 KiB: 2348 GB/s against 3089 at 2 stages).
+// the SM's 256 KiB is L1, which holds the checking warps' spilled registers.
 constexpr size_t kCmpSmemBudget = 192 * 1024;
 uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
   for (uint32_t n = 4; n > 2; --n)
@@ -768,10 +932,20 @@ uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
   return 2u;
 }
 
-// The dynamic shared memory limit of both instances, raised once per device
+namespace {
+// The kernel instance of a launch: pipeline depth, and whether a warp
+// checks one candidate or up to kMaxCands.
+using CmpKernel = void (*)(const CmpParams);
+CmpKernel compare_instance(uint32_t nstages, uint32_t K) {
+  if (K <= 1) return nstages == 2 ? compare_kernel<2, 1> : nstages == 3 ? compare_kernel<3, 1>
+                                                                         : compare_kernel<4, 1>;
+  return nstages == 2 ? compare_kernel<2, kMaxCands> : nstages == 3 ? compare_kernel<3, kMaxCands>
+                                                                     : compare_kernel<4, kMaxCands>;
+}
+
+// The dynamic shared memory limit of every instance, raised once per device
 // to the most any launch uses (a per-launch call would add its host latency
 // to every compare).  0: not yet, 1: done; a failure is returned every time.
-namespace {
 constexpr int kMaxDevices = 64;
 std::atomic<int> g_smem_set[kMaxDevices];
 std::mutex g_smem_mutex;
@@ -784,13 +958,11 @@ int prepare_compare(size_t smem) {
   if (g_smem_set[dev].load(std::memory_order_acquire)) return (int)cudaSuccess;
   std::lock_guard<std::mutex> lock(g_smem_mutex);
   if (g_smem_set[dev].load(std::memory_order_relaxed)) return (int)cudaSuccess;
-  if ((e = cudaFuncSetAttribute(compare_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)kMaxSmemPerCta)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(compare_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)kMaxSmemPerCta)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(compare_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)kMaxSmemPerCta)) != cudaSuccess)
-    return (int)e;
+  for (uint32_t n = 2; n <= 4; ++n)
+    for (uint32_t k : {1u, 2u})
+      if ((e = cudaFuncSetAttribute(compare_instance(n, k), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kMaxSmemPerCta)) != cudaSuccess)
+        return (int)e;
   g_smem_set[dev].store(1, std::memory_order_release);
   return (int)cudaSuccess;
 }
@@ -800,8 +972,7 @@ int launch_compare(const CmpParams &p, int grid, void *stream) {
   const size_t smem = compare_smem_bytes(p.K, p.tile_bytes, p.nstages);
   const int rc = prepare_compare(smem);
   if (rc != (int)cudaSuccess) return rc;
-  auto kern = p.nstages == 2 ? compare_kernel<2> : p.nstages == 3 ? compare_kernel<3> : compare_kernel<4>;
-  kern<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
+  compare_instance(p.nstages, p.K)<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }
 

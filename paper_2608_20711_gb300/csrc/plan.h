@@ -28,7 +28,7 @@ constexpr int kTileChunks = 1024;
 constexpr uint64_t kTileBytes = (uint64_t)kChunkBytes * kTileChunks;  // 16 KiB
 constexpr uint32_t kGuardSegBytes = 4096;
 constexpr int kMaxCands = 8;            // candidates per batched launch
-constexpr int kConsumerWarps = 16;      // compare: checking warps per CTA
+constexpr int kConsumerWarps = 15;      // compare: checking warps per CTA (+ 1 feeding: 128 registers each)
 constexpr int kStages = 4;              // compare: deepest shared-memory pipeline (2 to 4 stages per launch)
 constexpr size_t kMaxSmemPerCta = 232448;   // GB300: 227 KiB of shared memory per CTA (opt-in)
 constexpr int kCmpThreads = (kConsumerWarps + 1) * 32;   // + one producer warp

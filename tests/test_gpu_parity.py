@@ -280,11 +280,11 @@ def test_compare_subnormal_differences(ctx, oracle, dtype):
 @pytest.mark.parametrize("k", [1, 8])
 def test_partial_tiles_of_every_shape(ctx, oracle, k):
     """Region sizes that leave the last tile of each region at every
-    fraction of a tile, for the single (16 KiB tiles) and the batched
-    (4 KiB tiles) launch; dense differences keep the exact-path queue busy."""
+    fraction of a tile, for the single (15 KiB tiles) and the batched
+    (7.5 KiB tiles) launch; dense differences keep the exact-path queue busy."""
     rng = np.random.default_rng(100 + k)
     regs = []
-    tile = TILE if k == 1 else 4096
+    tile = 15360 if k == 1 else 7680
     for i, frac in enumerate(np.linspace(0.02, 0.98, 23)):
         dt = ["f16", "bf16", "f32", "f8e4m3", "i8"][i % 5]
         nb = tile * int(rng.integers(1, 4)) + int(frac * tile) + int(rng.integers(0, 16))
