@@ -653,6 +653,19 @@ def run_e2e(setup, args, device, world, barrier):
 
     for _ in range(2):
         e2e_step()
+    # the same host-to-device copies alone: the link's rate for these buffers
+    torch.cuda.synchronize(device)
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    h2d_ms = []
+    for _ in range(2):
+        c0.record(copy_stream)
+        with torch.cuda.stream(copy_stream):
+            for d, h in pairs:
+                d.copy_(h, non_blocking=True)
+        c1.record(copy_stream)
+        c1.synchronize()
+        h2d_ms.append(c0.elapsed_time(c1))
+    h2d_s = min(h2d_ms) / 1e3
     barrier()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -665,6 +678,7 @@ def run_e2e(setup, args, device, world, barrier):
     return {"value": round(world * step_bytes * args.steps / el / 1e9, 1), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "ms_per_step": round(el / args.steps * 1e3, 3),
+            "h2d_gbs": round(h2d / h2d_s / 1e9, 1), "h2d_ms": round(h2d_s * 1e3, 3),
             "overlap": "host-to-device copies on a copy stream, concurrent with the fill"}
 
 
