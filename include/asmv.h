@@ -456,13 +456,25 @@ int asmv_abi_version(void);
  * its reserved address space left untouched, and one that times candidate
  * kernels cannot take the device-wide synchronisation an allocation may
  * bring; neither can create a context, whose workspace and staging are
- * allocated.  This call needs no context and allocates nothing: the launch
- * plan and the statistics live in a file-scope device array of
- * ASMV_NOALLOC_SCRATCH_BYTES that every GPU loading this library holds
- * until the process exits, staged through a static host buffer.
- *   - Runs on the calling thread's current CUDA device.  The first call on
- *     a device looks up that device's address of the array (and the SM
- *     count); make that first call before any stream capture.
+ * allocated.  This call needs no context, and once the library's device
+ * code is loaded on a device it allocates nothing: the launch plan and the
+ * statistics live in a file-scope device array of
+ * ASMV_NOALLOC_SCRATCH_BYTES, staged through a static host buffer.
+ *   - Loading.  With lazy module loading (the CUDA default) the library's
+ *     device code, and this array with it, is placed in device memory the
+ *     first time the context uses it, so the first call on a device (or any
+ *     earlier call of this library on it) does allocate.  A caller that
+ *     reserves or replays fixed addresses must make one call of its own
+ *     (an empty table, n = 0 with valid tolerances, does not load; use a
+ *     one-region table) before it reserves them.  The array then stays in
+ *     the context until the context is destroyed.
+ *   - Runs on the calling thread's current CUDA device.  Every call looks
+ *     up the array's address in the current context (this allocates
+ *     nothing), so a context that was reset and created again is handled.
+ *   - Stream capture: the call copies its plan from pageable host memory
+ *     and synchronises its stream, both of which are illegal while a stream
+ *     is being captured.  It must not be called while its stream, or any
+ *     other stream, is being captured.
  *   - ref/cand/n/tol/out_host/stream as asmv_compare (one candidate).
  *   - The plan must fit the scratch: regions (32 B each, plus one), one
  *     candidate address (8 B) and one statistics entry (64 B) per region,

@@ -281,6 +281,14 @@ def _stream_handle(stream) -> Optional[int]:
     return int(stream)
 
 
+def _same_lengths(ref: Sequence, cands: Sequence[Sequence]):
+    """The C calls read as many candidate regions as there are reference
+    regions: a shorter candidate table would be read past its end."""
+    for j, c in enumerate(cands):
+        if len(c) != len(ref):
+            raise ValueError("candidate %d has %d regions, the reference %d" % (j, len(c), len(ref)))
+
+
 class Context:
     """One asmv context on one CUDA device (not thread-safe)."""
 
@@ -346,6 +354,7 @@ class Context:
         return stats_dicts(out, len(regions))
 
     def compare(self, ref: Sequence, cand: Sequence, tol, stream=None) -> List[dict]:
+        _same_lengths(ref, [cand])
         ra, ca = region_array(ref), region_array(cand)
         out = (Stats * max(1, len(ref)))()
         self._check(self._lib.asmv_compare(self._h, ra, ca, len(ref), tol_array(tol)
@@ -355,6 +364,7 @@ class Context:
 
     def compare_batched(self, ref: Sequence, cands: Sequence[Sequence], tol,
                         stream=None) -> List[List[dict]]:
+        _same_lengths(ref, cands)
         n, k = len(ref), len(cands)
         ra = region_array(ref)
         cas = [region_array(c) for c in cands]
@@ -385,6 +395,7 @@ class Context:
                    tau: float = TAU, stream=None):
         """asmv_compare_eq: (stats, eq) with stats[j][i] as compare_batched
         and eq[j][i] the Eq. 1 terms of candidate j on region i."""
+        _same_lengths(ref, cands)
         n, k = len(ref), len(cands)
         ra = region_array(ref)
         cas = [region_array(c) for c in cands]
@@ -407,6 +418,7 @@ class Context:
         (int64, shape (n, 1 + 2k, D), D = EQ_DIGITS, or EQ64_DIGITS when a
         region is binary64): the per-shard result of a check split across
         processes (see eq_from_digits)."""
+        _same_lengths(ref, cands)
         n, k = len(ref), len(cands)
         ra = region_array(ref)
         nd = digits_per_slot([ra[i].dtype for i in range(n)])
@@ -570,7 +582,9 @@ def compare_noalloc(ref: Sequence, cand: Sequence, tol, stream=None) -> List[dic
     """asmv_compare_noalloc: the check of one candidate on the current CUDA
     device, for callers that must not allocate device memory (no context;
     the plan and statistics live in the library's fixed device scratch).
-    Raises AsmvError on a non-OK status."""
+    Raises AsmvError on a non-OK status, ValueError when the candidate's
+    table is not as long as the reference's."""
+    _same_lengths(ref, [cand])
     L = lib()
     ra, ca = region_array(ref), region_array(cand)
     out = (Stats * max(1, len(ref)))()

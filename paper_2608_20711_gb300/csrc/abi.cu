@@ -20,6 +20,7 @@
 #include "asmv.h"
 #include "plan.h"
 #include "eq64.h"
+#include "nvtx_range.h"
 
 using namespace asmv;
 
@@ -562,6 +563,7 @@ int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds) {
 
 int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed,
               asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_fill");
   if (ctx == nullptr) return ASMV_EINVAL;
   int rc = check_table(regions, n, true);
   if (rc != ASMV_OK) return rc;
@@ -736,6 +738,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
 
 int asmv_guard_check(asmv_ctx *ctx, const asmv_region *regions, size_t n, asmv_stats *out_host,
                      asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_guard_check");
   if (ctx == nullptr || (n > 0 && out_host == nullptr)) return ASMV_EINVAL;
   int rc = check_table(regions, n, false);
   if (rc != ASMV_OK) return rc;
@@ -760,6 +763,7 @@ static int check_pairs(const asmv_region *ref, const asmv_region *const *cands, 
 
 int asmv_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cand, size_t n,
                  const asmv_tol *tol, asmv_stats *out_host, asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_compare");
   if (ctx == nullptr || (n > 0 && (out_host == nullptr || cand == nullptr)) || !tol_ok(tol))
     return ASMV_EINVAL;
   const asmv_region *cands[1] = {cand};
@@ -774,6 +778,7 @@ int asmv_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cand,
 int asmv_compare_batched(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
                          size_t k, size_t n, const asmv_tol *tol, asmv_stats *out_host,
                          asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_compare_batched");
   if (ctx == nullptr || k == 0 || cands == nullptr || (n > 0 && out_host == nullptr) || !tol_ok(tol))
     return ASMV_EINVAL;
   if (k > (size_t)0x7FFFFFFF / (n ? n : 1)) return ASMV_EINVAL;
@@ -1030,6 +1035,7 @@ extern "C" {
 int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
                     size_t k, size_t n, const asmv_tol *tol, double theta, double tau,
                     asmv_stats *stats_host, asmv_eq *eq_host, asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_compare_eq");
   int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, eq_host);
   if (rc != ASMV_OK) return rc;
   if (!theta_tau_ok(theta, tau)) return ASMV_EINVAL;
@@ -1052,6 +1058,7 @@ int asmv_compare_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *co
 int asmv_compare_eq_digits(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *const *cands,
                            size_t k, size_t n, const asmv_tol *tol, asmv_stats *stats_host,
                            int64_t *digits_host, asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_compare_eq_digits");
   int rc = check_eq_call(ctx, ref, cands, k, n, tol, stats_host, digits_host);
   if (rc != ASMV_OK) return rc;
   if (n == 0) return ASMV_OK;
@@ -1219,11 +1226,13 @@ static int run_copy(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *a
 
 int asmv_restore(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *src, size_t n,
                  asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_restore");
   return run_copy(ctx, regions, src, n, stream, true);
 }
 
 int asmv_capture(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *dst, size_t n,
                  asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_capture");
   return run_copy(ctx, regions, dst, n, stream, false);
 }
 
@@ -1256,8 +1265,7 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 namespace {
 
 alignas(256) unsigned char g_noalloc_host[kNoAllocBytes];   // host image of the same layout
-unsigned char *g_noalloc_dev[kNoAllocMaxDevices];            // scratch address per device
-int g_noalloc_sms[kNoAllocMaxDevices];
+int g_noalloc_sms[kNoAllocMaxDevices];                       // SM count per device (0: not yet read)
 AddrRangeFn g_noalloc_range = nullptr;
 bool g_noalloc_range_looked_up = false;
 std::mutex g_noalloc_mutex;
@@ -1265,13 +1273,17 @@ std::mutex g_noalloc_mutex;
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // Set-up for the current device (under the mutex): the device address of
-// the scratch array, the SM count and the address-range lookup.
-int noalloc_setup(int dev) {
+// the scratch array in the current context, the SM count and the
+// address-range lookup.  The address is looked up on every call, not kept:
+// a context that was reset and created again loads the module anew, and the
+// array may then sit elsewhere (the lookup allocates nothing).
+int noalloc_setup(int dev, unsigned char **scratch) {
   if (dev < 0 || dev >= kNoAllocMaxDevices) return ASMV_EINVAL;
-  if (g_noalloc_dev[dev]) return ASMV_OK;
   void *p = nullptr;
   cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess || p == nullptr) { cudaGetLastError(); return ASMV_ECUDA; }
+  *scratch = (unsigned char *)p;
+  if (g_noalloc_sms[dev]) return ASMV_OK;
   int sms = 0;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
     cudaGetLastError();
@@ -1288,13 +1300,15 @@ int noalloc_setup(int dev) {
     g_noalloc_range_looked_up = true;
   }
   g_noalloc_sms[dev] = sms;
-  g_noalloc_dev[dev] = (unsigned char *)p;
   return ASMV_OK;
 }
 
 // Device-memory check of one allocation on the current device (no context).
-int noalloc_check_span(int dev, uint64_t alloc, uint64_t total) {
+// `last` is the allocation range the previous region was found in: a region
+// inside it needs no driver query.
+int noalloc_check_span(int dev, uint64_t alloc, uint64_t total, std::pair<uint64_t, uint64_t> &last) {
   if (total == 0) return ASMV_OK;
+  if (alloc >= last.first && alloc + total <= last.second) return ASMV_OK;
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, (const void *)alloc) != cudaSuccess) {
     cudaGetLastError();
@@ -1310,6 +1324,7 @@ int noalloc_check_span(int dev, uint64_t alloc, uint64_t total) {
     size_t size = 0;
     if (g_noalloc_range(&base, &size, alloc) != 0) return ASMV_EINVAL;
     if (alloc + total > base + size) return ASMV_EINVAL;
+    last = std::make_pair((uint64_t)base, (uint64_t)(base + size));
   }
   return ASMV_OK;
 }
@@ -1347,6 +1362,7 @@ size_t noalloc_put_guards(GuardSeg *out, const asmv_region &r, uint8_t kind, uin
 extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *cand, size_t n,
                                     const asmv_tol *tol, asmv_stats *out_host,
                                     asmv_stream_t stream) {
+  ASMV_NVTX_RANGE("asmv_compare_noalloc");
   if ((n > 0 && (out_host == nullptr || cand == nullptr)) || !tol_ok(tol)) return ASMV_EINVAL;
   int rc = check_table(ref, n, false);
   if (rc != ASMV_OK) return rc;
@@ -1369,13 +1385,15 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   std::lock_guard<std::mutex> lock(g_noalloc_mutex);
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return ASMV_ECUDA; }
-  if ((rc = noalloc_setup(dev)) != ASMV_OK) return rc;
+  unsigned char *dscr = nullptr;
+  if ((rc = noalloc_setup(dev, &dscr)) != ASMV_OK) return rc;
+  std::pair<uint64_t, uint64_t> last_ref(0, 0), last_cand(0, 0);
   for (size_t i = 0; i < n; ++i) {
     uint64_t pb, tot;
     region_extent(ref[i], &pb, &tot);
-    if ((rc = noalloc_check_span(dev, ref[i].alloc, tot)) != ASMV_OK) return rc;
+    if ((rc = noalloc_check_span(dev, ref[i].alloc, tot, last_ref)) != ASMV_OK) return rc;
     region_extent(cand[i], &pb, &tot);
-    if ((rc = noalloc_check_span(dev, cand[i].alloc, tot)) != ASMV_OK) return rc;
+    if ((rc = noalloc_check_span(dev, cand[i].alloc, tot, last_cand)) != ASMV_OK) return rc;
   }
 
   const uint32_t tile_bytes = compare_tile_bytes(1);
@@ -1405,7 +1423,6 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   cr[n].tile0 = tile;
   std::memset(&st[n], 0, sizeof(StatsDev));          // the error word starts at zero
 
-  unsigned char *dscr = g_noalloc_dev[dev];
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e = cudaMemcpyAsync(dscr, g_noalloc_host, total, cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return ASMV_ECUDA;

@@ -9,6 +9,7 @@
 #include <cuda_runtime.h>
 
 #include "asmv.h"
+#include "nvtx_range.h"
 
 namespace {
 
@@ -60,6 +61,7 @@ int asmv_commit_gate(int all_eq, double s_cand, double s_best, double cv,
 
 int asmv_time_launches(asmv_launch_fn fn, void *user, int warmup, size_t r,
                        double *samples_ms, asmv_stream_t stream, int *cuda_error) {
+  ASMV_NVTX_RANGE("asmv_time_launches");
   if (fn == nullptr || samples_ms == nullptr || r == 0 || warmup < 0) return ASMV_EINVAL;
   const cudaStream_t s = (cudaStream_t)stream;
   std::vector<cudaEvent_t> ev(2 * r, nullptr);

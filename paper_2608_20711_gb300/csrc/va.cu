@@ -15,6 +15,7 @@
 #include <cuda_runtime.h>
 
 #include "asmv.h"
+#include "nvtx_range.h"
 
 struct asmv_va {
   int device;
@@ -108,6 +109,7 @@ int asmv_va_granularity(int device, size_t *out) {
 }
 
 int asmv_va_map(int device, uint64_t addr, size_t bytes, asmv_va **out) {
+  ASMV_NVTX_RANGE("asmv_va_map");
   if (out == nullptr || bytes == 0) return ASMV_EINVAL;
   int prev;
   if (!enter_device(device, &prev)) return ASMV_ECUDA;
@@ -160,6 +162,7 @@ uint64_t asmv_va_address(const asmv_va *va) { return va ? (uint64_t)va->addr : 0
 size_t asmv_va_size(const asmv_va *va) { return va ? va->size : 0; }
 
 int asmv_va_unmap(asmv_va *va) {
+  ASMV_NVTX_RANGE("asmv_va_unmap");
   if (va == nullptr) return ASMV_EINVAL;
   int prev;
   if (!enter_device(va->device, &prev)) return ASMV_ECUDA;

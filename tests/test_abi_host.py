@@ -153,3 +153,21 @@ def test_strided_regions_cover_each_element_once():
                                                    [s // 2 * 8 for s in view.strides])
         assert covered == view_idx.ravel().tolist()
         assert len(regs) <= view.size
+
+
+def test_candidate_tables_must_match_the_reference_length():
+    """Every wrapper refuses a candidate table of another length before it
+    reaches the C call, which would read n candidate regions."""
+    ref = [asmv.make_region(0x10000, 8, "f32"), asmv.make_region(0x20000, 8, "f32")]
+    short = ref[:1]
+    with pytest.raises(ValueError):
+        asmv.compare_noalloc(ref, short, {"f32": (0.0, 0.0)})
+    ctx = asmv.Context.__new__(asmv.Context)          # no device needed: the check comes first
+    with pytest.raises(ValueError):
+        ctx.compare(ref, short, {"f32": (0.0, 0.0)})
+    with pytest.raises(ValueError):
+        ctx.compare_batched(ref, [ref, short], {"f32": (0.0, 0.0)})
+    with pytest.raises(ValueError):
+        ctx.compare_eq(ref, [short], {"f32": (0.0, 0.0)})
+    with pytest.raises(ValueError):
+        ctx.compare_eq_digits(ref, [ref + ref], {"f32": (0.0, 0.0)})
