@@ -625,9 +625,12 @@ __device__ __forceinline__ TileInfo tile_info(const CmpRegion &r, uint64_t t, ui
   return ti;
 }
 
-// Pipeline position shared by a consumer warp's calls.
+// Pipeline position shared by a consumer warp's calls: the next stage and
+// the phase its full barrier completes next (the stage index wraps at the
+// launch's depth, and the phase flips with each wrap).
 struct Cursor {
-  uint32_t u;          // stage uses consumed so far
+  uint32_t s;          // stage of the next tile
+  uint32_t ph;         // parity of its full barrier's next phase
   uint32_t ok;         // every wait succeeded
 };
 
@@ -643,15 +646,20 @@ __device__ __forceinline__ void check_chunk(const CmpParams &p, uint32_t ri, con
                                             Cand (&cs)[KMAX], uint32_t &found, uint32_t &retry) {
   constexpr int E = Fmt<DT>::E;
   const uint64_t full_chunks = r.bytes >> 4;
+  // With one candidate the reference side is prepared only for a chunk that
+  // differs (most chunks of a nearly equal candidate do not); with several,
+  // once before the candidates.
+  constexpr bool kScreened = !is_int_dt<DT>() && DT != kF64;
   const uint4 R = STAGED ? stage[0] : load_chunk(r.ref, c, full_chunks, r.bytes, false);
   RefPrep<DT> P;
-  if (!is_int_dt<DT>() && DT != kF64) prepare<DT>(R, bnd, P);
+  if (kScreened && KMAX > 1) prepare<DT>(R, bnd, P);
 #pragma unroll
   for (int k = 0; k < KMAX; ++k) {
     if (k >= (int)K) break;
     const uint4 C = STAGED ? stage[(1 + k) * tbc]
                            : load_chunk(p.cands[(size_t)k * p.nregions + ri], c, full_chunks, r.bytes, false);
     if (((R.x ^ C.x) | (R.y ^ C.y) | (R.z ^ C.z) | (R.w ^ C.w)) == 0u) continue;
+    if (kScreened && KMAX == 1) prepare<DT>(R, bnd, P);
     uint32_t bad = 0;
     if (is_int_dt<DT>() || DT == kF64 || screen_chunk<DT>(P, C, ex[k].th, cs[k], bad)) {
       if (!try_push(R, C, c * E, (uint32_t)k, q)) retry |= 1u << k;
@@ -693,10 +701,9 @@ __device__ __forceinline__ void requeue(const CmpParams &p, uint32_t ri, const u
 
 // A warp's share of the tiles [t, t_end) of region ri, every candidate:
 // for every tile, wait for its stage, check rows warp, warp + 15, ... of 32
-// chunks, release the stage; then merge the region's statistics.  NST is
-// the launch's pipeline depth (stage u % NST, phase (u / NST) & 1), KMAX
+// chunks, release the stage; then merge the region's statistics.  KMAX is
 // the most candidates the instance checks.
-template <uint32_t DT, uint32_t NST, int KMAX>
+template <uint32_t DT, int KMAX>
 __device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, uint64_t t_end,
                                  uint32_t warp, Cursor *cur) {
   constexpr int E = Fmt<DT>::E;
@@ -722,10 +729,10 @@ __device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, ui
     cs[k].cnt = 0u; cs[k].cm = 0u;
   }
   uint32_t found = 0;                      // bit k: this lane's first mismatch for k is recorded
-  uint32_t u = cur->u;
-  for (; t < t_end; ++t, ++u) {
-    const uint32_t s = u % NST;
-    if (!mbar_wait(smem_addr(&full[s]), (u / NST) & 1u, kWaitRounds)) { cur->ok = 0; break; }
+  const uint32_t nst = p.nstages;
+  uint32_t s = cur->s, ph = cur->ph;
+  for (; t < t_end; ++t) {
+    if (!mbar_wait(smem_addr(&full[s]), ph, kWaitRounds)) { cur->ok = 0; break; }
     const TileInfo ti = tile_info(r, t, TB);
     const uint4 *stage = reinterpret_cast<const uint4 *>(cmp_smem + kStageOff + (size_t)s * stage_bytes);
     const uint64_t c0 = ti.off >> 4;
@@ -749,8 +756,10 @@ __device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, ui
     // queued entries are copies, so the stage is released at once
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
+    if (++s == nst) { s = 0; ph ^= 1u; }
   }
-  cur->u = u;
+  cur->s = s;
+  cur->ph = ph;
   if (!cur->ok) return;
   __syncwarp();
   if (q->count) drain<DT>(warp, K, tol);
@@ -781,10 +790,10 @@ __device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, ui
   __syncwarp();
 }
 
-template <uint32_t NST, int KMAX>
+template <int KMAX>
 __device__ __forceinline__ void run_dispatch(const CmpParams &p, uint32_t ri, uint64_t t, uint64_t t_end,
                                              uint32_t warp, Cursor *cur) {
-#define ASMV_RUN(DT) run<DT, NST, KMAX>(p, ri, t, t_end, warp, cur)
+#define ASMV_RUN(DT) run<DT, KMAX>(p, ri, t, t_end, warp, cur)
   switch (p.regions[ri].dtype) {
     case kF32: ASMV_RUN(kF32); break;
     case kBF16: ASMV_RUN(kBF16); break;
@@ -836,11 +845,11 @@ __device__ void guard_phase(const CmpParams &p, uint32_t warp, uint32_t nwarps) 
 // holds the reference tile and the K candidate tiles (tile_bytes each);
 // full[s] completes when its bulk copies land, empty[s] when every
 // consumer warp has finished with it.
-template <uint32_t NST, int KMAX>
+template <int KMAX>
 __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_constant__ CmpParams p) {
   uint64_t *full = reinterpret_cast<uint64_t *>(cmp_smem);
   uint64_t *empty = full + kStages;
-  constexpr uint32_t nst = NST;                              // pipeline depth, 2 to 4
+  const uint32_t nst = p.nstages;                            // pipeline depth, 2 to 4
   unsigned char *bufs = cmp_smem + kStageOff;
   const uint32_t K = p.K, TB = p.tile_bytes;
   const uint32_t stage_bytes = (1 + K) * TB;
@@ -861,11 +870,10 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_co
     // producer
     if (lane == 0 && t0 < t1) {
       uint32_t ri = find_region(p.regions, p.nregions, t0);
-      uint32_t u = 0;
+      uint32_t u = 0, s = 0, ph = 0;       // tiles issued; stage and phase of the next
       for (uint64_t t = t0; t < t1 && ok; ++t, ++u) {
         while (p.regions[ri + 1].tile0 <= t) ++ri;
-        const uint32_t s = u % nst;
-        if (u >= nst && !mbar_wait(smem_addr(&empty[s]), ((u / nst) & 1u) ^ 1u, p.wait_rounds)) {
+        if (u >= nst && !mbar_wait(smem_addr(&empty[s]), ph ^ 1u, p.wait_rounds)) {
           ok = false;
           break;
         }
@@ -880,6 +888,7 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_co
           for (uint32_t k = 0; k < K; ++k)
             bulk_load(dst + (1 + k) * TB, p.cands[(size_t)k * p.nregions + ri] + ti.off, nb, fb);
         }
+        if (++s == nst) { s = 0; ph ^= 1u; }
       }
       if (!ok) atomicOr(p.err, 1u);
       // Let every copy issued land before the CTA can exit: consumers that
@@ -892,14 +901,15 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_co
   } else if (t0 < t1) {
     // consumers: one call per run of tiles of the same region
     Cursor cur;
-    cur.u = 0;
+    cur.s = 0;
+    cur.ph = 0;
     cur.ok = 1;
     uint32_t ri = find_region(p.regions, p.nregions, t0);
     uint64_t t = t0;
     while (t < t1 && cur.ok) {
       while (p.regions[ri + 1].tile0 <= t) ++ri;
       const uint64_t t_end = umin64(t1, p.regions[ri + 1].tile0);
-      run_dispatch<NST, KMAX>(p, ri, t, t_end, warp, &cur);
+      run_dispatch<KMAX>(p, ri, t, t_end, warp, &cur);
       t = t_end;
     }
     if (!cur.ok && lane == 0) atomicOr(p.err, 1u);
@@ -933,14 +943,11 @@ uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
 }
 
 namespace {
-// The kernel instance of a launch: pipeline depth, and whether a warp
-// checks one candidate or up to kMaxCands.
+// The kernel instance of a launch: whether a warp checks one candidate or
+// up to kMaxCands (the pipeline depth is a launch parameter).
 using CmpKernel = void (*)(const CmpParams);
-CmpKernel compare_instance(uint32_t nstages, uint32_t K) {
-  if (K <= 1) return nstages == 2 ? compare_kernel<2, 1> : nstages == 3 ? compare_kernel<3, 1>
-                                                                         : compare_kernel<4, 1>;
-  return nstages == 2 ? compare_kernel<2, kMaxCands> : nstages == 3 ? compare_kernel<3, kMaxCands>
-                                                                     : compare_kernel<4, kMaxCands>;
+CmpKernel compare_instance(uint32_t K) {
+  return K <= 1 ? compare_kernel<1> : compare_kernel<kMaxCands>;
 }
 
 // The dynamic shared memory limit of every instance, raised once per device
@@ -958,21 +965,21 @@ int prepare_compare(size_t smem) {
   if (g_smem_set[dev].load(std::memory_order_acquire)) return (int)cudaSuccess;
   std::lock_guard<std::mutex> lock(g_smem_mutex);
   if (g_smem_set[dev].load(std::memory_order_relaxed)) return (int)cudaSuccess;
-  for (uint32_t n = 2; n <= 4; ++n)
-    for (uint32_t k : {1u, 2u})
-      if ((e = cudaFuncSetAttribute(compare_instance(n, k), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)kMaxSmemPerCta)) != cudaSuccess)
-        return (int)e;
+  for (uint32_t k : {1u, 2u})
+    if ((e = cudaFuncSetAttribute(compare_instance(k), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)kMaxSmemPerCta)) != cudaSuccess)
+      return (int)e;
   g_smem_set[dev].store(1, std::memory_order_release);
   return (int)cudaSuccess;
 }
 }  // namespace
 
 int launch_compare(const CmpParams &p, int grid, void *stream) {
+  if (p.nstages < 2 || p.nstages > (uint32_t)kStages) return (int)cudaErrorInvalidValue;
   const size_t smem = compare_smem_bytes(p.K, p.tile_bytes, p.nstages);
   const int rc = prepare_compare(smem);
   if (rc != (int)cudaSuccess) return rc;
-  compare_instance(p.nstages, p.K)<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
+  compare_instance(p.K)<<<grid, kCmpThreads, smem, (cudaStream_t)stream>>>(p);
   return (int)cudaGetLastError();
 }
 

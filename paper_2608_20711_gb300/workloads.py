@@ -227,6 +227,7 @@ WORKLOADS = {
                                                      input_bytes=1 << 30, input_regions=8),
     "batched_gemm_fp16_4kx16k": lambda: batched_gemm(rows=4096, cols=16384,
                                                      input_bytes=512 << 20, input_regions=4),
+    "snapshot_4096_1g": lambda: snapshot(total_bytes=1 << 30),
 }
 
 
