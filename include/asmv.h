@@ -164,6 +164,7 @@ typedef struct {
 #define ASMV_ECUDA (-2)     /* a CUDA runtime call failed; see asmv_ctx_cuda_error */
 #define ASMV_ETIMEOUT (-3)  /* a bounded device wait expired */
 #define ASMV_ENOMEM (-4)    /* workspace or staging allocation failed */
+#define ASMV_EBOUNDS (-5)   /* debug-bounds build only: a device access fell outside its allocation */
 
 typedef struct asmv_ctx asmv_ctx;
 
@@ -440,6 +441,28 @@ uint64_t asmv_ctx_launches(const asmv_ctx *ctx);
  * null ctx. */
 #define ASMV_WAIT_ROUNDS 20000u
 int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds);
+
+/* The debug-bounds build.  libasmv_debug.so is this library compiled with
+ * device bounds checks (ASMV_DEBUG_BOUNDS=1): every region descriptor and
+ * guard segment carries the allocation it lies in, and every global load
+ * and store of the fill, the compare (bulk copies into shared memory, the
+ * byte-granular reads of ragged chunks, the guard reads) and the restore /
+ * capture is checked against it.  An access outside is skipped, never
+ * made: the kernel sets a bit in the launch's error word and goes on, and
+ * the call returns ASMV_EBOUNDS (the fill and the restore then read the
+ * word back and synchronise their stream).  Results are otherwise those of
+ * the normal build, bit for bit.  The Eq. 1 sums kernels are not checked.
+ * asmv_debug_bounds() returns 1 in that build and 0 in the normal one. */
+int asmv_debug_bounds(void);
+
+/* Test hook of the debug-bounds build: every later asmv_fill on ctx runs its
+ * payload loop `bytes` past the end of each non-empty payload, while the
+ * allocations it checks against stay those of the table, so the checks
+ * refuse the extra stores.  A test gives the region an allocation larger
+ * than the table says, so that even an unchecked store would stay inside
+ * real memory.  0 turns it off.  ASMV_EINVAL for a null ctx, and in the
+ * normal build, where the hook does not exist. */
+int asmv_ctx_debug_widen(asmv_ctx *ctx, uint64_t bytes);
 
 /* Static description of a status code. */
 const char *asmv_strerror(int status);

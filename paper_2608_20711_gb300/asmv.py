@@ -15,7 +15,10 @@ from typing import Dict, Iterable, List, Optional, Sequence
 import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "libasmv.so")
+# ASMV_DEBUG_BOUNDS=1 in the environment loads the debug-bounds build
+# (libasmv_debug.so: every device access checked against its allocation).
+DEBUG_BOUNDS = os.environ.get("ASMV_DEBUG_BOUNDS", "0") not in ("", "0")
+LIB_PATH = os.path.join(HERE, "libasmv_debug.so" if DEBUG_BOUNDS else "libasmv.so")
 
 # asmv_dtype / asmv_dist codes
 F32, BF16, F16, F8E4M3, I32, I8, U8_OPAQUE = range(7)
@@ -27,7 +30,7 @@ DTYPE_CODE = {"f32": F32, "bf16": BF16, "f16": F16, "f8e4m3": F8E4M3, "i32": I32
               "f8e5m2fnuz": F8E5M2FNUZ, "f64": F64, "i16": I16, "i64": I64}
 DIST_CODE = {"raw": DIST_RAW, "uniform": DIST_UNIFORM, "normal": DIST_NORMAL,
              "int_range": DIST_INT_RANGE, "none": DIST_NONE}
-OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM = 0, -1, -2, -3, -4
+OK, EINVAL, ECUDA, ETIMEOUT, ENOMEM, EBOUNDS = 0, -1, -2, -3, -4, -5
 
 
 def dtype_code(dtype) -> int:
@@ -94,7 +97,8 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_timing_summary", "asmv_commit_gate", "asmv_time_launches",
                  "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
                  "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds",
-                 "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base")
+                 "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base",
+                 "asmv_debug_bounds", "asmv_ctx_debug_widen")
 EQ_DIGITS = 20                           # signed 64-bit digits per exact Eq. 1 sum
 EQ64_DIGITS = 136                        # ... when the region table holds a binary64 region
 NOALLOC_SCRATCH_BYTES = 1 << 20
@@ -117,7 +121,8 @@ def lib():
     global _lib
     if _lib is None:
         if not os.path.exists(LIB_PATH):
-            raise RuntimeError("libasmv.so is not built: run paper_2608_20711_gb300.build.build()")
+            raise RuntimeError("%s is not built: run paper_2608_20711_gb300.build.build(%s)"
+                               % (os.path.basename(LIB_PATH), "debug_bounds=True" if DEBUG_BOUNDS else ""))
         L = ctypes.CDLL(LIB_PATH)
         vp, sz = ctypes.c_void_p, ctypes.c_size_t
         RP, SP, TP = ctypes.POINTER(Region), ctypes.POINTER(Stats), ctypes.POINTER(Tol)
@@ -135,6 +140,8 @@ def lib():
         L.asmv_ctx_launches.argtypes = [vp]
         L.asmv_ctx_launches.restype = ctypes.c_uint64
         L.asmv_ctx_set_wait_rounds.argtypes = [vp, ctypes.c_uint32]
+        L.asmv_debug_bounds.argtypes = []
+        L.asmv_ctx_debug_widen.argtypes = [vp, ctypes.c_uint64]
         L.asmv_strerror.argtypes = [ctypes.c_int]
         L.asmv_strerror.restype = ctypes.c_char_p
         L.asmv_abi_version.argtypes = []
@@ -325,6 +332,12 @@ class Context:
     @property
     def launches(self) -> int:
         return int(self._lib.asmv_ctx_launches(self._h))
+
+    def debug_widen(self, nbytes: int):
+        """Test hook of the debug-bounds build (asmv_ctx_debug_widen): later
+        fills run each payload loop nbytes past its end, and the device
+        checks refuse those stores (the call returns EBOUNDS)."""
+        self._check(self._lib.asmv_ctx_debug_widen(self._h, int(nbytes)))
 
     def set_wait_rounds(self, rounds: int = None):
         """Bound of the compare pipeline's device waits (tries of up to

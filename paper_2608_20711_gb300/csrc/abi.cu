@@ -28,11 +28,13 @@ static_assert(sizeof(asmv_region) == 56, "asmv_region layout");
 static_assert(sizeof(asmv_stats) == 64, "asmv_stats layout");
 static_assert(sizeof(asmv_eq) == 40, "asmv_eq layout");
 static_assert(sizeof(StatsDev) == sizeof(asmv_stats), "device statistics layout");
-static_assert(sizeof(CopyRegion) == 48, "copy region layout");
+static_assert(sizeof(CopyRegion) == 48 + (ASMV_DEBUG_BOUNDS ? 32 : 0), "copy region layout");
 static_assert(kWaitRounds == ASMV_WAIT_ROUNDS, "default wait bound");
 static_assert(kEqDigits == ASMV_EQ_DIGITS, "Eq. 1 digits");
 static_assert(kEq64Digits == ASMV_EQ64_DIGITS, "Eq. 1 digits of binary64");
-static_assert(sizeof(FillRegion) == 64 && sizeof(CmpRegion) == 32 && sizeof(GuardSeg) == 32,
+static_assert(sizeof(FillRegion) == 64 + (ASMV_DEBUG_BOUNDS ? 16 : 0) &&
+                  sizeof(CmpRegion) == 32 + (ASMV_DEBUG_BOUNDS ? 16 : 0) &&
+                  sizeof(GuardSeg) == 32 + (ASMV_DEBUG_BOUNDS ? 16 : 0),
               "plan layouts");
 
 namespace {
@@ -151,7 +153,7 @@ TolF make_tolf(const asmv_tol &t) {
 uint64_t tiles_of(uint64_t payload_bytes) { return (payload_bytes + kTileBytes - 1) / kTileBytes; }
 
 void add_guard_segments(std::vector<GuardSeg> &segs, uint64_t ptr, uint64_t offset, uint64_t len,
-                        uint8_t canary, uint8_t kind, uint32_t stats) {
+                        uint8_t canary, uint8_t kind, uint32_t stats, uint64_t alloc, uint64_t total) {
   for (uint64_t o = 0; o < len; o += kGuardSegBytes) {
     GuardSeg g;
     std::memset(&g, 0, sizeof g);
@@ -161,6 +163,11 @@ void add_guard_segments(std::vector<GuardSeg> &segs, uint64_t ptr, uint64_t offs
     g.stats = stats;
     g.canary = canary;
     g.kind = kind;
+#if ASMV_DEBUG_BOUNDS
+    g.alloc = Span{alloc, alloc + total};
+#else
+    (void)alloc; (void)total;
+#endif
     segs.push_back(g);
   }
 }
@@ -168,10 +175,10 @@ void add_guard_segments(std::vector<GuardSeg> &segs, uint64_t ptr, uint64_t offs
 void add_region_guards(std::vector<GuardSeg> &segs, const asmv_region &r, uint8_t kind, uint32_t stats) {
   uint64_t pb, tot;
   region_extent(r, &pb, &tot);
-  if (r.guard_lo) add_guard_segments(segs, r.alloc, 0, r.guard_lo, r.canary, kind, stats);
+  if (r.guard_lo) add_guard_segments(segs, r.alloc, 0, r.guard_lo, r.canary, kind, stats, r.alloc, tot);
   if (r.guard_hi)
     add_guard_segments(segs, r.alloc + r.guard_lo + pb, (uint64_t)r.guard_lo + pb, r.guard_hi,
-                       r.canary, kind, stats);
+                       r.canary, kind, stats, r.alloc, tot);
 }
 
 StatsDev empty_stats() {
@@ -225,6 +232,7 @@ struct asmv_ctx {
   uint64_t launches = 0;
   uint32_t wait_rounds = kWaitRounds;
   AddrRangeFn addr_range = nullptr;
+  uint64_t debug_widen = 0;       // debug-bounds build: bytes added to each fill's loop bound
 };
 
 namespace {
@@ -329,6 +337,29 @@ int after_launch(asmv_ctx *ctx, cudaStream_t s) {
   return ASMV_OK;
 }
 
+// Host staging a call reserves for reading back its launch's error word:
+// only the debug-bounds build has one for the fill and the restore.
+constexpr size_t debug_err_bytes() { return ASMV_DEBUG_BOUNDS ? 256 : 0; }
+
+#if ASMV_DEBUG_BOUNDS
+// The debug-bounds build finishes a fill or restore by reading its error
+// word back (the call then synchronises its stream): ASMV_EBOUNDS if an
+// access fell outside its allocation.
+int debug_finish(asmv_ctx *ctx, size_t err_off, size_t img_bytes, cudaStream_t s) {
+  cudaError_t e;
+  unsigned char *host = ctx->hst + ((img_bytes + 255) & ~(size_t)255);
+  if ((e = cudaMemcpyAsync(host, (unsigned char *)ctx->dws + err_off, sizeof(uint32_t),
+                           cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+    return fail_cuda(ctx, e);
+  if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return fail_cuda(ctx, e);
+  ctx->staged_pending = false;
+  ctx->ws_pending = false;
+  uint32_t err;
+  std::memcpy(&err, host, sizeof err);
+  return (err & kErrBounds) ? ASMV_EBOUNDS : ASMV_OK;
+}
+#endif
+
 int grid_for(asmv_ctx *ctx, uint64_t ntiles, size_t nsegs, int ctas_per_sm) {
   const uint64_t cap = (uint64_t)ctx->sms * (uint64_t)ctas_per_sm;
   uint64_t g = std::max<uint64_t>(ntiles, (nsegs + kWarps - 1) / kWarps);
@@ -349,6 +380,7 @@ int readback(asmv_ctx *ctx, size_t stats_off, size_t img_bytes, size_t count, cu
   ctx->ws_pending = false;
   uint32_t err;
   std::memcpy(&err, host + count * sizeof(StatsDev), sizeof err);
+  if (err & kErrBounds) return ASMV_EBOUNDS;         // an access outside its allocation (debug build)
   if (err) return ASMV_ETIMEOUT;                     // a bounded device wait expired
   std::memcpy(out, host, count * sizeof(asmv_stats));
   if (ref_n) {
@@ -471,6 +503,7 @@ const char *asmv_strerror(int status) {
     case ASMV_ECUDA: return "CUDA runtime error";
     case ASMV_ETIMEOUT: return "bounded device wait expired";
     case ASMV_ENOMEM: return "out of memory (workspace or staging)";
+    case ASMV_EBOUNDS: return "a device access fell outside its allocation (debug-bounds build)";
     default: return "unknown status";
   }
 }
@@ -561,6 +594,14 @@ int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds) {
   return ASMV_OK;
 }
 
+int asmv_debug_bounds(void) { return ASMV_DEBUG_BOUNDS; }
+
+int asmv_ctx_debug_widen(asmv_ctx *ctx, uint64_t bytes) {
+  if (ctx == nullptr || !ASMV_DEBUG_BOUNDS) return ASMV_EINVAL;
+  ctx->debug_widen = bytes;
+  return ASMV_OK;
+}
+
 int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed,
               asmv_stream_t stream) {
   ASMV_NVTX_RANGE("asmv_fill");
@@ -599,6 +640,10 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
       f.ilo = (int64_t)r.p0;
       f.ispan = (uint64_t)((int64_t)r.p1 - (int64_t)r.p0);
     }
+#if ASMV_DEBUG_BOUNDS
+    f.alloc = Span{r.alloc, r.alloc + tot};
+    if (f.bytes) f.bytes += ctx->debug_widen;       // the test hook: loop past the payload
+#endif
     tile += (f.bytes + kFillTileBytes - 1) / kFillTileBytes;
     if (f.bytes != 0 && f.dist == ASMV_DIST_NORMAL) {
       const uint32_t sz = (uint32_t)kDtypeSize[r.dtype];
@@ -613,10 +658,17 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   Image img;
   const size_t o_regs = img.add(fr.data(), fr.size() * sizeof(FillRegion));
   const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
+#if ASMV_DEBUG_BOUNDS
+  const uint32_t zero = 0;
+  const size_t o_err = img.add(&zero, sizeof zero);
+#endif
   unsigned char *dev = nullptr;
   cudaStream_t s = (cudaStream_t)stream;
-  if ((rc = stage(ctx, img, 0, s, &dev)) != ASMV_OK) return rc;
+  if ((rc = stage(ctx, img, debug_err_bytes(), s, &dev)) != ASMV_OK) return rc;
   FillParams p;
+#if ASMV_DEBUG_BOUNDS
+  p.err = (uint32_t *)(dev + o_err);
+#endif
   p.regions = (const FillRegion *)(dev + o_regs);
   p.segs = (const GuardSeg *)(dev + o_segs);
   p.ntiles = tile;
@@ -638,7 +690,12 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
     if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
     ctx->timed = true;
   }
+#if ASMV_DEBUG_BOUNDS
+  if ((rc = after_launch(ctx, s)) != ASMV_OK) return rc;
+  return debug_finish(ctx, o_err, img.bytes.size(), s);
+#else
   return after_launch(ctx, s);
+#endif
 }
 
 // Shared body of guard_check / compare / compare_batched.
@@ -653,6 +710,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
 
   std::vector<CmpRegion> cr(n + 1);
   std::vector<uint64_t> caddr(guard_only ? 0 : k * n);
+  std::vector<Span> callocs(ASMV_DEBUG_BOUNDS && !guard_only ? k * n : 0);   // debug-bounds build
   std::vector<GuardSeg> segs;
   uint64_t tile = 0;
   const uint32_t tile_bytes = compare_tile_bytes((uint32_t)std::min<size_t>(std::max<size_t>(k, 1), kMaxCands));
@@ -666,11 +724,19 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
     c.bytes = guard_only ? 0 : pb;
     c.tile0 = tile;
     c.dtype = r.dtype;
+#if ASMV_DEBUG_BOUNDS
+    c.alloc = Span{r.alloc, r.alloc + tot};
+#endif
     bool vec = (c.ref % 16) == 0;
     for (size_t j = 0; j < caddr.size() / (n ? n : 1); ++j) {
       const uint64_t a = cands[j][i].alloc + cands[j][i].guard_lo;
       caddr[j * n + i] = a;
       vec = vec && (a % 16) == 0;
+      if (!callocs.empty()) {
+        uint64_t cpb, ctot;
+        region_extent(cands[j][i], &cpb, &ctot);
+        callocs[j * n + i] = Span{cands[j][i].alloc, cands[j][i].alloc + ctot};
+      }
     }
     c.vec = vec;
     tile += (c.bytes + tile_bytes - 1) / tile_bytes;
@@ -694,6 +760,8 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
   const size_t o_cand = img.add(caddr.data(), caddr.size() * sizeof(uint64_t));
   const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
   const size_t o_stats = img.add(st.data(), st.size() * sizeof(StatsDev));
+  const size_t o_callocs = img.add(callocs.data(), callocs.size() * sizeof(Span));
+  (void)o_callocs;
   unsigned char *dev = nullptr;
   if ((rc = stage(ctx, img, st.size() * sizeof(StatsDev), s, &dev)) != ASMV_OK) return rc;
 
@@ -718,6 +786,9 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
     p.K = (uint32_t)kg;
     p.nstages = compare_stages(p.K, tile_bytes);
     p.cands = (const uint64_t *)(dev + o_cand) + g * kMaxCands * n;
+#if ASMV_DEBUG_BOUNDS
+    p.cand_allocs = (const Span *)(dev + o_callocs) + g * kMaxCands * n;
+#endif
     p.stats = (StatsDev *)(dev + o_stats) + g * kMaxCands * n;
     p.nsegs = (g == 0) ? (uint32_t)segs.size() : 0u;
     if (guard_only) p.ntiles = 0;
@@ -1192,6 +1263,12 @@ static int run_copy(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *a
     c.bytes = pb;
     c.tile0 = tile;
     c.vec = (c.dst % 16 == 0) && (c.src % 16 == 0);
+#if ASMV_DEBUG_BOUNDS
+    // the region's allocation on one side, the caller's buffer [addr, addr + payload) on the other
+    const Span region_alloc{r.alloc, r.alloc + tot}, buffer{addrs[i], addrs[i] + pb};
+    c.dst_alloc = restore ? region_alloc : buffer;
+    c.src_alloc = restore ? buffer : region_alloc;
+#endif
     tile += tiles_of(pb);
     if (restore) add_region_guards(segs, r, kSegFill, (uint32_t)i);
   }
@@ -1201,11 +1278,18 @@ static int run_copy(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *a
   Image img;
   const size_t o_regs = img.add(cr.data(), cr.size() * sizeof(CopyRegion));
   const size_t o_segs = img.add(segs.data(), segs.size() * sizeof(GuardSeg));
+#if ASMV_DEBUG_BOUNDS
+  const uint32_t zero = 0;
+  const size_t o_err = img.add(&zero, sizeof zero);
+#endif
   unsigned char *dev = nullptr;
   const cudaStream_t s = (cudaStream_t)stream;
-  if ((rc = stage(ctx, img, 0, s, &dev)) != ASMV_OK) return rc;
+  if ((rc = stage(ctx, img, debug_err_bytes(), s, &dev)) != ASMV_OK) return rc;
   CopyParams p;
   std::memset(&p, 0, sizeof p);
+#if ASMV_DEBUG_BOUNDS
+  p.err = (uint32_t *)(dev + o_err);
+#endif
   p.regions = (const CopyRegion *)(dev + o_regs);
   p.segs = (const GuardSeg *)(dev + o_segs);
   p.ntiles = tile;
@@ -1221,7 +1305,12 @@ static int run_copy(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *a
     if ((e = cudaEventRecord(ctx->t1, s)) != cudaSuccess) return fail_cuda(ctx, e);
     ctx->timed = true;
   }
+#if ASMV_DEBUG_BOUNDS
+  if ((rc = after_launch(ctx, s)) != ASMV_OK) return rc;
+  return debug_finish(ctx, o_err, img.bytes.size(), s);
+#else
   return after_launch(ctx, s);
+#endif
 }
 
 int asmv_restore(asmv_ctx *ctx, const asmv_region *regions, const uint64_t *src, size_t n,
@@ -1352,6 +1441,9 @@ size_t noalloc_put_guards(GuardSeg *out, const asmv_region &r, uint8_t kind, uin
       g.stats = stats;
       g.canary = r.canary;
       g.kind = kind;
+#if ASMV_DEBUG_BOUNDS
+      g.alloc = Span{r.alloc, r.alloc + tot};
+#endif
     }
   }
   return k;
@@ -1379,7 +1471,8 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   const size_t o_cand = align256(o_regs + (n + 1) * sizeof(CmpRegion));
   const size_t o_segs = align256(o_cand + n * sizeof(uint64_t));
   const size_t o_stats = align256(o_segs + nsegs * sizeof(GuardSeg));
-  const size_t total = o_stats + (n + 1) * sizeof(StatsDev);
+  const size_t o_callocs = align256(o_stats + (n + 1) * sizeof(StatsDev));   // debug-bounds build
+  const size_t total = ASMV_DEBUG_BOUNDS ? o_callocs + n * sizeof(Span) : o_stats + (n + 1) * sizeof(StatsDev);
   if (total > kNoAllocBytes) return ASMV_EINVAL;      // beyond the fixed scratch
 
   std::lock_guard<std::mutex> lock(g_noalloc_mutex);
@@ -1413,6 +1506,14 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
     c.tile0 = tile;
     c.dtype = ref[i].dtype;
     caddr[i] = cand[i].alloc + cand[i].guard_lo;
+#if ASMV_DEBUG_BOUNDS
+    c.alloc = Span{ref[i].alloc, ref[i].alloc + tot};
+    {
+      uint64_t cpb, ctot;
+      region_extent(cand[i], &cpb, &ctot);
+      ((Span *)(g_noalloc_host + o_callocs))[i] = Span{cand[i].alloc, cand[i].alloc + ctot};
+    }
+#endif
     c.vec = (c.ref % 16) == 0 && (caddr[i] % 16) == 0;
     tile += (pb + tile_bytes - 1) / tile_bytes;
     ks += noalloc_put_guards(segs + ks, ref[i], kSegRef, (uint32_t)i);
@@ -1434,6 +1535,9 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   p.stats = (StatsDev *)(dscr + o_stats);
   p.seg_stats = p.stats;
   p.err = (uint32_t *)(p.stats + n);
+#if ASMV_DEBUG_BOUNDS
+  p.cand_allocs = (const Span *)(dscr + o_callocs);
+#endif
   p.ntiles = tile;
   p.nregions = (uint32_t)n;
   p.nsegs = (uint32_t)ks;
@@ -1453,6 +1557,7 @@ extern "C" int asmv_compare_noalloc(const asmv_region *ref, const asmv_region *c
   if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return ASMV_ECUDA;
   uint32_t err;
   std::memcpy(&err, &st[n], sizeof err);
+  if (err & kErrBounds) return ASMV_EBOUNDS;
   if (err) return ASMV_ETIMEOUT;
   std::memcpy(out_host, st, n * sizeof(asmv_stats));
   return ASMV_OK;

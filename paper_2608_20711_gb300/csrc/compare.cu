@@ -572,6 +572,19 @@ __device__ __forceinline__ uint4 load_chunk(uint64_t base, uint64_t c, uint64_t 
   return load_bytes(base + 16 * c, (uint32_t)umin64(16, bytes - 16 * c));
 }
 
+// Chunk c of region ri read from device memory: the reference (k < 0) or
+// candidate k.  In the debug-bounds build a read outside the allocation is
+// skipped (zeros) and reported.
+__device__ __forceinline__ uint4 load_region_chunk(const CmpParams &p, uint32_t ri, const CmpRegion &r, int k,
+                                                   uint64_t c) {
+  const uint64_t base = k < 0 ? r.ref : p.cands[(size_t)k * p.nregions + ri];
+#if ASMV_DEBUG_BOUNDS
+  const Span sp = k < 0 ? r.alloc : p.cand_allocs[(size_t)k * p.nregions + ri];
+  if (!in_alloc(sp, base + 16 * c, umin64(16, r.bytes - 16 * c), p.err)) return make_uint4(0u, 0u, 0u, 0u);
+#endif
+  return load_chunk(base, c, r.bytes >> 4, r.bytes, false);
+}
+
 // ---------------------------------------------------------------- pipeline
 // mbarrier helpers (shared::cta addresses).  Waits are bounded: after
 // `rounds` tries of up to kWaitHintNs each, the wait reports failure.  The
@@ -645,19 +658,17 @@ __device__ __forceinline__ void check_chunk(const CmpParams &p, uint32_t ri, con
                                             const Bounds &bnd, Queue *q, ExactStats *ex,
                                             Cand (&cs)[KMAX], uint32_t &found, uint32_t &retry) {
   constexpr int E = Fmt<DT>::E;
-  const uint64_t full_chunks = r.bytes >> 4;
   // With one candidate the reference side is prepared only for a chunk that
   // differs (most chunks of a nearly equal candidate do not); with several,
   // once before the candidates.
   constexpr bool kScreened = !is_int_dt<DT>() && DT != kF64;
-  const uint4 R = STAGED ? stage[0] : load_chunk(r.ref, c, full_chunks, r.bytes, false);
+  const uint4 R = STAGED ? stage[0] : load_region_chunk(p, ri, r, -1, c);
   RefPrep<DT> P;
   if (kScreened && KMAX > 1) prepare<DT>(R, bnd, P);
 #pragma unroll
   for (int k = 0; k < KMAX; ++k) {
     if (k >= (int)K) break;
-    const uint4 C = STAGED ? stage[(1 + k) * tbc]
-                           : load_chunk(p.cands[(size_t)k * p.nregions + ri], c, full_chunks, r.bytes, false);
+    const uint4 C = STAGED ? stage[(1 + k) * tbc] : load_region_chunk(p, ri, r, k, c);
     if (((R.x ^ C.x) | (R.y ^ C.y) | (R.z ^ C.z) | (R.w ^ C.w)) == 0u) continue;
     if (kScreened && KMAX == 1) prepare<DT>(R, bnd, P);
     uint32_t bad = 0;
@@ -684,14 +695,12 @@ __device__ __forceinline__ void requeue(const CmpParams &p, uint32_t ri, const u
   constexpr int E = Fmt<DT>::E;
   Queue *q = queue_of(warp);
   const CmpRegion r = p.regions[ri];
-  const uint64_t full_chunks = r.bytes >> 4;
   while (__any_sync(0xFFFFFFFFu, retry)) {
     drain<DT>(warp, K, tol);
     while (retry) {
       const uint32_t k = __ffs(retry) - 1;
-      const uint4 R = staged ? stage[0] : load_chunk(r.ref, c, full_chunks, r.bytes, false);
-      const uint4 C = staged ? stage[(size_t)(1 + k) * tbc]
-                             : load_chunk(p.cands[(size_t)k * p.nregions + ri], c, full_chunks, r.bytes, false);
+      const uint4 R = staged ? stage[0] : load_region_chunk(p, ri, r, -1, c);
+      const uint4 C = staged ? stage[(size_t)(1 + k) * tbc] : load_region_chunk(p, ri, r, (int)k, c);
       if (!try_push(R, C, c * E, k, q)) break;
       retry &= retry - 1;
     }
@@ -706,7 +715,6 @@ __device__ __forceinline__ void requeue(const CmpParams &p, uint32_t ri, const u
 template <uint32_t DT, int KMAX>
 __device__ __noinline__ void run(const CmpParams &p, uint32_t ri, uint64_t t, uint64_t t_end,
                                  uint32_t warp, Cursor *cur) {
-  constexpr int E = Fmt<DT>::E;
   const CmpRegion r = p.regions[ri];
   const uint32_t K = p.K, TB = p.tile_bytes, lane = threadIdx.x & 31;
   const uint32_t stage_bytes = (1 + K) * TB, tbc = TB >> 4;
@@ -819,6 +827,9 @@ __device__ void guard_phase(const CmpParams &p, uint32_t warp, uint32_t nwarps) 
   const uint64_t nw = (uint64_t)gridDim.x * nwarps;
   for (uint64_t s = gw; s < p.nsegs; s += nw) {
     const GuardSeg g = p.segs[s];
+#if ASMV_DEBUG_BOUNDS
+    if (!in_alloc(g.alloc, g.ptr, g.len, p.err)) continue;
+#endif
     const uint8_t *src = reinterpret_cast<const uint8_t *>(g.ptr);
     unsigned long long bad = 0, first = ~0ull;
     for (uint32_t j = lane; j < g.len; j += 32) {
@@ -879,8 +890,17 @@ __global__ void __launch_bounds__(kCmpThreads, 1) compare_kernel(const __grid_co
         }
         const CmpRegion r = p.regions[ri];
         const TileInfo ti = tile_info(r, t, TB);
-        const uint32_t nb = ti.nsm * 16u;
+        uint32_t nb = ti.nsm * 16u;
         const uint32_t fb = smem_addr(&full[s]);
+#if ASMV_DEBUG_BOUNDS
+        // a tile with any copy outside its allocation is not copied (its
+        // stage is left as it was; the launch reports the error)
+        bool inside = in_alloc(r.alloc, r.ref + ti.off, nb, p.err);
+        for (uint32_t k = 0; k < K; ++k)
+          inside = inside && in_alloc(p.cand_allocs[(size_t)k * p.nregions + ri],
+                                      p.cands[(size_t)k * p.nregions + ri] + ti.off, nb, p.err);
+        if (!inside) nb = 0;
+#endif
         mbar_arrive_tx(fb, nb * (1 + K));
         if (nb) {
           const uint32_t dst = smem_addr(bufs + (size_t)s * stage_bytes);

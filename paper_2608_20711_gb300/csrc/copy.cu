@@ -19,7 +19,8 @@
 namespace asmv {
 namespace {
 
-__device__ __forceinline__ void copy_tile(const CopyRegion &r, uint64_t t) {
+__device__ __forceinline__ void copy_tile(const CopyRegion &r, uint64_t t, uint32_t *err) {
+  (void)err;
   const uint64_t off = t * kTileBytes;
   const uint64_t nb = umin64(kTileBytes, r.bytes - off);
   const uint32_t nch = (uint32_t)((nb + 15) / 16);
@@ -31,6 +32,9 @@ __device__ __forceinline__ void copy_tile(const CopyRegion &r, uint64_t t) {
     if (c < nch) {
       const uint64_t a = r.src + off + 16ull * c;
       const uint32_t n = (uint32_t)umin64(16, nb - 16ull * c);
+#if ASMV_DEBUG_BOUNDS
+      if (!in_alloc(r.src_alloc, a, n, err)) { v[k] = make_uint4(0u, 0u, 0u, 0u); continue; }
+#endif
       v[k] = (r.vec && n == 16) ? ldg16(a) : load_bytes(a, n);
     }
   }
@@ -40,6 +44,9 @@ __device__ __forceinline__ void copy_tile(const CopyRegion &r, uint64_t t) {
     if (c < nch) {
       const uint64_t a = r.dst + off + 16ull * c;
       const uint32_t n = (uint32_t)umin64(16, nb - 16ull * c);
+#if ASMV_DEBUG_BOUNDS
+      if (!in_alloc(r.dst_alloc, a, n, err)) continue;
+#endif
       if (r.vec && n == 16) stg16(a, v[k]);
       else store_bytes(a, v[k], n);
     }
@@ -54,13 +61,20 @@ __global__ void __launch_bounds__(kThreads) copy_kernel(const CopyParams p) {
     for (uint64_t t = t0; t < t1; ++t) {
       while (p.regions[ri + 1].tile0 <= t) ++ri;
       const CopyRegion r = p.regions[ri];
-      copy_tile(r, t - r.tile0);
+#if ASMV_DEBUG_BOUNDS
+      copy_tile(r, t - r.tile0, p.err);
+#else
+      copy_tile(r, t - r.tile0, nullptr);
+#endif
     }
   }
   const uint32_t lane = threadIdx.x & 31;
   const uint64_t warp = b * kWarps + (threadIdx.x >> 5), nw = G * kWarps;
   for (uint64_t s = warp; s < p.nsegs; s += nw) {
     const GuardSeg g = p.segs[s];
+#if ASMV_DEBUG_BOUNDS
+    if (!in_alloc(g.alloc, g.ptr, g.len, p.err)) continue;
+#endif
     uint8_t *dst = reinterpret_cast<uint8_t *>(g.ptr);
     for (uint32_t j = lane; j < g.len; j += 32) dst[j] = g.canary;
   }

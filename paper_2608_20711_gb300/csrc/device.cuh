@@ -75,6 +75,20 @@ __device__ __forceinline__ void store_bytes(uint64_t addr, uint4 v, uint32_t n) 
     if (j < n) p[j] = (uint8_t)(w[j >> 2] >> (8 * (j & 3)));
 }
 
+// The debug-bounds build's check of an access [a, a + n) against the
+// allocation it belongs to: true when inside; otherwise it sets kErrBounds
+// in *err and the caller skips the access.  The normal build always passes.
+__device__ __forceinline__ bool in_alloc(const Span &s, uint64_t a, uint64_t n, uint32_t *err) {
+#if ASMV_DEBUG_BOUNDS
+  if (a >= s.lo && a <= s.hi && n <= s.hi - a) return true;
+  atomicOr(err, kErrBounds);
+  return false;
+#else
+  (void)s; (void)a; (void)n; (void)err;
+  return true;
+#endif
+}
+
 // Region owning tile t: the last i with tile0[i] <= t (regions with no
 // tiles share their successor's tile0 and are skipped).
 template <class R>

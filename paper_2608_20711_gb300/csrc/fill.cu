@@ -34,18 +34,24 @@ __device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
 __device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const uint8_t *tab, float v[4]) {
   float2 z0, z1;
   box_muller2(w, tab, z0, z1);
-  const float2 a = __fadd2_rn(f2(mean), __fmul2_rn(f2(sd), z0));
-  const float2 b = __fadd2_rn(f2(mean), __fmul2_rn(f2(sd), z1));
-  v[0] = a.x; v[1] = b.x; v[2] = a.y; v[3] = b.y;
+  // multiply, then add, each rounded: scalar _rn operations, which are never
+  // contracted (a packed multiply followed by a packed add was fused into
+  // one multiply-add whatever their rounding modifiers)
+  v[0] = __fadd_rn(mean, __fmul_rn(sd, z0.x));
+  v[1] = __fadd_rn(mean, __fmul_rn(sd, z1.x));
+  v[2] = __fadd_rn(mean, __fmul_rn(sd, z0.y));
+  v[3] = __fadd_rn(mean, __fmul_rn(sd, z1.y));
 }
 
 // uniform_of for the four words of a block, two per packed instruction.
 __device__ __forceinline__ void uniform4(uint4 w, float lo, float width, float v[4]) {
-  const float2 fa = __fmul2_rn(make_float2(__uint2float_rn(w.x >> 8), __uint2float_rn(w.y >> 8)), f2(0x1p-24f));
-  const float2 fb = __fmul2_rn(make_float2(__uint2float_rn(w.z >> 8), __uint2float_rn(w.w >> 8)), f2(0x1p-24f));
-  const float2 a = __fadd2_rn(f2(lo), __fmul2_rn(fa, f2(width)));
-  const float2 b = __fadd2_rn(f2(lo), __fmul2_rn(fb, f2(width)));
-  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+  const float2 fa = fmul2(make_float2(__uint2float_rn(w.x >> 8), __uint2float_rn(w.y >> 8)), f2(0x1p-24f));
+  const float2 fb = fmul2(make_float2(__uint2float_rn(w.z >> 8), __uint2float_rn(w.w >> 8)), f2(0x1p-24f));
+  // f (exact) times the width, then plus lo, each rounded (scalar _rn: never contracted)
+  v[0] = __fadd_rn(lo, __fmul_rn(fa.x, width));
+  v[1] = __fadd_rn(lo, __fmul_rn(fa.y, width));
+  v[2] = __fadd_rn(lo, __fmul_rn(fb.x, width));
+  v[3] = __fadd_rn(lo, __fmul_rn(fb.y, width));
 }
 
 // UNIFORM of the narrow formats: v = lo + (k scale) width, k a 16-bit or
@@ -66,6 +72,9 @@ struct Keys {
   uint32_t offT;            // angle table entry 0
   uint32_t offR16;          // 16-bit radius chord "entry 1776" (the bias of F' >> 19)
   uint32_t offR8;           // 8-bit radius entry 0
+#if ASMV_DEBUG_BOUNDS
+  uint32_t *err;
+#endif
 };
 
 __device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id, uint64_t b) {
@@ -182,10 +191,17 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
   return make_uint4(out[0], out[1], out[2], out[3]);
 }
 
-__device__ __forceinline__ void store_chunk(const FillRegion &r, uint64_t c, uint64_t full, uint4 v) {
+__device__ __forceinline__ void store_chunk(const FillRegion &r, const Keys &K, uint64_t c, uint64_t full,
+                                            uint4 v) {
   const uint64_t addr = r.payload + 16 * c;
+  const uint32_t n = (uint32_t)umin64(16, r.bytes - 16 * c);
+#if ASMV_DEBUG_BOUNDS
+  if (!in_alloc(r.alloc, addr, n, K.err)) return;
+#else
+  (void)K;
+#endif
   if (r.vec && c < full) stg16(addr, v);
-  else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * c));
+  else store_bytes(addr, v, n);
 }
 
 // Thread t makes chunks t + 2 k kFillThreads and t + (2 k + 1) kFillThreads
@@ -204,8 +220,8 @@ __device__ void fill_tile(const FillRegion &r, const Keys &K, uint64_t tile_in_r
     const uint64_t ca = c0 + i, cb = c0 + (two ? i2 : i);
     const uint4 va = make_chunk<DIST, DT>(r, K, ca);
     const uint4 vb = make_chunk<DIST, DT>(r, K, cb);
-    store_chunk(r, ca, full, va);
-    if (two) store_chunk(r, cb, full, vb);
+    store_chunk(r, K, ca, full, va);
+    if (two) store_chunk(r, K, cb, full, vb);
   }
 }
 
@@ -283,10 +299,13 @@ __global__ void __launch_bounds__(kFillThreads) fill_kernel(const __grid_constan
   // so regions of very different cost per tile (NORMAL against RAW) spread
   // evenly over the SMs.
   if (b < p.ntiles) {
-    const Keys K = {p.key0, p.key1, sm, sm + L.ln + 16u * (lane % kLnCopies),
-                    L.angle + 8u * (lane % kAngleCopies),
-                    L.rad16 + 8u * (lane % kRad16Copies) - 1776u * 8u * kRad16Copies,
-                    L.rad8 + 4u * (lane % kRad8Copies)};
+    Keys K = {p.key0, p.key1, sm, sm + L.ln + 16u * (lane % kLnCopies),
+              L.angle + 8u * (lane % kAngleCopies),
+              L.rad16 + 8u * (lane % kRad16Copies) - 1776u * 8u * kRad16Copies,
+              L.rad8 + 4u * (lane % kRad8Copies)};
+#if ASMV_DEBUG_BOUNDS
+    K.err = p.err;
+#endif
     uint32_t ri = find_region(p.regions, p.nregions, b);
     for (uint64_t t = b; t < p.ntiles; t += G) {
       if (p.regions[ri + 1].tile0 <= t) ri = next_region(p.regions, p.nregions, ri, t);
@@ -298,6 +317,9 @@ __global__ void __launch_bounds__(kFillThreads) fill_kernel(const __grid_constan
   const uint64_t warp = b * kFillWarps + (threadIdx.x >> 5), nw = G * kFillWarps;
   for (uint64_t s = warp; s < p.nsegs; s += nw) {
     const GuardSeg g = p.segs[s];
+#if ASMV_DEBUG_BOUNDS
+    if (!in_alloc(g.alloc, g.ptr, g.len, p.err)) continue;
+#endif
     uint8_t *dst = reinterpret_cast<uint8_t *>(g.ptr);
     for (uint32_t j = lane; j < g.len; j += 32) dst[j] = g.canary;
   }

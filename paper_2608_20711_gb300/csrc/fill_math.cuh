@@ -139,44 +139,65 @@ __device__ __forceinline__ void box_muller(uint32_t w0, uint32_t w1, const uint8
 // z0 = (z0 of pair a, z0 of pair b), z1 likewise.
 __device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
 
+// Packed multiply and add (PTX with the rounding modifier).  A packed
+// multiply whose result feeds a packed add may still be fused into one
+// multiply-add, rounding once where the specification rounds twice, so
+// they are used only where the product is exact or is not added: where the
+// specification multiplies and then adds, the scalar __fmul_rn / __fadd_rn
+// are used, which are never contracted.
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  float2 d;
+  asm("mul.rn.f32x2 %0, %1, %2;"
+      : "=l"(*reinterpret_cast<unsigned long long *>(&d))
+      : "l"(*reinterpret_cast<unsigned long long *>(&a)), "l"(*reinterpret_cast<unsigned long long *>(&b)));
+  return d;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  float2 d;
+  asm("add.rn.f32x2 %0, %1, %2;"
+      : "=l"(*reinterpret_cast<unsigned long long *>(&d))
+      : "l"(*reinterpret_cast<unsigned long long *>(&a)), "l"(*reinterpret_cast<unsigned long long *>(&b)));
+  return d;
+}
+
 __device__ __forceinline__ void box_muller2(uint4 w, const uint8_t *tab, float2 &z0, float2 &z1) {
   // ln(k 2^-24), k = (w >> 8) + 1
   const uint32_t ka = (w.x >> 8) + 1u, kb = (w.z >> 8) + 1u;
-  const float2 u = __fmul2_rn(make_float2(__uint2float_rn(ka), __uint2float_rn(kb)), f2(0x1p-24f));
+  const float2 u = fmul2(make_float2(__uint2float_rn(ka), __uint2float_rn(kb)), f2(0x1p-24f));
   const uint32_t ba = __float_as_uint(u.x), bb = __float_as_uint(u.y);
   const uint32_t ma = ba & 0x7FFFFFu, mb = bb & 0x7FFFFFu;
   const float4 ta = ln_row(tab, (ma + (1u << 15)) >> 16), tb = ln_row(tab, (mb + (1u << 15)) >> 16);
   const float2 m = make_float2(__uint_as_float(ma | 0x3F800000u), __uint_as_float(mb | 0x3F800000u));
   const float2 r = __ffma2_rn(m, make_float2(ta.x, tb.x), f2(-1.0f));
-  const float2 r2 = __fmul2_rn(r, r);
+  const float2 r2 = fmul2(r, r);
   float2 p = __ffma2_rn(r, f2(-0.25f), f2(ASMV_THIRD));
   p = __ffma2_rn(r, p, f2(-0.5f));
   const float2 lp = __ffma2_rn(r2, p, r);
-  const float2 ef = __fadd2_rn(make_float2(__int_as_float(0x4B400000 + (int)(ba >> 23) - 127),
+  const float2 ef = fadd2(make_float2(__int_as_float(0x4B400000 + (int)(ba >> 23) - 127),
                                            __int_as_float(0x4B400000 + (int)(bb >> 23) - 127)),
                                f2(-12582912.0f));
   const float2 hi = __ffma2_rn(ef, f2(ASMV_LN2_HI), make_float2(ta.y, tb.y));
   const float2 lo = __ffma2_rn(ef, f2(ASMV_LN2_LO), make_float2(ta.z, tb.z));
-  const float2 l = __fadd2_rn(hi, __fadd2_rn(lo, lp));
+  const float2 l = fadd2(hi, fadd2(lo, lp));
   // radius: sqrt_radius of -2 ln(u) per lane
-  const float2 x = __fmul2_rn(f2(-2.0f), l);
+  const float2 x = fmul2(f2(-2.0f), l);
   const float2 rs = make_float2(rsqrtf(x.x), rsqrtf(x.y));
-  const float2 s = __fmul2_rn(x, rs);
+  const float2 s = fmul2(x, rs);
   const float2 e = __ffma2_rn(make_float2(-s.x, -s.y), s, x);
-  const float2 y = __ffma2_rn(e, __fmul2_rn(f2(0.5f), rs), s);
+  const float2 y = __ffma2_rn(e, fmul2(f2(0.5f), rs), s);
   const float2 rho = make_float2(x.x == 0.0f ? x.x : y.x, x.y == 0.0f ? x.y : y.y);
   // sin and cos of 2 pi k 2^-24, k = w >> 8
   const uint32_t kc = w.y >> 8, kd = w.w >> 8;
   const uint32_t qa = (kc + (1u << 21)) >> 22, qb = (kd + (1u << 21)) >> 22;
   const int32_t ra = (int32_t)kc - (int32_t)(qa << 22), rb = (int32_t)kd - (int32_t)(qb << 22);
-  const float2 t = __fadd2_rn(make_float2(__int_as_float(0x40400000 + ra), __int_as_float(0x40400000 + rb)),
+  const float2 t = fadd2(make_float2(__int_as_float(0x40400000 + ra), __int_as_float(0x40400000 + rb)),
                               f2(-3.0f));
-  const float2 t2 = __fmul2_rn(t, t);
+  const float2 t2 = fmul2(t, t);
   float2 sp = __ffma2_rn(t2, f2(ASMV_S9), f2(ASMV_S7));
   sp = __ffma2_rn(t2, sp, f2(ASMV_S5));
   sp = __ffma2_rn(t2, sp, f2(ASMV_S3));
   sp = __ffma2_rn(t2, sp, f2(ASMV_S1));
-  const float2 sv = __fmul2_rn(t, sp);
+  const float2 sv = fmul2(t, sp);
   float2 cp = __ffma2_rn(t2, f2(ASMV_C10), f2(ASMV_C8));
   cp = __ffma2_rn(t2, cp, f2(ASMV_C6));
   cp = __ffma2_rn(t2, cp, f2(ASMV_C4));
@@ -189,8 +210,8 @@ __device__ __forceinline__ void box_muller2(uint4 w, const uint8_t *tab, float2 
                                 __uint_as_float(__float_as_uint(sb) ^ ((qb & 2u) << 30)));
   const float2 cs = make_float2(__uint_as_float(__float_as_uint(ca) ^ (((qa + 1u) & 2u) << 30)),
                                 __uint_as_float(__float_as_uint(cb) ^ (((qb + 1u) & 2u) << 30)));
-  z0 = __fmul2_rn(rho, cs);
-  z1 = __fmul2_rn(rho, sn);
+  z0 = fmul2(rho, cs);
+  z1 = fmul2(rho, sn);
 }
 
 // ---------------------------------------------------------------- narrow formats

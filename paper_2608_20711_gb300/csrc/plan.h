@@ -19,7 +19,25 @@
 #pragma once
 #include <stdint.h>
 
+// The debug-bounds build (compiled with ASMV_DEBUG_BOUNDS=1 into
+// libasmv_debug.so) gives every region descriptor and guard segment the
+// allocation it lies in, and the fill, compare and restore kernels check
+// each global access against it: an access outside is skipped and sets
+// kErrBounds in the launch's error word, which the call returns as
+// ASMV_EBOUNDS.  The normal build carries none of it.
+#ifndef ASMV_DEBUG_BOUNDS
+#define ASMV_DEBUG_BOUNDS 0
+#endif
+
 namespace asmv {
+
+constexpr uint32_t kErrTimeout = 1u;    // a bounded wait gave up
+constexpr uint32_t kErrBounds = 2u;     // an access fell outside its allocation (debug-bounds build)
+
+// [lo, hi) of one allocation (debug-bounds build).
+struct Span {
+  uint64_t lo, hi;
+};
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
@@ -58,6 +76,9 @@ struct FillRegion {
   float f0, f1;         // UNIFORM: lo, width; NORMAL: mean, std (fp32)
   int64_t ilo;          // INT_RANGE: lo
   uint64_t ispan;       // INT_RANGE: hi - lo
+#if ASMV_DEBUG_BOUNDS
+  Span alloc;           // the region's allocation
+#endif
 };
 
 // One region of a compare launch (32 B).  Candidate payload addresses live
@@ -68,6 +89,9 @@ struct CmpRegion {
   uint64_t tile0;
   uint32_t dtype;
   uint32_t vec;         // reference and every candidate payload 16-byte aligned
+#if ASMV_DEBUG_BOUNDS
+  Span alloc;           // the reference's allocation
+#endif
 };
 
 // A guard band segment (32 B).
@@ -79,6 +103,9 @@ struct GuardSeg {
   uint8_t canary;
   uint8_t kind;         // kSeg*
   uint8_t pad_[6];
+#if ASMV_DEBUG_BOUNDS
+  Span alloc;           // the allocation the band belongs to
+#endif
 };
 
 // fp32 screening thresholds and exact fp64 tolerances of one float dtype.
@@ -144,6 +171,9 @@ struct FillParams {
   // Philox key of each of the 10 rounds: (seed lo, seed hi) advanced by the
   // Weyl increments, precomputed on the host (kernel-parameter operands)
   uint32_t key0[10], key1[10];
+#if ASMV_DEBUG_BOUNDS
+  uint32_t *err;               // kErrBounds
+#endif
 };
 
 struct CmpParams {
@@ -152,7 +182,7 @@ struct CmpParams {
   const GuardSeg *segs;
   StatsDev *stats;             // [K][nregions] (this launch's candidates)
   StatsDev *seg_stats;         // guard segments index from here
-  uint32_t *err;               // set non-zero when a bounded wait expires
+  uint32_t *err;               // kErrTimeout when a bounded wait expires (kErrBounds)
   uint64_t ntiles;
   uint32_t nregions;
   uint32_t nsegs;
@@ -161,6 +191,9 @@ struct CmpParams {
   uint32_t wait_rounds;        // bound of the producer's wait for a free stage (tries)
   uint32_t nstages;            // pipeline depth of this launch: 2, 3 or 4 (compare_stages)
   TolF tol[kNDtypes];
+#if ASMV_DEBUG_BOUNDS
+  const Span *cand_allocs;     // [K][nregions] the candidates' allocations
+#endif
 };
 
 // The Eq. 1 sums (eqsum.cu).  Each sum of a region is kept as kEqDigits
@@ -197,6 +230,9 @@ struct CopyRegion {
   uint64_t dst, src, bytes, tile0;
   uint32_t vec;         // src and dst both 16-byte aligned
   uint32_t pad_[3];
+#if ASMV_DEBUG_BOUNDS
+  Span dst_alloc, src_alloc;   // the allocations written and read
+#endif
 };
 
 struct CopyParams {
@@ -205,6 +241,9 @@ struct CopyParams {
   uint64_t ntiles;             // tiles of kTileBytes
   uint32_t nregions;
   uint32_t nsegs;
+#if ASMV_DEBUG_BOUNDS
+  uint32_t *err;               // kErrBounds
+#endif
 };
 
 // Launchers (defined in fill.cu / compare.cu / eqsum.cu / copy.cu).  Return a cudaError_t.

@@ -171,3 +171,22 @@ def test_candidate_tables_must_match_the_reference_length():
         ctx.compare_eq(ref, [short], {"f32": (0.0, 0.0)})
     with pytest.raises(ValueError):
         ctx.compare_eq_digits(ref, [ref + ref], {"f32": (0.0, 0.0)})
+
+
+def test_debug_bounds_build_exports_the_same_calls():
+    """libasmv_debug.so (the same sources with device bounds checks) exports
+    every declared call and says which build it is; the widening hook exists
+    only there."""
+    from paper_2608_20711_gb300 import build
+    path = build.build(debug_bounds=True)
+    D = ctypes.CDLL(path)
+    for name in _declared_functions():
+        assert hasattr(D, name), name
+    L = _lib()
+    assert D.asmv_debug_bounds() == 1
+    assert L.asmv_debug_bounds() == 0
+    D.asmv_ctx_debug_widen.argtypes = [ctypes.c_void_p, ctypes.c_uint64]
+    assert D.asmv_ctx_debug_widen(None, 0) == asmv.EINVAL
+    assert L.asmv_ctx_debug_widen(None, 0) == asmv.EINVAL
+    D.asmv_strerror.restype = ctypes.c_char_p
+    assert b"allocation" in D.asmv_strerror(asmv.EBOUNDS)

@@ -45,6 +45,10 @@ FILL_CASES = [
     ("i8", "int_range", -100, 100), ("u8", "int_range", 0, 256), ("i8", "raw", 0, 0),
     ("u8", "raw", 0, 0), ("f32", "raw", 0, 0), ("f16", "raw", 0, 0), ("i32", "raw", 0, 0),
     ("f32", "none", 0, 0),
+    # widths and scales whose products are inexact: the multiply and the add round separately
+    ("f32", "uniform", -2.0, 3.0), ("f32", "normal", 0.3, 1.7), ("f64", "uniform", -2.0, 3.0),
+    ("f64", "normal", 0.3, 1.7), ("f16", "uniform", -2.0, 3.0), ("bf16", "normal", 0.3, 1.7),
+    ("f8e4m3", "normal", 0.3, 1.7),
 ]
 
 
