@@ -244,7 +244,9 @@ template <uint32_t DT> __device__ __forceinline__ constexpr bool is_int_dt() {
 // their candidate, as copies, and re-examined element by element,
 // lane-parallel, once the queue is half full after a row and when the
 // warp's run over a region ends, instead of diverging inside the screen.
-constexpr uint32_t kQueue = 32;           // chunk entries per warp
+// 24 entries per warp leave room for three stages of the 8-candidate launch
+// in the 227 KiB a CTA may take (with 32 it gets two: 5262 against 5772 GB/s).
+constexpr uint32_t kQueue = 24;           // chunk entries per warp
 
 struct QEntry {
   uint4 R, C;                             // the raw 16-byte chunks
@@ -952,10 +954,10 @@ uint32_t compare_tile_bytes(uint32_t K) {
   return K <= 1 ? 15360u : 7680u;
 }
 
-// The deepest pipeline (4, 3, else 2 stages) within kCmpSmemBudget of shared
-// memory.  The budget stays below the 227 KiB a CTA may take: the rest of
-// the SM's 256 KiB is L1, which holds the checking warps' spilled registers.
-constexpr size_t kCmpSmemBudget = 192 * 1024;
+// The deepest pipeline (4, 3, else 2 stages) within the 227 KiB of shared
+// memory a CTA may take (the checking loop spills nothing, so L1 needs
+// little of the SM's 256 KiB).
+constexpr size_t kCmpSmemBudget = kMaxSmemPerCta;
 uint32_t compare_stages(uint32_t K, uint32_t tile_bytes) {
   for (uint32_t n = 4; n > 2; --n)
     if (compare_smem_bytes(K, tile_bytes, n) <= kCmpSmemBudget) return n;
