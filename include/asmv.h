@@ -442,6 +442,13 @@ uint64_t asmv_ctx_launches(const asmv_ctx *ctx);
 #define ASMV_WAIT_ROUNDS 20000u
 int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds);
 
+/* Bound the SMs that the launches of ctx may occupy: every later call sizes
+ * its persistent grid as if the device had `sms` SMs (0, or a value at or
+ * above the device's count, restores all of them), which leaves the other
+ * SMs to work on other streams.  Results do not depend on the bound.
+ * ASMV_EINVAL for a null ctx or a negative count. */
+int asmv_ctx_set_sm_limit(asmv_ctx *ctx, int sms);
+
 /* The debug-bounds build.  libasmv_debug.so is this library compiled with
  * device bounds checks (ASMV_DEBUG_BOUNDS=1): every region descriptor and
  * guard segment carries the allocation it lies in, and every global load

@@ -98,7 +98,7 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
                  "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds",
                  "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base",
-                 "asmv_debug_bounds", "asmv_ctx_debug_widen")
+                 "asmv_debug_bounds", "asmv_ctx_debug_widen", "asmv_ctx_set_sm_limit")
 EQ_DIGITS = 20                           # signed 64-bit digits per exact Eq. 1 sum
 EQ64_DIGITS = 136                        # ... when the region table holds a binary64 region
 NOALLOC_SCRATCH_BYTES = 1 << 20
@@ -141,6 +141,7 @@ def lib():
         L.asmv_ctx_launches.restype = ctypes.c_uint64
         L.asmv_ctx_set_wait_rounds.argtypes = [vp, ctypes.c_uint32]
         L.asmv_debug_bounds.argtypes = []
+        L.asmv_ctx_set_sm_limit.argtypes = [vp, ctypes.c_int]
         L.asmv_ctx_debug_widen.argtypes = [vp, ctypes.c_uint64]
         L.asmv_strerror.argtypes = [ctypes.c_int]
         L.asmv_strerror.restype = ctypes.c_char_p
@@ -332,6 +333,11 @@ class Context:
     @property
     def launches(self) -> int:
         return int(self._lib.asmv_ctx_launches(self._h))
+
+    def set_sm_limit(self, sms: int = 0):
+        """asmv_ctx_set_sm_limit: later launches of this context size their
+        grids for at most `sms` SMs (0: all), leaving the rest to other work."""
+        self._check(self._lib.asmv_ctx_set_sm_limit(self._h, int(sms)))
 
     def debug_widen(self, nbytes: int):
         """Test hook of the debug-bounds build (asmv_ctx_debug_widen): later

@@ -233,6 +233,7 @@ struct asmv_ctx {
   uint32_t wait_rounds = kWaitRounds;
   AddrRangeFn addr_range = nullptr;
   uint64_t debug_widen = 0;       // debug-bounds build: bytes added to each fill's loop bound
+  int sm_limit = 0;               // SMs a launch may occupy (0: all of them)
 };
 
 namespace {
@@ -360,8 +361,14 @@ int debug_finish(asmv_ctx *ctx, size_t err_off, size_t img_bytes, cudaStream_t s
 }
 #endif
 
+// The SMs a launch of ctx may occupy: all of the device's, or the limit
+// set with asmv_ctx_set_sm_limit.
+uint64_t sms_of(const asmv_ctx *ctx) {
+  return (uint64_t)((ctx->sm_limit > 0 && ctx->sm_limit < ctx->sms) ? ctx->sm_limit : ctx->sms);
+}
+
 int grid_for(asmv_ctx *ctx, uint64_t ntiles, size_t nsegs, int ctas_per_sm) {
-  const uint64_t cap = (uint64_t)ctx->sms * (uint64_t)ctas_per_sm;
+  const uint64_t cap = sms_of(ctx) * (uint64_t)ctas_per_sm;
   uint64_t g = std::max<uint64_t>(ntiles, (nsegs + kWarps - 1) / kWarps);
   g = std::min<uint64_t>(g, cap);
   return (int)std::max<uint64_t>(g, 1);
@@ -594,6 +601,12 @@ int asmv_ctx_set_wait_rounds(asmv_ctx *ctx, uint32_t rounds) {
   return ASMV_OK;
 }
 
+int asmv_ctx_set_sm_limit(asmv_ctx *ctx, int sms) {
+  if (ctx == nullptr || sms < 0) return ASMV_EINVAL;
+  ctx->sm_limit = sms;
+  return ASMV_OK;
+}
+
 int asmv_debug_bounds(void) { return ASMV_DEBUG_BOUNDS; }
 
 int asmv_ctx_debug_widen(asmv_ctx *ctx, uint64_t bytes) {
@@ -795,7 +808,7 @@ static int run_compare(asmv_ctx *ctx, const asmv_region *ref, const asmv_region 
     // one CTA per SM: the shared-memory pipeline sizes itself to the SM
     const uint64_t segs_per_cta = kConsumerWarps + 1;
     const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(
-        std::max<uint64_t>(p.ntiles, (p.nsegs + segs_per_cta - 1) / segs_per_cta), (uint64_t)ctx->sms));
+        std::max<uint64_t>(p.ntiles, (p.nsegs + segs_per_cta - 1) / segs_per_cta), sms_of(ctx)));
     if ((e = (cudaError_t)launch_compare(p, grid, s)) != cudaSuccess) return fail_cuda(ctx, e);
     ctx->launches += 1;
   }
@@ -947,7 +960,7 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   p.ntiles = tile;
   p.nregions = (uint32_t)n;
   p.nslots = (uint32_t)nslots;
-  const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tile, (uint64_t)ctx->sms * ctx->eq_ctas));
+  const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(tile, sms_of(ctx) * ctx->eq_ctas));
   Eq64Params p64;
   std::memset(&p64, 0, sizeof p64);
   p64.regions = (const CmpRegion *)(dev + o_regs64);
@@ -956,7 +969,7 @@ static int run_eq(asmv_ctx *ctx, const asmv_region *ref, const asmv_region *cons
   p64.nregions = (uint32_t)n64;
   p64.nslots = (uint32_t)nslots;
   const int grid64 =
-      (int)std::max<uint64_t>(1, std::min<uint64_t>(tile64, (uint64_t)ctx->sms * ctx->eq64_ctas));
+      (int)std::max<uint64_t>(1, std::min<uint64_t>(tile64, sms_of(ctx) * ctx->eq64_ctas));
   if (ctx->timing && (e = cudaEventRecord(ctx->t0, s)) != cudaSuccess) return fail_cuda(ctx, e);
   for (size_t g = 0; g * kMaxCands < k; ++g) {
     p.K = p64.K = (uint32_t)std::min<size_t>(kMaxCands, k - g * kMaxCands);

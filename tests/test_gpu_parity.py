@@ -371,3 +371,30 @@ def test_radius_sqrt_matches_ieee_on_its_whole_domain(tmp_path):
     out = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert out.returncode == 0, out.stdout + out.stderr
     assert "differing 0 " in out.stdout
+
+
+def test_sm_limit_changes_no_result(ctx, oracle):
+    """A context whose launches are bounded to a few SMs fills the same bytes
+    and finds the same statistics (the grids are persistent, their size only
+    spreads the tiles differently)."""
+    regs = _cmp_table(51, n_regions=6)
+    size = _place(regs)
+    ref = oracle_fill_arena(oracle, regs, size, 51)
+    cand = _perturb_host(ref, regs, 52, dense=True)
+    dref, dcand = to_device(ref), to_device(cand)
+    rr = asmv.regions_in_arena(regs, dref.data_ptr())
+    cr = asmv.regions_in_arena(regs, dcand.data_ptr())
+    full = ctx.compare(rr, cr, TOL)
+    dev = device_arena(size, 0x3C)
+    try:
+        ctx.set_sm_limit(5)
+        small = ctx.compare(rr, cr, TOL)
+        ctx.fill(asmv.regions_in_arena(regs, dev.data_ptr()), seed=51)
+    finally:
+        ctx.set_sm_limit(0)
+    got = to_host(dev)
+    want = oracle_fill_arena(oracle, regs, size, 51, base=np.full(size, 0x3C, np.uint8))
+    assert np.array_equal(got, want)
+    for r, a, b in zip(regs, full, small):
+        assert_stats_equal(b, a, r.name)
+        assert_stats_equal(a, oracle_region_stats(oracle, ref, r, cand, r, TOL), r.name)
