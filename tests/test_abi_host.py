@@ -18,9 +18,8 @@ HEADER = os.path.join(ROOT, "include", "asmv.h")
 
 
 def _lib():
-    if not os.path.exists(asmv.LIB_PATH):
-        from paper_2608_20711_gb300 import build
-        build.build()
+    from paper_2608_20711_gb300 import build
+    build.build()                      # rebuilds only when a source is newer than the library
     return asmv.lib()
 
 
