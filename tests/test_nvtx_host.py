@@ -68,10 +68,8 @@ def probe(tmp_path_factory):
 
 
 def test_every_launching_call_opens_and_closes_one_range(probe):
-    from paper_2608_20711_gb300 import asmv
-    if not os.path.exists(asmv.LIB_PATH):
-        from paper_2608_20711_gb300 import build
-        build.build()
+    from paper_2608_20711_gb300 import build
+    build.build()                      # rebuilds only when a source is newer than the library
     env = dict(os.environ, NVTX_INJECTION64_PATH=probe)
     r = subprocess.run([sys.executable, "-c", CHILD, ROOT, probe], env=env, capture_output=True, text=True,
                        timeout=120)
