@@ -13,11 +13,11 @@
 // payloads are written with 128-bit stores; unaligned payloads and the
 // short last chunk with byte stores.
 //
-// Roofline: HBM writes of payload + guard bytes.  Philox costs 20 wide
-// multiplies per block on the FMA-heavy pipe, so a RAW fill is co-limited by
-// the block rate; NORMAL adds its transform, which makes the fill
-// issue-bound for every NORMAL format.  Each thread computes two chunks at a
-// time so that the two Philox chains overlap.
+// Roofline: HBM writes of payload + guard bytes.  Philox costs 18 wide
+// multiplies per block on the FMA-heavy pipe (20, less two formed once per
+// tile), so a RAW fill is co-limited by the block rate; NORMAL adds its
+// transform, which makes the fill issue-bound for every NORMAL format.  Each
+// thread computes two chunks at a time so that the two Philox chains overlap.
 #include "fill_math.cuh"
 #include "ln_table.h"
 
@@ -77,8 +77,17 @@ struct Keys {
 #endif
 };
 
-__device__ __forceinline__ uint4 payload_block(const Keys &K, uint32_t region_id, uint64_t b) {
-  return philox10_keyed(make_uint4((uint32_t)b, (uint32_t)(b >> 32), region_id, 0u), K.k0, K.k1);
+__device__ __forceinline__ uint4 payload_block(const Keys &K, const PhiloxPre &Q, uint64_t b) {
+  return philox10_pre((uint32_t)b, Q, K.k0, K.k1);
+}
+// The first Philox block of chunk c, for the blocks per chunk (1/2, 1, 2 or 4)
+// that make_chunk takes.
+static_assert((kFillTileChunks & (kFillTileChunks - 1)) == 0, "a tile's Philox blocks share the high word");
+template <uint32_t DIST, uint32_t DT>
+__device__ __forceinline__ uint64_t first_block(uint64_t c) {
+  if (DIST == kRaw) return c;
+  if (DIST == kIntRange) return DT == kI64 ? c >> 1 : DT == kI16 ? 2 * c : DT == kI32 ? c : 4 * c;
+  return DT == kF64 ? c >> 1 : c;
 }
 
 // Four fp32 values of one block (fp32 formats), per float distribution.
@@ -100,11 +109,11 @@ __device__ __forceinline__ uint32_t pack_fp8(uint32_t DT, const float v[4]) {
 
 // The 16 bytes of chunk c.
 template <uint32_t DIST, uint32_t DT>
-__device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, uint64_t c) {
-  if (DIST == kRaw) return payload_block(K, r.region_id, c);
+__device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, const PhiloxPre &Q, uint64_t c) {
+  if (DIST == kRaw) return payload_block(K, Q, c);
   if (DIST == kIntRange) {
     if (DT == kI64) {                           // 2 elements: words 2(c mod 2), +1 of block c/2
-      const uint4 w = payload_block(K, r.region_id, c >> 1);
+      const uint4 w = payload_block(K, Q, c >> 1);
       const uint32_t wa = (c & 1) ? w.z : w.x, wb = (c & 1) ? w.w : w.y;
       const int64_t a = r.ilo + (int64_t)(((uint64_t)wa * r.ispan) >> 32);
       const int64_t b = r.ilo + (int64_t)(((uint64_t)wb * r.ispan) >> 32);
@@ -115,21 +124,21 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
       uint32_t out[4];
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
-        const uint4 w = payload_block(K, r.region_id, 2 * c + q);
+        const uint4 w = payload_block(K, Q, 2 * c + q);
         out[2 * q] = (int_of(w.x, r.ilo, r.ispan) & 0xFFFFu) | (int_of(w.y, r.ilo, r.ispan) << 16);
         out[2 * q + 1] = (int_of(w.z, r.ilo, r.ispan) & 0xFFFFu) | (int_of(w.w, r.ilo, r.ispan) << 16);
       }
       return make_uint4(out[0], out[1], out[2], out[3]);
     }
     if (DT == kI32) {
-      const uint4 w = payload_block(K, r.region_id, c);
+      const uint4 w = payload_block(K, Q, c);
       return make_uint4(int_of(w.x, r.ilo, r.ispan), int_of(w.y, r.ilo, r.ispan),
                         int_of(w.z, r.ilo, r.ispan), int_of(w.w, r.ilo, r.ispan));
     } else {                                    // 8-bit: 16 elements, blocks 4c..4c+3
       uint32_t out[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const uint4 w = payload_block(K, r.region_id, 4 * c + q);
+        const uint4 w = payload_block(K, Q, 4 * c + q);
         out[q] = (int_of(w.x, r.ilo, r.ispan) & 0xFFu) | ((int_of(w.y, r.ilo, r.ispan) & 0xFFu) << 8) |
                  ((int_of(w.z, r.ilo, r.ispan) & 0xFFu) << 16) | (int_of(w.w, r.ilo, r.ispan) << 24);
       }
@@ -138,7 +147,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
   }
   // UNIFORM / NORMAL on float dtypes
   if (DT == kF64) {                             // 2 elements: words 2(c mod 2), +1 of block c/2
-    const uint4 w = payload_block(K, r.region_id, c >> 1);
+    const uint4 w = payload_block(K, Q, c >> 1);
     float v0, v1;
     if (DIST == kNormal) {
       float z0, z1;
@@ -156,11 +165,11 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
   }
   if (DT == kF32) {
     float v[4];
-    float4_of<DIST>(payload_block(K, r.region_id, c), r, K, v);
+    float4_of<DIST>(payload_block(K, Q, c), r, K, v);
     return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
                       __float_as_uint(v[3]));
   }
-  const uint4 w = payload_block(K, r.region_id, c);   // the narrow formats: block c
+  const uint4 w = payload_block(K, Q, c);       // the narrow formats: block c
   const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
   uint32_t out[4];
   if (DT == kBF16 || DT == kF16) {              // 8 elements: a pair (or two fractions) per word
@@ -213,13 +222,16 @@ __device__ void fill_tile(const FillRegion &r, const Keys &K, uint64_t tile_in_r
   const uint64_t nchunks = (r.bytes + 15) >> 4;
   const uint64_t full = r.bytes >> 4;
   const uint32_t nloc = (uint32_t)umin64(kFillTileChunks, nchunks - c0);
+  // A tile's blocks [first_block(c0), first_block(c0 + kFillTileChunks)) start
+  // at a multiple of their count, a power of two below 2^32: one high word.
+  const PhiloxPre Q = philox_pre(r.region_id, (uint32_t)(first_block<DIST, DT>(c0) >> 32), K.k0);
 #pragma unroll 1
   for (uint32_t i = threadIdx.x; i < nloc; i += 2 * kFillThreads) {
     const uint32_t i2 = i + kFillThreads;
     const bool two = i2 < nloc;
     const uint64_t ca = c0 + i, cb = c0 + (two ? i2 : i);
-    const uint4 va = make_chunk<DIST, DT>(r, K, ca);
-    const uint4 vb = make_chunk<DIST, DT>(r, K, cb);
+    const uint4 va = make_chunk<DIST, DT>(r, K, Q, ca);
+    const uint4 vb = make_chunk<DIST, DT>(r, K, Q, cb);
     store_chunk(r, K, ca, full, va);
     if (two) store_chunk(r, K, cb, full, vb);
   }
@@ -264,18 +276,6 @@ __device__ void fill_tile_dispatch(const FillRegion &r, const Keys &K, uint64_t 
   }
 }
 
-// The region of tile t when it lies past region ri: a binary search over
-// the regions after ri (the table's sentinel entry bounds it).
-__device__ __noinline__ uint32_t next_region(const FillRegion *regs, uint32_t n, uint32_t ri,
-                                             uint64_t t) {
-  uint32_t lo = ri + 1, hi = n;     // regs[lo].tile0 <= t < regs[hi].tile0
-  while (hi - lo > 1) {
-    const uint32_t mid = (lo + hi) >> 1;
-    if (regs[mid].tile0 <= t) lo = mid; else hi = mid;
-  }
-  return lo;
-}
-
 // Copy `entries` table entries of T into shared memory at `off`, `copies`
 // copies of each side by side.
 template <class T>
@@ -306,11 +306,23 @@ __global__ void __launch_bounds__(kFillThreads) fill_kernel(const __grid_constan
 #if ASMV_DEBUG_BOUNDS
     K.err = p.err;
 #endif
-    uint32_t ri = find_region(p.regions, p.nregions, b);
-    for (uint64_t t = b; t < p.ntiles; t += G) {
-      if (p.regions[ri + 1].tile0 <= t) ri = next_region(p.regions, p.nregions, ri, t);
-      const FillRegion r = p.regions[ri];
-      fill_tile_dispatch(r, K, t - r.tile0);
+    // The region records of the CTA's next kTileBatch tiles: one binary
+    // search per thread, all in flight together, copied to shared memory.
+    // (A search per tile, with 4096 regions, held every warp of the CTA for
+    // a dozen dependent loads each time the CTA stepped into a new region.)
+    constexpr uint32_t kTileBatch = 128;
+    __shared__ FillRegion tile_region[kTileBatch];
+    for (uint64_t t0 = b; t0 < p.ntiles; t0 += G * kTileBatch) {
+      const uint64_t tt = t0 + threadIdx.x * G;
+      __syncthreads();
+      if (threadIdx.x < kTileBatch && tt < p.ntiles)
+        tile_region[threadIdx.x] = p.regions[find_region(p.regions, p.nregions, tt)];
+      __syncthreads();
+      const uint32_t nt = (uint32_t)umin64(kTileBatch, (p.ntiles - t0 + G - 1) / G);
+      for (uint32_t j = 0; j < nt; ++j) {
+        const FillRegion r = tile_region[j];
+        fill_tile_dispatch(r, K, t0 + j * G - r.tile0);
+      }
     }
   }
   // guard bands: one warp per segment

@@ -22,10 +22,33 @@ __device__ __forceinline__ void mul_wide(uint32_t a, uint32_t m, uint32_t &hi, u
       : "=r"(hi), "=r"(lo) : "r"(a), "r"(m));
 }
 
-__device__ __forceinline__ uint4 philox10_keyed(uint4 x, const uint32_t *k0, const uint32_t *k1) {
+// The fill's counter is (b_lo, b_hi, region_id, 0) for block b of a region.
+// Two products of rounds 0 and 1 depend only on region_id and b_hi: B*region_id
+// in round 0, and A times round 0's first output word, hi(B*region_id) ^ b_hi
+// ^ k0, in round 1.  A tile computes them once (PhiloxPre), and each block
+// then costs 18 wide products instead of 20.
+struct PhiloxPre {
+  uint32_t x0, blo0, ahi1, alo1;      // round 0's words x0, x1; round 1's A*x0
+};
+__device__ __forceinline__ PhiloxPre philox_pre(uint32_t region_id, uint32_t b_hi, const uint32_t *k0) {
+  PhiloxPre q;
+  uint32_t bhi0;
+  mul_wide(region_id, 0xCD9E8D57u, bhi0, q.blo0);
+  q.x0 = bhi0 ^ b_hi ^ k0[0];
+  mul_wide(q.x0, 0xD2511F53u, q.ahi1, q.alo1);
+  return q;
+}
+// Philox4x32-10 of the counter (b_lo, b_hi, region_id, 0), b_hi and
+// region_id given through q; k0[r], k1[r] are round r's keys.
+__device__ __forceinline__ uint4 philox10_pre(uint32_t b_lo, const PhiloxPre &q, const uint32_t *k0,
+                                              const uint32_t *k1) {
+  uint32_t ahi, alo, bhi, blo;
+  mul_wide(b_lo, 0xD2511F53u, ahi, alo);                        // round 0: x3 of the counter is 0
+  uint4 x = make_uint4(q.x0, q.blo0, ahi ^ k1[0], alo);
+  mul_wide(x.z, 0xCD9E8D57u, bhi, blo);                         // round 1
+  x = make_uint4(bhi ^ x.y ^ k0[1], blo, q.ahi1 ^ x.w ^ k1[1], q.alo1);
 #pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    uint32_t ahi, alo, bhi, blo;
+  for (int r = 2; r < 10; ++r) {
     mul_wide(x.x, 0xD2511F53u, ahi, alo);
     mul_wide(x.z, 0xCD9E8D57u, bhi, blo);
     x = make_uint4(bhi ^ x.y ^ k0[r], blo, ahi ^ x.w ^ k1[r], alo);

@@ -204,3 +204,28 @@ def test_region_beyond_2_pow_32_elements(ctx, oracle):
     cand[r.payload_offset + r.payload_bytes + 4000] ^= 0xFF          # high guard, past 2^33 bytes
     import types
     _check_compare(ctx, oracle, types.SimpleNamespace(tol=W.DEFAULT_TOL), ref, cand, regions=[r])
+
+
+def test_philox_block_numbers_past_2_pow_32(ctx, oracle):
+    """One int8 INT_RANGE region of 2^34 + 4099 elements (16 GiB): its
+    chunks take four Philox blocks each, so the blocks of elements from 2^34
+    on have a high counter word of 1.  Ranges on both sides of that element
+    and the tail match the oracle byte for byte."""
+    n = (1 << 34) + 4099
+    r = W.Region("wide", "i8", n, "int_range", -100, 27, 256, 256, 0xC3, 9)
+    r.offset = 0
+    seed = 77
+    torch = torch_cuda()
+    dev = torch.zeros(r.alloc_bytes + 64, dtype=torch.uint8, device="cuda")
+    ctx.fill(asmv.regions_in_arena([r], dev.data_ptr()), seed=seed)
+    torch.cuda.synchronize()
+    for a, b in (((1 << 34) - 4096, (1 << 34) + 4096), ((1 << 33) - 777, (1 << 33) + 333), (n - 5000, n)):
+        got = dev[r.payload_offset + a:r.payload_offset + b].cpu().numpy()
+        want = np.zeros(b, np.uint8)
+        oracle.fill_payload(want, ORACLE_DTYPE[r.dtype], ORACLE_DIST[r.dist], a, b, r.region_id, r.p0, r.p1,
+                            seed)
+        np.testing.assert_array_equal(got, want[a:], err_msg="[%d, %d)" % (a, b))
+    hi = dev[r.payload_offset + r.payload_bytes:r.offset + r.alloc_bytes].cpu().numpy()
+    assert (hi == r.canary).all()
+    del dev
+    torch.cuda.empty_cache()
