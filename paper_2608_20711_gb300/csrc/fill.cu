@@ -200,17 +200,19 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
   return make_uint4(out[0], out[1], out[2], out[3]);
 }
 
-__device__ __forceinline__ void store_chunk(const FillRegion &r, const Keys &K, uint64_t c, uint64_t full,
-                                            uint4 v) {
-  const uint64_t addr = r.payload + 16 * c;
-  const uint32_t n = (uint32_t)umin64(16, r.bytes - 16 * c);
+// Chunk i of a tile whose first chunk, c0 of the payload, is at `base`: one
+// 16-byte store for the tile's chunks below nvec, byte stores for the rest
+// (the payload's short last chunk, every chunk of an unaligned payload).
+__device__ __forceinline__ void store_chunk(const FillRegion &r, const Keys &K, uint64_t base, uint64_t c0,
+                                            uint32_t i, uint32_t nvec, uint4 v) {
+  const uint64_t addr = base + 16 * i;
 #if ASMV_DEBUG_BOUNDS
-  if (!in_alloc(r.alloc, addr, n, K.err)) return;
+  if (!in_alloc(r.alloc, addr, umin64(16, r.bytes - 16 * (c0 + i)), K.err)) return;
 #else
   (void)K;
 #endif
-  if (r.vec && c < full) stg16(addr, v);
-  else store_bytes(addr, v, n);
+  if (i < nvec) stg16(addr, v);
+  else store_bytes(addr, v, (uint32_t)umin64(16, r.bytes - 16 * (c0 + i)));
 }
 
 // Thread t makes chunks t + 2 k kFillThreads and t + (2 k + 1) kFillThreads
@@ -225,15 +227,16 @@ __device__ void fill_tile(const FillRegion &r, const Keys &K, uint64_t tile_in_r
   // A tile's blocks [first_block(c0), first_block(c0 + kFillTileChunks)) start
   // at a multiple of their count, a power of two below 2^32: one high word.
   const PhiloxPre Q = philox_pre(r.region_id, (uint32_t)(first_block<DIST, DT>(c0) >> 32), K.k0);
+  const uint32_t nvec = r.vec ? (uint32_t)umin64(nloc, full > c0 ? full - c0 : 0) : 0u;
+  const uint64_t base = r.payload + 16 * c0;
 #pragma unroll 1
   for (uint32_t i = threadIdx.x; i < nloc; i += 2 * kFillThreads) {
     const uint32_t i2 = i + kFillThreads;
     const bool two = i2 < nloc;
-    const uint64_t ca = c0 + i, cb = c0 + (two ? i2 : i);
-    const uint4 va = make_chunk<DIST, DT>(r, K, Q, ca);
-    const uint4 vb = make_chunk<DIST, DT>(r, K, Q, cb);
-    store_chunk(r, K, ca, full, va);
-    if (two) store_chunk(r, K, cb, full, vb);
+    const uint4 va = make_chunk<DIST, DT>(r, K, Q, c0 + i);
+    const uint4 vb = make_chunk<DIST, DT>(r, K, Q, c0 + (two ? i2 : i));
+    store_chunk(r, K, base, c0, i, nvec, va);
+    if (two) store_chunk(r, K, base, c0, i2, nvec, vb);
   }
 }
 
