@@ -31,7 +31,7 @@ __device__ __forceinline__ float uniform_of(uint32_t w, float lo, float width) {
 
 // v = mean + sd*z for the four normals of a block, two per packed
 // instruction: v[0], v[2] from z0 of the two pairs, v[1], v[3] from z1.
-__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, const uint8_t *tab, float v[4]) {
+__device__ __forceinline__ void normal4(uint4 w, float mean, float sd, uint32_t tab, float v[4]) {
   float2 z0, z1;
   box_muller2(w, tab, z0, z1);
   // multiply, then add, each rounded: scalar _rn operations, which are never
@@ -64,11 +64,11 @@ __device__ __forceinline__ uint32_t int_of(uint32_t w, int64_t lo, uint64_t span
   return (uint32_t)(lo + (int64_t)(((uint64_t)w * span) >> 32));
 }
 
-// Round keys of a launch and this lane's copies of the shared-memory tables.
+// Round keys of a launch and the shared-memory addresses of this lane's
+// copies of the tables.
 struct Keys {
   const uint32_t *k0, *k1;
-  const uint8_t *sm;
-  const uint8_t *ln;        // ln reduction row 0 (fp32 / binary64 NORMAL)
+  uint32_t ln;              // ln reduction row 0 (fp32 / binary64 NORMAL)
   uint32_t offT;            // angle table entry 0
   uint32_t offR16;          // 16-bit radius chord "entry 1776" (the bias of F' >> 19)
   uint32_t offR8;           // 8-bit radius entry 0
@@ -177,7 +177,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     for (int q = 0; q < 4; ++q) {
       float a, b;
       if (DIST == kNormal) {
-        normal16_pair(ww[q], K.sm, K.offR16, K.offT, r.f0, r.f1, a, b);
+        normal16_pair(ww[q], K.offR16, K.offT, r.f0, r.f1, a, b);
       } else {
         a = uniform_frac(ww[q] & 0xFFFFu, 0x1p-16f, r.f0, r.f1);
         b = uniform_frac(ww[q] >> 16, 0x1p-16f, r.f0, r.f1);
@@ -189,7 +189,7 @@ __device__ __forceinline__ uint4 make_chunk(const FillRegion &r, const Keys &K, 
     for (int q = 0; q < 4; ++q) {
       float v[4];
       if (DIST == kNormal) {
-        normal8_word(ww[q], K.sm, K.offR8, K.offT, r.f0, r.f1, v);
+        normal8_word(ww[q], K.offR8, K.offT, r.f0, r.f1, v);
       } else {
 #pragma unroll
         for (int e = 0; e < 4; ++e) v[e] = uniform_frac((ww[q] >> (8 * e)) & 0xFFu, 0x1p-8f, r.f0, r.f1);
@@ -302,10 +302,11 @@ __global__ void __launch_bounds__(kFillThreads) fill_kernel(const __grid_constan
   // so regions of very different cost per tile (NORMAL against RAW) spread
   // evenly over the SMs.
   if (b < p.ntiles) {
-    Keys K = {p.key0, p.key1, sm, sm + L.ln + 16u * (lane % kLnCopies),
-              L.angle + 8u * (lane % kAngleCopies),
-              L.rad16 + 8u * (lane % kRad16Copies) - 1776u * 8u * kRad16Copies,
-              L.rad8 + 4u * (lane % kRad8Copies)};
+    const uint32_t sm32 = (uint32_t)__cvta_generic_to_shared(sm);
+    Keys K = {p.key0, p.key1, sm32 + L.ln + 16u * (lane % kLnCopies),
+              sm32 + L.angle + 8u * (lane % kAngleCopies),
+              sm32 + L.rad16 + 8u * (lane % kRad16Copies) - 1776u * 8u * kRad16Copies,
+              sm32 + L.rad8 + 4u * (lane % kRad8Copies)};
 #if ASMV_DEBUG_BOUNDS
     K.err = p.err;
 #endif

@@ -15,7 +15,7 @@ __global__ void check(unsigned long long *bad, unsigned int *first) {
   __syncthreads();
   const unsigned int k = blockIdx.x * blockDim.x + threadIdx.x + 1u;   // 1 .. 2^24
   if (k > (1u << 24)) return;
-  const uint8_t *row0 = reinterpret_cast<const uint8_t *>(tab) + 16u * (threadIdx.x % asmv::kLnCopies);
+  const uint32_t row0 = (uint32_t)__cvta_generic_to_shared(tab) + 16u * (threadIdx.x % asmv::kLnCopies);
   const float x = __fmul_rn(-2.0f, asmv::ln_u24(k, row0));
   if (__float_as_uint(__fsqrt_rn(x)) != __float_as_uint(asmv::sqrt_radius(x))) {
     atomicAdd(bad, 1ull);

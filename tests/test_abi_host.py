@@ -189,3 +189,17 @@ def test_debug_bounds_build_exports_the_same_calls():
     assert L.asmv_ctx_debug_widen(None, 0) == asmv.EINVAL
     D.asmv_strerror.restype = ctypes.c_char_p
     assert b"allocation" in D.asmv_strerror(asmv.EBOUNDS)
+
+
+def test_gpu_test_helpers_compile(tmp_path):
+    """The CUDA helper that the GPU tests build against the fill's headers
+    still compiles for sm_103a (compile only: no GPU here)."""
+    import shutil
+    import subprocess
+    if shutil.which("nvcc") is None:
+        pytest.skip("nvcc not on PATH")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    subprocess.check_call(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17", "-c",
+                           "-I", os.path.join(root, "paper_2608_20711_gb300", "csrc"),
+                           "-o", str(tmp_path / "radius_sqrt_check.o"),
+                           os.path.join(root, "tests", "helpers", "radius_sqrt_check.cu")])
