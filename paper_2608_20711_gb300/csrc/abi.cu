@@ -626,15 +626,29 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   std::pair<uint64_t, uint64_t> last(0, 0);
   if ((rc = check_device_table(ctx, regions, n, last)) != ASMV_OK) return rc;
 
+  // The kernel's tiles follow the table, and CTA b takes tiles b, b + G, ...,
+  // so the table lists the regions grouped by the code that fills them (a
+  // RAW region is the same whatever its dtype): a CTA then runs one kind for
+  // many tiles in a row instead of switching code, and the instruction
+  // cache, almost at every tile.  No byte depends on the order: a region's
+  // stream is addressed by its id and its own chunk index.
+  std::vector<uint32_t> ord(n);
+  for (size_t i = 0; i < n; ++i) ord[i] = (uint32_t)i;
+  const auto kind = [&](uint32_t i) {
+    const asmv_region &r = regions[i];
+    return r.dist * 64u + (r.dist == ASMV_DIST_RAW ? 0u : r.dtype);
+  };
+  std::stable_sort(ord.begin(), ord.end(), [&](uint32_t a, uint32_t b) { return kind(a) < kind(b); });
   std::vector<FillRegion> fr(n + 1);
   std::vector<GuardSeg> segs;
   uint64_t tile = 0;
   uint32_t needs = 0;   // the shared-memory tables the launch's NORMAL regions use
-  for (size_t i = 0; i < n; ++i) {
+  for (size_t j = 0; j < n; ++j) {
+    const size_t i = ord[j];
     const asmv_region &r = regions[i];
     uint64_t pb, tot;
     region_extent(r, &pb, &tot);
-    FillRegion &f = fr[i];
+    FillRegion &f = fr[j];
     std::memset(&f, 0, sizeof f);
     f.payload = r.alloc + r.guard_lo;
     f.bytes = (r.dist == ASMV_DIST_NONE) ? 0 : pb;
