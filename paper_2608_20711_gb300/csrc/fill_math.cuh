@@ -286,7 +286,9 @@ __device__ __forceinline__ uint32_t bit15_mask(uint32_t w) {
 // A table entry at shared-memory address `addr`.  The explicit 32-bit
 // shared address takes one multiply-add per lookup; through a generic
 // pointer the address was formed in 64 bits (16 GiB of fp8 NORMAL: 5.59 ->
-// 5.16 ms).
+// 5.16 ms).  The asm is not volatile and declares no memory use: every
+// address depends on a chunk's Philox words, computed inside the tile loop,
+// so no load can be moved above the barrier after the tables are copied in.
 template <class T> __device__ __forceinline__ T lds(uint32_t addr);
 template <> __device__ __forceinline__ float lds<float>(uint32_t addr) {
   float v;
