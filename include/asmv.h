@@ -415,6 +415,15 @@ int asmv_va_unmap(asmv_va *va);
  * Makes no CUDA call.  Returns ASMV_OK or ASMV_EINVAL. */
 int asmv_check_regions(const asmv_region *regions, size_t n, int for_fill);
 
+/* The order in which asmv_fill lays out the table's tiles (Sec. 3.4, Tier 1:
+ * the fill itself does not depend on it): order[k] is the table index of the
+ * k-th region, the regions grouped by the code that fills them
+ * (distribution, then dtype; RAW of any dtype is one kind) and in table
+ * order within a kind.  order holds n entries, owned by the caller.  Host
+ * only, no CUDA call; returns ASMV_EINVAL for a table asmv_fill would reject
+ * (order untouched) or a null order with n > 0. */
+int asmv_fill_order(const asmv_region *regions, size_t n, uint32_t *order);
+
 /* Kernel timing: when enabled, each call records CUDA events around its
  * kernel launch on the call's stream; asmv_ctx_kernel_ms then returns the
  * device time of the last call's kernel (waiting for it to finish).

@@ -98,7 +98,8 @@ ABI_FUNCTIONS = ("asmv_ctx_create", "asmv_ctx_destroy", "asmv_fill", "asmv_guard
                  "asmv_restore", "asmv_capture", "asmv_va_granularity", "asmv_va_map",
                  "asmv_va_address", "asmv_va_size", "asmv_va_unmap", "asmv_ctx_set_wait_rounds",
                  "asmv_compare_eq_digits", "asmv_eq_from_digits", "asmv_eq_digit_base",
-                 "asmv_debug_bounds", "asmv_ctx_debug_widen", "asmv_ctx_set_sm_limit")
+                 "asmv_debug_bounds", "asmv_ctx_debug_widen", "asmv_ctx_set_sm_limit",
+                 "asmv_fill_order")
 EQ_DIGITS = 20                           # signed 64-bit digits per exact Eq. 1 sum
 EQ64_DIGITS = 136                        # ... when the region table holds a binary64 region
 NOALLOC_SCRATCH_BYTES = 1 << 20
@@ -134,6 +135,7 @@ def lib():
         L.asmv_compare.argtypes = [vp, RP, RP, sz, TP, SP, vp]
         L.asmv_compare_batched.argtypes = [vp, RP, ctypes.POINTER(RP), sz, sz, TP, SP, vp]
         L.asmv_check_regions.argtypes = [RP, sz, ctypes.c_int]
+        L.asmv_fill_order.argtypes = [RP, sz, ctypes.POINTER(ctypes.c_uint32)]
         L.asmv_ctx_set_timing.argtypes = [vp, ctypes.c_int]
         L.asmv_ctx_kernel_ms.argtypes = [vp, ctypes.POINTER(ctypes.c_float)]
         L.asmv_ctx_cuda_error.argtypes = [vp]
@@ -275,6 +277,17 @@ def check_regions(regions: Sequence, for_fill: bool = False) -> int:
     """Host-only table validation (no GPU needed); returns the status."""
     arr = region_array(regions)
     return lib().asmv_check_regions(arr, len(regions), 1 if for_fill else 0)
+
+
+def fill_order(regions: Sequence) -> List[int]:
+    """The order asmv_fill lays out the regions' tiles in (host only);
+    raises AsmvError for a table the fill would reject."""
+    arr = region_array(regions)
+    out = (ctypes.c_uint32 * max(1, len(regions)))()
+    rc = lib().asmv_fill_order(arr, len(regions), out)
+    if rc != OK:
+        raise AsmvError(rc, lib().asmv_strerror(rc).decode())
+    return [int(out[k]) for k in range(len(regions))]
 
 
 def _stream_handle(stream) -> Optional[int]:

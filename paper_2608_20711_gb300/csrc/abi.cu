@@ -519,6 +519,30 @@ int asmv_check_regions(const asmv_region *regions, size_t n, int for_fill) {
   return check_table(regions, n, for_fill != 0);
 }
 
+// The order in which asmv_fill lays out a table's tiles: the regions grouped
+// by the code that fills them (distribution, then dtype; RAW of any dtype is
+// one kind), in table order within a kind.  The kernel's CTAs take tiles
+// round robin, so a CTA then runs one kind for many tiles in a row instead of
+// switching code, and the instruction cache, almost at every tile.  No byte
+// depends on the order: a region's Philox stream is addressed by its id and
+// its own chunk index.
+static void fill_order(const asmv_region *regions, size_t n, uint32_t *ord) {
+  for (size_t i = 0; i < n; ++i) ord[i] = (uint32_t)i;
+  const auto kind = [&](uint32_t i) {
+    const asmv_region &r = regions[i];
+    return r.dist * 64u + (r.dist == ASMV_DIST_RAW ? 0u : r.dtype);
+  };
+  std::stable_sort(ord, ord + n, [&](uint32_t a, uint32_t b) { return kind(a) < kind(b); });
+}
+
+int asmv_fill_order(const asmv_region *regions, size_t n, uint32_t *order) {
+  if (n != 0 && order == nullptr) return ASMV_EINVAL;
+  const int rc = check_table(regions, n, true);
+  if (rc != ASMV_OK) return rc;
+  fill_order(regions, n, order);
+  return ASMV_OK;
+}
+
 int asmv_ctx_create(asmv_ctx **out, int device) {
   if (out == nullptr) return ASMV_EINVAL;
   *out = nullptr;
@@ -626,19 +650,8 @@ int asmv_fill(asmv_ctx *ctx, const asmv_region *regions, size_t n, uint64_t seed
   std::pair<uint64_t, uint64_t> last(0, 0);
   if ((rc = check_device_table(ctx, regions, n, last)) != ASMV_OK) return rc;
 
-  // The kernel's tiles follow the table, and CTA b takes tiles b, b + G, ...,
-  // so the table lists the regions grouped by the code that fills them (a
-  // RAW region is the same whatever its dtype): a CTA then runs one kind for
-  // many tiles in a row instead of switching code, and the instruction
-  // cache, almost at every tile.  No byte depends on the order: a region's
-  // stream is addressed by its id and its own chunk index.
-  std::vector<uint32_t> ord(n);
-  for (size_t i = 0; i < n; ++i) ord[i] = (uint32_t)i;
-  const auto kind = [&](uint32_t i) {
-    const asmv_region &r = regions[i];
-    return r.dist * 64u + (r.dist == ASMV_DIST_RAW ? 0u : r.dtype);
-  };
-  std::stable_sort(ord.begin(), ord.end(), [&](uint32_t a, uint32_t b) { return kind(a) < kind(b); });
+  std::vector<uint32_t> ord(n);              // the tiles' region order (fill_order)
+  fill_order(regions, n, ord.data());
   std::vector<FillRegion> fr(n + 1);
   std::vector<GuardSeg> segs;
   uint64_t tile = 0;

@@ -74,6 +74,38 @@ def test_region_table_validation():
     assert asmv.check_regions([], for_fill=True) == asmv.OK
 
 
+def test_fill_order_groups_regions_by_kind():
+    """The tile order of asmv_fill: a permutation of the table, grouped by
+    (distribution, dtype) with RAW of any dtype one kind, table order kept
+    within a kind; rejected tables leave the output untouched."""
+    _lib()
+    rng = random.Random(9)
+    kinds = [("raw", "i8", 0, 0), ("raw", "i32", 0, 0), ("raw", "f16", 0, 0),
+             ("normal", "f16", 0.0, 1.0), ("normal", "f32", 0.0, 1.0), ("normal", "bf16", 0.0, 1.0),
+             ("uniform", "f16", -1.0, 1.0), ("int_range", "i32", 0, 100), ("none", "f32", 0, 0)]
+    regs, addr = [], 1 << 24
+    for i in range(300):
+        dist, dt, p0, p1 = rng.choice(kinds)
+        regs.append(dict(alloc=addr, n_elems=rng.randrange(0, 5000), dtype=dt, dist=dist, p0=p0, p1=p1,
+                         guard_lo=64, guard_hi=64, region_id=i))
+        addr += 64 + 4 * 5000 + 64 + 256
+    order = asmv.fill_order(regs)
+    assert sorted(order) == list(range(len(regs)))
+
+    def kind(i):
+        r = asmv.make_region(**regs[i])
+        return (r.dist, 0 if r.dist == asmv.DIST_RAW else r.dtype)
+    keys = [kind(i) for i in order]
+    assert keys == sorted(keys)
+    for k in set(keys):                  # stable: table order within a kind
+        idx = [i for i in order if kind(i) == k]
+        assert idx == sorted(idx)
+    assert kind(order[0])[0] == asmv.DIST_RAW        # RAW first, every dtype together
+    assert asmv.fill_order([]) == []
+    with pytest.raises(asmv.AsmvError):
+        asmv.fill_order([regs[0], dict(regs[0], alloc=regs[0]["alloc"] + 8)])   # overlapping
+
+
 def _exact(digits, base):
     v = sum(int(d) << (32 * k) for k, d in enumerate(digits))
     return float(Fraction(v) * Fraction(2) ** base) if base >= 0 else v / (1 << -base)
